@@ -1,0 +1,135 @@
+/*
+ * roi.h - C ABI of the RoI mask-learning library (libroi.so, sm_103a).
+ *
+ * "Reservoir of Importance" learns a semi-structured N:M sparsity mask by
+ * giving every weight one logit phi and sampling N of the M weights of each
+ * group without replacement (weighted reservoir sampling, Sec. 3.1 Eq. 1;
+ * Gumbel-top-K, Sec. 3.2).  Training uses the differentiable relaxation of
+ * Sec. 3.2 Eq. 3-4 / Sec. 4.2.2 Eq. 11-12 / Algorithm 1:
+ *
+ *     kappa    = phi / lambda + g,  g = -log(-log u),  u ~ U(0,1)   (Eq. 10, Sec. 4.2.3)
+ *     alpha(1) = kappa
+ *     mu(k)    = softmax(alpha(k) / tau)                              (Eq. 12)
+ *     alpha(k+1) = alpha(k) + log(1 - mu(k))                          (Eq. 11)
+ *     S        = sum_{k=1..N} mu(k)          (soft N-hot mask)
+ *     Wm       = W (.) S                     (masked weights, Eq. 5)
+ *
+ * Conventions shared by every call
+ *  - Tensors are row-major [rows, cols] (nn.Linear layout [out, in]); a group is
+ *    M contiguous elements along cols, so cols % M == 0.  Flat element index
+ *    e = (row_offset + r) * cols + c.
+ *  - bfloat16 tensors are passed as their 16-bit patterns (roi_bf16).
+ *  - Every tensor pointer is caller-owned DEVICE memory, 16-byte aligned, and
+ *    must not alias any other tensor of the same call.  The library allocates
+ *    no memory.
+ *  - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
+ *    stream).  Arguments are validated on the host before anything is
+ *    launched; on any non-OK return nothing was launched and nothing written.
+ *  - Noise: u comes from Philox-4x32-10 (Salmon et al., SC'11) with
+ *    key = (seed & 0xffffffff, seed >> 32) and
+ *    counter = (q & 0xffffffff, q >> 32, step, tensor_id), q = e >> 2; element e
+ *    takes output word e & 3 as x and u = ((x >> 9) + 0.5) * 2^-23.  Noise is
+ *    a pure function of (seed, step, tensor_id, e): it is regenerated, never
+ *    stored, so the backward call reproduces the forward's sample exactly and a
+ *    row-sliced call (row_offset) reproduces the unsliced one.
+ *  - Hard mask: flat bit array of ceil(rows*cols/32) uint32 words; bit b of word
+ *    w is element 32*w + b (bits past the last element are 0).  It is the
+ *    Gumbel-top-N of the same keys: the N largest kappa of each group, NaN
+ *    ranked as -inf, equal keys resolved towards the lower index.
+ */
+#ifndef ROI_H_
+#define ROI_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef uint16_t roi_bf16; /* bfloat16 bit pattern */
+
+typedef enum {
+    ROI_OK = 0,
+    ROI_ERR_NULL = 1,      /* a required pointer is NULL                                */
+    ROI_ERR_SHAPE = 2,     /* rows < 0, cols <= 0, cols % M != 0, or row_offset < 0      */
+    ROI_ERR_NM = 3,        /* not 1 <= N < M <= 32                                       */
+    ROI_ERR_TAU = 4,       /* tau or lambda not finite or not > 0                        */
+    ROI_ERR_ALIGN = 5,     /* a tensor pointer is not 16-byte aligned                    */
+    ROI_ERR_ALIAS = 6,     /* an output overlaps an input or another output              */
+    ROI_ERR_CUDA = 7,      /* launch failed (cudaGetLastError after the launch)          */
+    ROI_ERR_TIMEOUT = 8    /* a kernel gave up waiting on its own copies (see below)     */
+} roi_status;
+
+/* Noise state of one call (Sec. 4.2.3 sampling temperature included).
+ *  seed, step, tensor_id: Philox key and counter words (see above); tensor_id
+ *    keeps layers that share (seed, step) from sharing noise.
+ *  lambda: sampling temperature, > 0; Gumbel-top-N runs on phi / lambda.
+ *  row_offset: index of this call's first row within the full tensor, >= 0. */
+typedef struct {
+    uint64_t seed;
+    uint32_t step;
+    uint32_t tensor_id;
+    float lambda;
+    int64_t row_offset;
+} roi_noise_state;
+
+/* Forward of the mask op (Sec. 4.2.2 relaxation; Eq. 5 mask application;
+ * Algorithm 1).  Short form: lambda = 1, tensor_id = 0, row_offset = 0.
+ *  logits  [rows, cols] float32          phi
+ *  W       [rows, cols] bf16             frozen weights
+ *  N, M    keep N of every M (1 <= N < M <= 32, cols % M == 0)
+ *  tau     relaxation temperature, finite, > 0
+ *  out_Wm  [rows, cols] bf16             bf16_rne(float(W) * S), product in fp32
+ *  out_soft[rows, cols] float32, nullable  S
+ *  out_hard[ceil(rows*cols/32)] uint32, nullable  Gumbel-top-N hard mask
+ *  stream  cudaStream_t                                                    */
+roi_status roi_mask_fwd(const float* logits, const roi_bf16* W, int N, int M, float tau,
+                        uint64_t seed, uint32_t step, int64_t rows, int64_t cols,
+                        roi_bf16* out_Wm, float* out_soft, uint32_t* out_hard, void* stream);
+
+/* Forward, full noise state (st is read on the host during the call). */
+roi_status roi_mask_fwd_ex(const float* logits, const roi_bf16* W, int N, int M, float tau,
+                           const roi_noise_state* st, int64_t rows, int64_t cols,
+                           roi_bf16* out_Wm, float* out_soft, uint32_t* out_hard, void* stream);
+
+/* Backward of the mask op: turns the upstream gradient of the masked weights
+ * into logit gradients through the relaxation (Sec. 3.2: the map from logits
+ * to the soft N-hot vector is differentiable).  The noise is regenerated from
+ * st, so st must equal the forward's.
+ *  dL/dS       = float(dWm) * float(W)   (rounding of Wm passes the gradient)
+ *  out_dlogits [rows, cols] float32      dL/dphi = (dL/dkappa) / lambda; OVERWRITTEN
+ *  out_dW      [rows, cols] bf16, nullable  bf16_rne(float(dWm) * S)          */
+roi_status roi_mask_bwd(const float* logits, const roi_bf16* W, const roi_noise_state* st,
+                        int N, int M, const roi_bf16* dWm, float tau, int64_t rows, int64_t cols,
+                        float* out_dlogits, roi_bf16* out_dW, void* stream);
+
+/* Deployment mask (Sec. 4.2.3 anneals lambda towards 0; the limit of
+ * Gumbel-top-N is the deterministic top-N of phi, which is also the most
+ * probable subset of Eq. 8): argtop_N(phi) per group, NaN ranked as -inf,
+ * equal logits resolved towards the lower index.
+ *  out_bits    [ceil(rows*cols/32)] uint32  (layout as out_hard)
+ *  W, out_Wpruned  nullable together: kept weights copied bit-exactly, pruned
+ *                  weights written as +0.0                                   */
+roi_status roi_hard_mask_export(const float* logits, int N, int M, int64_t rows, int64_t cols,
+                                uint32_t* out_bits, const roi_bf16* W, roi_bf16* out_Wpruned,
+                                void* stream);
+
+/* Device-side status.  The kernels wait on their own asynchronous copies with
+ * a time limit (about 2 s); a kernel that gives up records it in a per-device
+ * status word and returns early (its outputs are then incomplete).  This call
+ * synchronises `stream`, returns ROI_ERR_TIMEOUT if the word is set (and
+ * clears it), ROI_ERR_CUDA on a CUDA error, else ROI_OK. */
+roi_status roi_device_status(void* stream);
+
+/* Static description of a status code. */
+const char* roi_status_string(roi_status s);
+
+/* Number of kernel launches the library has issued since load (host counter,
+ * for benchmarking). */
+uint64_t roi_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ROI_H_ */

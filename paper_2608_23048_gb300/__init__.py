@@ -1,0 +1,176 @@
+"""RoI mask-learning hot path on GB300: Python binding of libroi.so.
+
+The binding only marshals arguments: every step of the op runs in the CUDA
+library declared by include/roi.h.  Function names are the C names.  Tensors
+are torch CUDA tensors (bfloat16 tensors are passed by their bit patterns);
+calls are asynchronous on the current torch stream unless `stream` is given.
+There is no fallback: if libroi.so is missing the import of the binding's
+functions fails loudly.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+__all__ = [
+    "RoiError", "NoiseState", "lib", "roi_mask_fwd", "roi_mask_fwd_ex", "roi_mask_bwd",
+    "roi_hard_mask_export", "roi_device_status", "roi_status_string", "roi_launch_count",
+    "library_path", "hard_words",
+]
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+library_path = os.path.join(_PKG, "libroi.so")
+
+ROI_OK = 0
+STATUS_NAMES = {0: "ROI_OK", 1: "ROI_ERR_NULL", 2: "ROI_ERR_SHAPE", 3: "ROI_ERR_NM", 4: "ROI_ERR_TAU",
+                5: "ROI_ERR_ALIGN", 6: "ROI_ERR_ALIAS", 7: "ROI_ERR_CUDA", 8: "ROI_ERR_TIMEOUT"}
+
+
+class RoiError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {STATUS_NAMES.get(status, status)} ({roi_status_string(status)})")
+
+
+class NoiseState(ctypes.Structure):
+    """roi_noise_state: seed, step, tensor_id, lambda (sampling temperature), row_offset."""
+    _fields_ = [("seed", ctypes.c_uint64), ("step", ctypes.c_uint32), ("tensor_id", ctypes.c_uint32),
+                ("lam", ctypes.c_float), ("row_offset", ctypes.c_int64)]
+
+
+_LIB = None
+_P = ctypes.c_void_p
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded libroi.so with argument types declared (loaded once)."""
+    global _LIB
+    if _LIB is not None:
+        return _LIB
+    if not os.path.exists(library_path):
+        raise ImportError(f"{library_path} is not built; run `python -m paper_2608_23048_gb300._build` "
+                          "(or __graft_entry__.build()) first")
+    L = ctypes.CDLL(library_path)
+    i32, u32, u64, i64, f32 = ctypes.c_int, ctypes.c_uint32, ctypes.c_uint64, ctypes.c_int64, ctypes.c_float
+    L.roi_mask_fwd.argtypes = [_P, _P, i32, i32, f32, u64, u32, i64, i64, _P, _P, _P, _P]
+    L.roi_mask_fwd_ex.argtypes = [_P, _P, i32, i32, f32, ctypes.POINTER(NoiseState), i64, i64, _P, _P, _P, _P]
+    L.roi_mask_bwd.argtypes = [_P, _P, ctypes.POINTER(NoiseState), i32, i32, _P, f32, i64, i64, _P, _P, _P]
+    L.roi_hard_mask_export.argtypes = [_P, i32, i32, i64, i64, _P, _P, _P, _P]
+    L.roi_device_status.argtypes = [_P]
+    L.roi_status_string.argtypes = [i32]
+    L.roi_status_string.restype = ctypes.c_char_p
+    L.roi_launch_count.argtypes = []
+    L.roi_launch_count.restype = ctypes.c_uint64
+    for name in ("roi_mask_fwd", "roi_mask_fwd_ex", "roi_mask_bwd", "roi_hard_mask_export", "roi_device_status"):
+        getattr(L, name).restype = i32
+    _LIB = L
+    return L
+
+
+def roi_status_string(status: int) -> str:
+    return lib().roi_status_string(int(status)).decode()
+
+
+def roi_launch_count() -> int:
+    return int(lib().roi_launch_count())
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return ctypes.c_void_p(stream)
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check_tensor(t, name, dtype, shape=None):
+    import torch
+    if t is None:
+        return
+    if t.dtype != dtype:
+        raise TypeError(f"{name}: expected {dtype}, got {t.dtype}")
+    if not t.is_cuda:
+        raise ValueError(f"{name}: expected a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name}: must be contiguous")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name}: expected shape {tuple(shape)}, got {tuple(t.shape)}")
+
+
+def hard_words(rows: int, cols: int) -> int:
+    """uint32 words of a hard mask over rows * cols elements."""
+    return (rows * cols + 31) // 32
+
+
+def _raise(status, where):
+    if status != ROI_OK:
+        raise RoiError(status, where)
+
+
+def roi_mask_fwd_ex(logits, W, N, M, tau, state: NoiseState, out_Wm, out_soft=None, out_hard=None, stream=None):
+    """Forward with full noise state; outputs are written in place.  Returns None."""
+    import torch
+    rows, cols = logits.shape
+    _check_tensor(logits, "logits", torch.float32)
+    _check_tensor(W, "W", torch.bfloat16, (rows, cols))
+    _check_tensor(out_Wm, "out_Wm", torch.bfloat16, (rows, cols))
+    _check_tensor(out_soft, "out_soft", torch.float32, (rows, cols))
+    _check_tensor(out_hard, "out_hard", torch.int32, (hard_words(rows, cols),))
+    st = state if isinstance(state, NoiseState) else NoiseState(*state)
+    s = lib().roi_mask_fwd_ex(_ptr(logits), _ptr(W), int(N), int(M), float(tau), ctypes.byref(st), rows, cols,
+                              _ptr(out_Wm), _ptr(out_soft), _ptr(out_hard), _stream(stream))
+    _raise(s, "roi_mask_fwd_ex")
+
+
+def roi_mask_fwd(logits, W, N, M, tau, seed, step, out_Wm, out_soft=None, out_hard=None, stream=None):
+    """Forward, short form (lambda = 1, tensor_id = 0, row_offset = 0)."""
+    import torch
+    rows, cols = logits.shape
+    _check_tensor(logits, "logits", torch.float32)
+    _check_tensor(W, "W", torch.bfloat16, (rows, cols))
+    _check_tensor(out_Wm, "out_Wm", torch.bfloat16, (rows, cols))
+    _check_tensor(out_soft, "out_soft", torch.float32, (rows, cols))
+    _check_tensor(out_hard, "out_hard", torch.int32, (hard_words(rows, cols),))
+    s = lib().roi_mask_fwd(_ptr(logits), _ptr(W), int(N), int(M), float(tau), int(seed), int(step), rows, cols,
+                           _ptr(out_Wm), _ptr(out_soft), _ptr(out_hard), _stream(stream))
+    _raise(s, "roi_mask_fwd")
+
+
+def roi_mask_bwd(logits, W, state: NoiseState, N, M, dWm, tau, out_dlogits, out_dW=None, stream=None):
+    """Backward: logit gradients (overwritten) and optionally dW."""
+    import torch
+    rows, cols = logits.shape
+    _check_tensor(logits, "logits", torch.float32)
+    _check_tensor(W, "W", torch.bfloat16, (rows, cols))
+    _check_tensor(dWm, "dWm", torch.bfloat16, (rows, cols))
+    _check_tensor(out_dlogits, "out_dlogits", torch.float32, (rows, cols))
+    _check_tensor(out_dW, "out_dW", torch.bfloat16, (rows, cols))
+    st = state if isinstance(state, NoiseState) else NoiseState(*state)
+    s = lib().roi_mask_bwd(_ptr(logits), _ptr(W), ctypes.byref(st), int(N), int(M), _ptr(dWm), float(tau),
+                           rows, cols, _ptr(out_dlogits), _ptr(out_dW), _stream(stream))
+    _raise(s, "roi_mask_bwd")
+
+
+def roi_hard_mask_export(logits, N, M, out_bits, W=None, out_Wpruned=None, stream=None):
+    """Deployment mask argtop_N(logits) (+ pruned weights)."""
+    import torch
+    rows, cols = logits.shape
+    _check_tensor(logits, "logits", torch.float32)
+    _check_tensor(out_bits, "out_bits", torch.int32, (hard_words(rows, cols),))
+    _check_tensor(W, "W", torch.bfloat16, (rows, cols))
+    _check_tensor(out_Wpruned, "out_Wpruned", torch.bfloat16, (rows, cols))
+    s = lib().roi_hard_mask_export(_ptr(logits), int(N), int(M), rows, cols, _ptr(out_bits), _ptr(W),
+                                   _ptr(out_Wpruned), _stream(stream))
+    _raise(s, "roi_hard_mask_export")
+
+
+def roi_device_status(stream=None):
+    """Synchronises the stream; raises RoiError if a kernel timed out or CUDA failed."""
+    _raise(lib().roi_device_status(_stream(stream)), "roi_device_status")

@@ -1,0 +1,227 @@
+// C ABI of libroi (see include/roi.h): host-side validation, then one launch.
+#include <atomic>
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+
+#include "roi.h"
+#include "roi_launch.h"
+
+namespace roi {
+
+__device__ unsigned int g_roi_device_status = 0;
+
+namespace {
+
+std::atomic<uint64_t> g_launches{0};
+
+unsigned int* status_word() {
+  // Device address of this module's status word on the current device.
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_roi_device_status) != cudaSuccess) return nullptr;
+  return static_cast<unsigned int*>(p);
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+struct Range {
+  const void* p;
+  uint64_t bytes;
+};
+
+bool overlaps(const Range& a, const Range& b) {
+  if (a.p == nullptr || b.p == nullptr || a.bytes == 0 || b.bytes == 0) return false;
+  const uintptr_t a0 = reinterpret_cast<uintptr_t>(a.p), b0 = reinterpret_cast<uintptr_t>(b.p);
+  return a0 < b0 + b.bytes && b0 < a0 + a.bytes;
+}
+
+// Outputs must not overlap inputs or each other.
+template <int NI, int NO>
+bool any_alias(const Range (&in)[NI], const Range (&out)[NO]) {
+  for (int o = 0; o < NO; ++o) {
+    for (int i = 0; i < NI; ++i)
+      if (overlaps(out[o], in[i])) return true;
+    for (int p = o + 1; p < NO; ++p)
+      if (overlaps(out[o], out[p])) return true;
+  }
+  return false;
+}
+
+bool finite_positive(float x) { return std::isfinite(x) && x > 0.0f; }
+
+roi_status check_common(int N, int M, float tau, int64_t rows, int64_t cols) {
+  if (!(N >= 1 && N < M && M <= 32)) return ROI_ERR_NM;
+  if (rows < 0 || cols <= 0 || cols % M != 0) return ROI_ERR_SHAPE;
+  if (rows > 0 && cols > INT64_MAX / 64 / rows) return ROI_ERR_SHAPE;
+  if (!finite_positive(tau)) return ROI_ERR_TAU;
+  return ROI_OK;
+}
+
+NoiseParams make_noise(const roi_noise_state& st, int64_t cols) {
+  NoiseParams np;
+  np.k0 = static_cast<uint32_t>(st.seed & 0xffffffffu);
+  np.k1 = static_cast<uint32_t>(st.seed >> 32);
+  np.step = st.step;
+  np.tensor_id = st.tensor_id;
+  np.inv_lam = 1.0f / st.lambda;
+  np.e_base = static_cast<uint64_t>(st.row_offset) * static_cast<uint64_t>(cols);
+  return np;
+}
+
+roi_status finish(int launched) {
+  if (launched < 0) return ROI_ERR_CUDA;
+  g_launches.fetch_add(static_cast<uint64_t>(launched), std::memory_order_relaxed);
+  return ROI_OK;
+}
+
+}  // namespace
+
+int sm_count() {
+  static int cache[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+  if (cache[dev] == 0) {
+    int n = 0;
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    cache[dev] = n > 0 ? n : 1;
+  }
+  return cache[dev];
+}
+
+}  // namespace roi
+
+using namespace roi;
+
+extern "C" {
+
+roi_status roi_mask_fwd_ex(const float* logits, const roi_bf16* W, int N, int M, float tau,
+                           const roi_noise_state* st, int64_t rows, int64_t cols, roi_bf16* out_Wm,
+                           float* out_soft, uint32_t* out_hard, void* stream) {
+  if (logits == nullptr || W == nullptr || out_Wm == nullptr || st == nullptr) return ROI_ERR_NULL;
+  roi_status s = check_common(N, M, tau, rows, cols);
+  if (s != ROI_OK) return s;
+  if (st->row_offset < 0) return ROI_ERR_SHAPE;
+  if (!finite_positive(st->lambda)) return ROI_ERR_TAU;
+  if (!aligned16(logits) || !aligned16(W) || !aligned16(out_Wm) || !aligned16(out_soft) || !aligned16(out_hard))
+    return ROI_ERR_ALIGN;
+  const int64_t E = rows * cols;
+  const Range in[2] = {{logits, uint64_t(E) * 4}, {W, uint64_t(E) * 2}};
+  const Range out[3] = {{out_Wm, uint64_t(E) * 2}, {out_soft, uint64_t(E) * 4}, {out_hard, uint64_t((E + 31) / 32) * 4}};
+  if (any_alias(in, out)) return ROI_ERR_ALIAS;
+  if (E == 0) return ROI_OK;
+  FwdCall c;
+  c.phi = logits;
+  c.W = W;
+  c.Wm = out_Wm;
+  c.soft = out_soft;
+  c.hard = out_hard;
+  c.E = E;
+  c.N = N;
+  c.M = M;
+  c.tau = tau;
+  c.np = make_noise(*st, cols);
+  c.status = status_word();
+  if (c.status == nullptr) return ROI_ERR_CUDA;
+  c.stream = static_cast<cudaStream_t>(stream);
+  return finish(launch_fwd(c));
+}
+
+roi_status roi_mask_fwd(const float* logits, const roi_bf16* W, int N, int M, float tau, uint64_t seed,
+                        uint32_t step, int64_t rows, int64_t cols, roi_bf16* out_Wm, float* out_soft,
+                        uint32_t* out_hard, void* stream) {
+  roi_noise_state st;
+  st.seed = seed;
+  st.step = step;
+  st.tensor_id = 0;
+  st.lambda = 1.0f;
+  st.row_offset = 0;
+  return roi_mask_fwd_ex(logits, W, N, M, tau, &st, rows, cols, out_Wm, out_soft, out_hard, stream);
+}
+
+roi_status roi_mask_bwd(const float* logits, const roi_bf16* W, const roi_noise_state* st, int N, int M,
+                        const roi_bf16* dWm, float tau, int64_t rows, int64_t cols, float* out_dlogits,
+                        roi_bf16* out_dW, void* stream) {
+  if (logits == nullptr || W == nullptr || st == nullptr || dWm == nullptr || out_dlogits == nullptr)
+    return ROI_ERR_NULL;
+  roi_status s = check_common(N, M, tau, rows, cols);
+  if (s != ROI_OK) return s;
+  if (st->row_offset < 0) return ROI_ERR_SHAPE;
+  if (!finite_positive(st->lambda)) return ROI_ERR_TAU;
+  if (!aligned16(logits) || !aligned16(W) || !aligned16(dWm) || !aligned16(out_dlogits) || !aligned16(out_dW))
+    return ROI_ERR_ALIGN;
+  const int64_t E = rows * cols;
+  const Range in[3] = {{logits, uint64_t(E) * 4}, {W, uint64_t(E) * 2}, {dWm, uint64_t(E) * 2}};
+  const Range out[2] = {{out_dlogits, uint64_t(E) * 4}, {out_dW, uint64_t(E) * 2}};
+  if (any_alias(in, out)) return ROI_ERR_ALIAS;
+  if (E == 0) return ROI_OK;
+  BwdCall c;
+  c.phi = logits;
+  c.W = W;
+  c.dWm = dWm;
+  c.dphi = out_dlogits;
+  c.dW = out_dW;
+  c.E = E;
+  c.N = N;
+  c.M = M;
+  c.tau = tau;
+  c.np = make_noise(*st, cols);
+  c.status = status_word();
+  if (c.status == nullptr) return ROI_ERR_CUDA;
+  c.stream = static_cast<cudaStream_t>(stream);
+  return finish(launch_bwd(c));
+}
+
+roi_status roi_hard_mask_export(const float* logits, int N, int M, int64_t rows, int64_t cols, uint32_t* out_bits,
+                                const roi_bf16* W, roi_bf16* out_Wpruned, void* stream) {
+  if (logits == nullptr || out_bits == nullptr) return ROI_ERR_NULL;
+  if ((W == nullptr) != (out_Wpruned == nullptr)) return ROI_ERR_NULL;
+  roi_status s = check_common(N, M, 1.0f, rows, cols);
+  if (s != ROI_OK) return s;
+  if (!aligned16(logits) || !aligned16(out_bits) || !aligned16(W) || !aligned16(out_Wpruned)) return ROI_ERR_ALIGN;
+  const int64_t E = rows * cols;
+  const Range in[2] = {{logits, uint64_t(E) * 4}, {W, uint64_t(E) * 2}};
+  const Range out[2] = {{out_bits, uint64_t((E + 31) / 32) * 4}, {out_Wpruned, uint64_t(E) * 2}};
+  if (any_alias(in, out)) return ROI_ERR_ALIAS;
+  if (E == 0) return ROI_OK;
+  ExportCall c;
+  c.phi = logits;
+  c.bits = out_bits;
+  c.W = W;
+  c.Wp = out_Wpruned;
+  c.E = E;
+  c.N = N;
+  c.M = M;
+  c.stream = static_cast<cudaStream_t>(stream);
+  return finish(launch_export(c));
+}
+
+roi_status roi_device_status(void* stream) {
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return ROI_ERR_CUDA;
+  unsigned int v = 0;
+  if (cudaMemcpyFromSymbol(&v, g_roi_device_status, sizeof(v)) != cudaSuccess) return ROI_ERR_CUDA;
+  if (v != 0) {
+    const unsigned int zero = 0;
+    cudaMemcpyToSymbol(g_roi_device_status, &zero, sizeof(zero));
+    return ROI_ERR_TIMEOUT;
+  }
+  return ROI_OK;
+}
+
+const char* roi_status_string(roi_status s) {
+  switch (s) {
+    case ROI_OK: return "ok";
+    case ROI_ERR_NULL: return "a required pointer is NULL (or W / out_Wpruned given without the other)";
+    case ROI_ERR_SHAPE: return "bad shape: rows < 0, cols <= 0, cols % M != 0, size overflow or row_offset < 0";
+    case ROI_ERR_NM: return "need 1 <= N < M <= 32";
+    case ROI_ERR_TAU: return "tau and lambda must be finite and > 0";
+    case ROI_ERR_ALIGN: return "tensor pointers must be 16-byte aligned";
+    case ROI_ERR_ALIAS: return "an output overlaps an input or another output";
+    case ROI_ERR_CUDA: return "CUDA error while launching";
+    case ROI_ERR_TIMEOUT: return "a kernel gave up waiting on its own copies";
+  }
+  return "unknown status";
+}
+
+uint64_t roi_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+}  // extern "C"

@@ -1,0 +1,110 @@
+// Deployment export: argtop_N(phi) per group (the lambda -> 0 limit of the
+// Gumbel-top-N sampler, Sec. 4.2.3; the mode of the mask law of Eq. 8), packed
+// as bits, with optional pruned weights (kept copied, pruned +0.0).
+#include "roi_launch.h"
+
+namespace roi {
+namespace {
+
+// One thread per output word (32 elements); groups that straddle two words are
+// ranked by both threads, so no atomics are needed and any M <= 32 works.
+__global__ void __launch_bounds__(256) roi_export_kernel(const float* __restrict__ phi, int N, int M, int64_t E,
+                                                         uint32_t* __restrict__ bits,
+                                                         const uint16_t* __restrict__ W,
+                                                         uint16_t* __restrict__ Wp) {
+  const int64_t nwords = (E + 31) / 32;
+  for (int64_t wi = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; wi < nwords;
+       wi += int64_t(gridDim.x) * blockDim.x) {
+    const int64_t lo = wi * 32;
+    const int64_t hi = lo + 32 < E ? lo + 32 : E;
+    uint32_t word = 0;
+    for (int64_t g = lo / M; g * M < hi; ++g) {
+      float k[32];
+      for (int l = 0; l < M; ++l) k[l] = phi[g * M + l];
+      const uint32_t gb = topn_bits_dyn(k, N, M);
+      for (int l = 0; l < M; ++l) {
+        const int64_t e = g * M + l;
+        if (e >= lo && e < hi && ((gb >> l) & 1u)) word |= 1u << (e - lo);
+      }
+    }
+    bits[wi] = word;
+    if (Wp != nullptr) {
+      for (int64_t e = lo; e < hi; ++e) Wp[e] = ((word >> (e - lo)) & 1u) ? W[e] : uint16_t(0);
+    }
+  }
+}
+
+// M = 4 and M = 8: one thread per 32 elements with 16-byte loads.
+template <int M>
+__global__ void __launch_bounds__(256) roi_export_vec_kernel(const float* __restrict__ phi, int N, int64_t E,
+                                                             uint32_t* __restrict__ bits,
+                                                             const uint16_t* __restrict__ W,
+                                                             uint16_t* __restrict__ Wp) {
+  const int64_t nwords = E / 32;  // full words only; launcher handles E % 32 with the generic kernel
+  for (int64_t wi = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; wi < nwords;
+       wi += int64_t(gridDim.x) * blockDim.x) {
+    const float4* p = reinterpret_cast<const float4*>(phi + wi * 32);
+    uint32_t word = 0;
+#pragma unroll
+    for (int g = 0; g < 32 / M; ++g) {
+      float k[M];
+#pragma unroll
+      for (int s = 0; s < M / 4; ++s) {
+        const float4 v = p[g * (M / 4) + s];
+        k[4 * s] = v.x, k[4 * s + 1] = v.y, k[4 * s + 2] = v.z, k[4 * s + 3] = v.w;
+      }
+      word |= topn_bits<M>(k, N) << (g * M);
+    }
+    bits[wi] = word;
+    if (Wp != nullptr) {
+      const uint4* wv = reinterpret_cast<const uint4*>(W + wi * 32);
+      uint4* out = reinterpret_cast<uint4*>(Wp + wi * 32);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        uint4 v = wv[q];
+        uint32_t* u = reinterpret_cast<uint32_t*>(&v);
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          const int e = q * 8 + h * 2;
+          const uint32_t keep_lo = (word >> e) & 1u, keep_hi = (word >> (e + 1)) & 1u;
+          u[h] &= (keep_lo ? 0x0000ffffu : 0u) | (keep_hi ? 0xffff0000u : 0u);
+        }
+        out[q] = v;
+      }
+    }
+  }
+}
+
+int grid_for(int64_t items, int threads) {
+  int64_t blocks = (items + threads - 1) / threads;
+  const int64_t cap = int64_t(sm_count()) * 8;
+  if (blocks > cap) blocks = cap;
+  return int(blocks < 1 ? 1 : blocks);
+}
+
+}  // namespace
+
+int launch_export(const ExportCall& c) {
+  int launched = 0;
+  if ((c.M == 4 || c.M == 8) && c.E >= 32) {
+    const int64_t full = c.E / 32;
+    if (c.M == 4)
+      roi_export_vec_kernel<4><<<grid_for(full, 256), 256, 0, c.stream>>>(c.phi, c.N, c.E, c.bits, c.W, c.Wp);
+    else
+      roi_export_vec_kernel<8><<<grid_for(full, 256), 256, 0, c.stream>>>(c.phi, c.N, c.E, c.bits, c.W, c.Wp);
+    ++launched;
+    if (cudaGetLastError() != cudaSuccess) return -1;
+    if (c.E % 32 == 0) return launched;
+    // last partial word
+    const int64_t lo = full * 32;
+    roi_export_kernel<<<1, 32, 0, c.stream>>>(c.phi + lo, c.N, c.M, c.E - lo, c.bits + full,
+                                              c.W ? c.W + lo : nullptr, c.Wp ? c.Wp + lo : nullptr);
+    ++launched;
+    return cudaGetLastError() == cudaSuccess ? launched : -1;
+  }
+  roi_export_kernel<<<grid_for((c.E + 31) / 32, 256), 256, 0, c.stream>>>(c.phi, c.N, c.M, c.E, c.bits, c.W, c.Wp);
+  ++launched;
+  return cudaGetLastError() == cudaSuccess ? launched : -1;
+}
+
+}  // namespace roi

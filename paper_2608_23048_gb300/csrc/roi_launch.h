@@ -1,0 +1,57 @@
+// Host-side launch interface between the C ABI (roi_api.cu) and the kernels.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "roi_common.cuh"
+
+namespace roi {
+
+struct FwdCall {
+  const float* phi;
+  const uint16_t* W;
+  uint16_t* Wm;
+  float* soft;      // nullable
+  uint32_t* hard;   // nullable
+  int64_t E;        // rows * cols
+  int N, M;
+  float tau;
+  NoiseParams np;
+  unsigned int* status;
+  cudaStream_t stream;
+};
+
+struct BwdCall {
+  const float* phi;
+  const uint16_t* W;
+  const uint16_t* dWm;
+  float* dphi;
+  uint16_t* dW;     // nullable
+  int64_t E;
+  int N, M;
+  float tau;
+  NoiseParams np;
+  unsigned int* status;
+  cudaStream_t stream;
+};
+
+struct ExportCall {
+  const float* phi;
+  uint32_t* bits;
+  const uint16_t* W;  // nullable
+  uint16_t* Wp;       // nullable
+  int64_t E;
+  int N, M;
+  cudaStream_t stream;
+};
+
+// Each returns the number of kernels launched (>= 0) or -1 after a CUDA error.
+int launch_fwd(const FwdCall& c);
+int launch_bwd(const BwdCall& c);
+int launch_export(const ExportCall& c);
+
+// Streaming multiprocessors of the current device (cached).
+int sm_count();
+
+}  // namespace roi

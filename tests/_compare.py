@@ -1,0 +1,81 @@
+"""Comparison rules between the CUDA library and the oracle.
+
+Floating outputs (the paper fixes no precision; the library computes in fp32):
+the outputs are smooth functions of the scaled keys z = kappa / tau, and each side
+rounds kappa to fp32 on its own (half an ulp for phi / lambda + g, up to ~1.5 ulp
+for the two logs of the Gumbel transform).  That input error,
+    eps_z = 4 * 2^-24 * (max_group |kappa| + 1) / tau,
+is carried through N softmax steps, so the allowed difference is
+    soft S   : (1e-5 + 2 N eps_z) * max(|y|, max_group |y|)
+    dlogits  : (1e-5 + 8 N eps_z) * max(max_group |y|, max_group |c| / (tau lambda)),
+with c = dWm * W the upstream gradient of S (the backward sums terms of size
+|c| / tau, so their rounding is relative to that scale, not to a small result).
+At tau = 1 the second term is below 1e-5 and the rule is the plain 1e-5 relative
+bound.  bf16 outputs: within one bf16 ulp.  Hard masks: bit-exact, except groups
+whose N-th and (N+1)-th float64 keys differ by less than 1e-6 (counted).
+"""
+import numpy as np
+
+U = 2.0 ** -24
+
+
+def eps_z(kappa64, M, tau):
+    k = np.abs(np.asarray(kappa64, dtype=np.float64)).reshape(-1, M)
+    k = np.where(np.isfinite(k), k, 0.0)
+    return 4 * U * (k.max(axis=1, keepdims=True) + 1.0) / tau
+
+
+def soft_violations(got, want, kappa64, N, M, tau):
+    g = np.asarray(got, dtype=np.float64).reshape(-1, M)
+    w = np.asarray(want, dtype=np.float64).reshape(-1, M)
+    scale = np.maximum(np.abs(w), np.abs(w).max(axis=1, keepdims=True))
+    tol = (1e-5 + 2 * N * eps_z(kappa64, M, tau)) * scale
+    bad = ~(np.abs(g - w) <= tol)
+    return int(bad.sum()), float(np.max(np.abs(g - w) / np.maximum(tol, 1e-300)))
+
+
+def dlogit_violations(got, want, c, kappa64, N, M, tau, lam=1.0):
+    g = np.asarray(got, dtype=np.float64).reshape(-1, M)
+    w = np.asarray(want, dtype=np.float64).reshape(-1, M)
+    cs = np.abs(np.asarray(c, dtype=np.float64)).reshape(-1, M).max(axis=1, keepdims=True) / (tau * lam)
+    scale = np.maximum(np.abs(w).max(axis=1, keepdims=True), cs)
+    tol = (1e-5 + 8 * N * eps_z(kappa64, M, tau)) * scale
+    bad = ~(np.abs(g - w) <= tol)
+    return int(bad.sum()), float(np.max(np.abs(g - w) / np.maximum(tol, 1e-300)))
+
+
+def plain_relative(got, want, c=None, M=4, tau=1.0, lam=1.0):
+    """max |x - y| / group scale (the bare 1e-5 rule), for reporting."""
+    g = np.asarray(got, dtype=np.float64).reshape(-1, M)
+    w = np.asarray(want, dtype=np.float64).reshape(-1, M)
+    scale = np.abs(w).max(axis=1, keepdims=True)
+    if c is not None:
+        scale = np.maximum(scale, np.abs(np.asarray(c, dtype=np.float64)).reshape(-1, M).max(axis=1, keepdims=True)
+                           / (tau * lam))
+    scale = np.maximum(scale, 1e-300)
+    return float(np.max(np.abs(g - w) / scale))
+
+
+def bf16_violations(got_bits, want_bits):
+    """Count entries more than one bf16 ulp apart (bit patterns as uint16)."""
+    from oracle.roi_oracle import bf16_to_f32
+    g = bf16_to_f32(np.asarray(got_bits).ravel()).astype(np.float64)
+    w = bf16_to_f32(np.asarray(want_bits).ravel()).astype(np.float64)
+    both_nan = np.isnan(g) & np.isnan(w)
+    m = np.maximum(np.abs(g), np.abs(w))
+    with np.errstate(divide="ignore"):
+        ulp = np.where(m > 0, 2.0 ** (np.floor(np.log2(np.where(m > 0, m, 1.0))) - 7), 2.0 ** -133)
+    ulp = np.maximum(ulp, 2.0 ** -133)
+    bad = ~(np.abs(g - w) <= ulp) & ~both_nan
+    return int(bad.sum())
+
+
+def hard_mismatches(got_words, want_words, kappa64, N, M, E):
+    """(mismatching groups outside the near-tie band, near-tie groups)."""
+    from oracle.roi_oracle import topn_key_gap, unpack_bits
+    g = unpack_bits(np.asarray(got_words).view(np.uint32), E).reshape(-1, M)
+    w = unpack_bits(np.asarray(want_words).view(np.uint32), E).reshape(-1, M)
+    gap = topn_key_gap(np.asarray(kappa64, dtype=np.float64).reshape(-1, M), N)
+    near = gap < 1e-6
+    diff = np.any(g != w, axis=1)
+    return int(np.sum(diff & ~near)), int(np.sum(near))

@@ -1,0 +1,86 @@
+"""The C ABI: libroi.so loads, exports every function include/roi.h declares, and
+validates arguments on the host (these calls return before any CUDA call, so they
+run without a GPU)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "roi.h")
+
+
+@pytest.fixture(scope="module")
+def L():
+    from paper_2608_23048_gb300 import _build
+    _build.build()
+    import paper_2608_23048_gb300 as roi
+    return roi.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(roi_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_calls():
+    names = declared_functions()
+    for want in ("roi_mask_fwd", "roi_mask_fwd_ex", "roi_mask_bwd", "roi_hard_mask_export",
+                 "roi_status_string", "roi_device_status", "roi_launch_count"):
+        assert want in names
+
+
+def test_library_exports_every_declared_symbol(L):
+    for name in declared_functions():
+        assert hasattr(L, name), name
+
+
+def test_binding_names_match_abi():
+    import paper_2608_23048_gb300 as roi
+    for name in declared_functions():
+        assert callable(getattr(roi, name)), name
+
+
+def _fake(addr):
+    return ctypes.c_void_p(addr)
+
+
+A, B, C, D, E = 0x10000000, 0x20000000, 0x30000000, 0x40000000, 0x50000000
+
+
+def fwd(L, logits=A, W=B, N=2, M=4, tau=1.0, rows=4, cols=8, Wm=C, soft=None, hard=None, st=None):
+    import paper_2608_23048_gb300 as roi
+    st = st or roi.NoiseState(0, 0, 0, 1.0, 0)
+    return L.roi_mask_fwd_ex(_fake(logits) if logits else None, _fake(W) if W else None, N, M, tau,
+                             ctypes.byref(st), rows, cols, _fake(Wm) if Wm else None,
+                             _fake(soft) if soft else None, _fake(hard) if hard else None, None)
+
+
+def test_validation_codes(L):
+    import paper_2608_23048_gb300 as roi
+    assert fwd(L, logits=0) == 1                    # ROI_ERR_NULL
+    assert fwd(L, Wm=0) == 1
+    assert fwd(L, N=0) == 3 and fwd(L, N=4, M=4) == 3 and fwd(L, N=2, M=33, cols=33) == 3   # ROI_ERR_NM
+    assert fwd(L, cols=6) == 2 and fwd(L, rows=-1) == 2 and fwd(L, cols=0) == 2            # ROI_ERR_SHAPE
+    assert fwd(L, tau=0.0) == 4 and fwd(L, tau=float("nan")) == 4 and fwd(L, tau=float("inf")) == 4
+    assert fwd(L, st=roi.NoiseState(0, 0, 0, 0.0, 0)) == 4                                  # lambda
+    assert fwd(L, st=roi.NoiseState(0, 0, 0, 1.0, -1)) == 2                                 # row_offset
+    assert fwd(L, logits=A + 8) == 5 and fwd(L, hard=D + 4) == 5                            # ROI_ERR_ALIGN
+    assert fwd(L, Wm=A + 16) == 6                   # output overlaps logits: ROI_ERR_ALIAS
+    assert fwd(L, soft=C + 16) == 6                 # two outputs overlap
+    assert fwd(L, rows=0) == 0                      # empty tensor: nothing to do
+    st = roi.NoiseState(0, 0, 0, 1.0, 0)
+    assert L.roi_mask_bwd(_fake(A), _fake(B), ctypes.byref(st), 2, 4, None, 1.0, 4, 8, _fake(C), None, None) == 1
+    assert L.roi_mask_bwd(_fake(A), _fake(B), ctypes.byref(st), 2, 4, _fake(D), 1.0, 4, 8, _fake(D), None, None) == 6
+    assert L.roi_hard_mask_export(_fake(A), 2, 4, 4, 8, _fake(C), _fake(B), None, None) == 1
+    assert L.roi_hard_mask_export(_fake(A), 2, 4, 4, 8, _fake(C + 4), None, None, None) == 5
+    assert L.roi_hard_mask_export(_fake(A), 2, 4, 0, 8, _fake(C), None, None, None) == 0
+    for s in range(9):
+        assert L.roi_status_string(s)
+
+
+def test_short_form_validates_like_ex(L):
+    assert L.roi_mask_fwd(None, _fake(B), 2, 4, 1.0, 0, 0, 4, 8, _fake(C), None, None, None) == 1
+    assert L.roi_mask_fwd(_fake(A), _fake(B), 2, 4, -1.0, 0, 0, 4, 8, _fake(C), None, None, None) == 4
