@@ -1,0 +1,464 @@
+#!/usr/bin/env python
+"""Benchmark of the fused RoI mask forward + backward on a Qwen2.5-shaped layer set.
+
+One step = roi_mask_fwd over every tensor of the layer set (forward order), then
+roi_mask_bwd over every tensor (reverse order), with step-keyed noise (the step
+index is the Philox counter word), all on one CUDA stream.  Prints one JSON line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--set qwen2.5-7b] [--nm 2:4] [--tau 1.0]
+
+Under torchrun every rank runs its own full layer set (independent problems, no
+collective on the data path: weak scaling); rank 0 prints the max-over-ranks time.
+--impl reference times the CPU oracle (the plain statement of the method) on the
+host cores instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import workloads as WL  # noqa: E402
+
+METRIC = "fused RoI mask fwd+bwd groups/s and HBM GB/s (% of GB300 peak), 1 GPU"
+FWD_BYTES = 4 + 2 + 2 + 1 / 8     # logits, W in; Wm, hard bits out
+BWD_BYTES = 4 + 2 + 2 + 4         # logits, W, dWm in; dlogits out
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=100)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    p.add_argument("--set", default="qwen2.5-7b", choices=sorted(WL.LAYER_SETS))
+    p.add_argument("--nm", default="2:4")
+    p.add_argument("--tau", type=float, default=None)
+    p.add_argument("--e2e-steps", type=int, default=5)
+    p.add_argument("--cpu-seconds", type=float, default=12.0)
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+def config_for(args):
+    lset = WL.LAYER_SETS[args.set]
+    cfg = WL.CONFIGS[args.set]
+    N, M = map(int, args.nm.split(":"))
+    tau = args.tau if args.tau is not None else cfg.taus[0]
+    E = lset.elements
+    h, kv, i = lset.hidden, lset.kv, lset.inter
+    return {
+        "workload": (f"{args.set}-shaped layer set, {N}:{M}, tau={tau}, {lset.layers} layers x "
+                     f"{{q,o {h}x{h}; k,v {kv}x{h}; gate,up {i}x{h}; down {h}x{i}}}, "
+                     f"logits {cfg.logits}, step-keyed noise"),
+        "layer_set": args.set, "N": N, "M": M, "tau": tau, "lambda": 1.0,
+        "elements": E, "groups": E // M, "tensors": len(lset.tensors()),
+        "l2": "inputs larger than L2: every step streams the whole set (>90 GB for the 7B set)",
+    }
+
+
+# --------------------------------------------------------------------------
+# clocks during the timed region
+# --------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.idx = device_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [ln for ln in out.splitlines() if ln.strip()]
+        else:
+            self.lines = []
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx.append(float(f[1]))
+            except ValueError:
+                continue
+            for name, val in zip(names, f[4:8]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------
+# roofline denominators and counters
+# --------------------------------------------------------------------------
+def hbm_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash():
+    d = os.path.join(ROOT, "paper_2608_23048_gb300", "csrc")
+    h = hashlib.sha256()
+    for name in sorted(os.listdir(d)):
+        with open(os.path.join(d, name), "rb") as f:
+            h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel_tag: str):
+    """DRAM bytes per element of `kernel_tag` from profiles/dram_traffic.txt, if the
+    kernel sources are unchanged since that capture; else None."""
+    path = os.path.join(ROOT, "profiles", "dram_traffic.txt")
+    try:
+        lines = open(path).read().splitlines()
+    except OSError:
+        return None
+    want = kernel_source_hash()
+    for ln in lines:
+        if ln.startswith("#") or not ln.strip():
+            continue
+        kv = dict(x.split("=", 1) for x in ln.split() if "=" in x)
+        if kv.get("kernel") == kernel_tag and kv.get("sources") == want:
+            return float(kv["dram_bytes_per_element"])
+    return None
+
+
+# --------------------------------------------------------------------------
+# CPU oracle timing (cpu_baseline and --impl reference)
+# --------------------------------------------------------------------------
+def _oracle_chunk(job):
+    """Runs in a spawned worker: oracle fwd + bwd over `rows` rows of a tensor."""
+    import numpy as np
+    import workloads as W
+    from oracle import roi_oracle as O
+    rows, cols, N, M, tau, kind, seed, step, row_offset = job
+    Wt, phi, dWm = W.make_inputs(rows, cols, kind, seed)
+    ph, Wb, dWb = phi.numpy(), W.bf16_bits(Wt), W.bf16_bits(dWm)
+    t0 = time.perf_counter()
+    O.mask_fwd(ph, Wb, N, M, tau, seed, step, row_offset=row_offset)
+    O.mask_bwd(ph, Wb, dWb, N, M, tau, seed, step, row_offset=row_offset)
+    return time.perf_counter() - t0, rows * cols // M
+
+
+def oracle_pool(cores):
+    import multiprocessing as mp
+    return mp.get_context("spawn").Pool(cores)
+
+
+def time_oracle(pool, cores, cfg, cols, rows_per_job, jobs, step=0):
+    N, M, tau = cfg["N"], cfg["M"], cfg["tau"]
+    kind = WL.CONFIGS[cfg["layer_set"]].logits
+    work = [(rows_per_job, cols, N, M, tau, kind, 1000 + j, step, j * rows_per_job) for j in range(jobs)]
+    res = pool.map(_oracle_chunk, work, chunksize=1)
+    groups = sum(g for _, g in res)
+    # the jobs run side by side, one per process: the slowest bounds the wall time
+    return groups, max(t for t, _ in res)
+
+
+def calibrate_rows(pool, cores, cfg, cols, target_s, max_rows):
+    """Rows per job so that one job of the oracle takes about target_s seconds:
+    grow the job until it takes a quarter of the target, then scale linearly."""
+    rows = 4
+    time_oracle(pool, cores, cfg, cols, rows, cores)      # workers pay their imports here
+    while True:
+        _, t = time_oracle(pool, cores, cfg, cols, rows, cores)
+        if t >= target_s / 4 or rows * 4 > max_rows:
+            break
+        rows *= 4
+    return max(1, min(max_rows, int(rows * target_s / max(t, 1e-6))))
+
+
+def cpu_baseline(cfg, seconds, cores=None):
+    """Oracle (float64, as it stands) on the host cores over rows of the set's largest tensor."""
+    cores = cores or os.cpu_count() or 1
+    lset = WL.LAYER_SETS[cfg["layer_set"]]
+    rows_full, cols = lset.shape("gate")
+    pool = oracle_pool(cores)
+    try:
+        rows_per_job = calibrate_rows(pool, cores, cfg, cols, seconds, rows_full // cores)
+        g, wall = time_oracle(pool, cores, cfg, cols, rows_per_job, cores)
+    finally:
+        pool.close()
+        pool.join()
+    return {"value": g / wall, "unit": "groups/s", "cores": cores, "kind": "oracle",
+            "sample": (f"{cores} x {rows_per_job} rows of the {cfg['layer_set']} gate_proj shape "
+                       f"({rows_per_job * cores} x {cols}, {g} groups), float64 oracle fwd+bwd, "
+                       f"{wall:.1f} s wall on {cores} processes")}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    cfg = config_for(args)
+    cores = os.cpu_count() or 1
+    lset = WL.LAYER_SETS[cfg["layer_set"]]
+    _, cols = lset.shape("gate")
+    pool = oracle_pool(cores)
+    budget = 120.0  # seconds of oracle work for the whole --steps/--warmup run
+    try:
+        per_step = min(10.0, budget / max(1, args.steps + args.warmup))
+        rows_per_job = calibrate_rows(pool, cores, cfg, cols, per_step, 4096)
+        for w in range(args.warmup):
+            time_oracle(pool, cores, cfg, cols, rows_per_job, cores, step=w)
+        tot_g, tot_t = 0, 0.0
+        for s in range(args.steps):
+            g, wall = time_oracle(pool, cores, cfg, cols, rows_per_job, cores, step=args.warmup + s)
+            tot_g += g
+            tot_t += wall
+    finally:
+        pool.close()
+        pool.join()
+    value = tot_g / tot_t
+    sample = (f"each step: {cores} x {rows_per_job} rows of the gate_proj shape x {cols} "
+              f"({tot_g // max(1, args.steps)} groups), float64 oracle fwd+bwd")
+    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": "groups/s", "n_gpus": args.gpus,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_t / max(1, args.steps),
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+           "data": "synthetic", "config": cfg,
+           "cpu_baseline": {"value": value, "unit": "groups/s", "cores": cores, "kind": "oracle", "sample": sample},
+           "e2e": {"value": value, "unit": "groups/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+# --------------------------------------------------------------------------
+# our arm
+# --------------------------------------------------------------------------
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    cfg = config_for(args)
+    N, M, tau = cfg["N"], cfg["M"], cfg["tau"]
+
+    # the oracle pool is spawned before the first CUDA call
+    base = None
+    if rank == 0 and not args.no_cpu_baseline:
+        base = cpu_baseline(cfg, args.cpu_seconds)
+
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    from paper_2608_23048_gb300 import _build
+    if rank == 0:
+        _build.build()
+    if world > 1:
+        dist.barrier()
+    import paper_2608_23048_gb300 as roi
+    roi.lib()
+
+    lset = WL.LAYER_SETS[args.set]
+    kind = WL.CONFIGS[args.set].logits
+    tensors = []
+    for layer, p, rows, cols in lset.tensors():
+        W, phi, dWm = WL.make_inputs(rows, cols, kind, WL.tensor_seed(layer, p) + 7919 * rank, device=dev)
+        tensors.append({
+            "id": layer * len(WL.PROJS) + p, "rows": rows, "cols": cols, "phi": phi, "W": W, "dWm": dWm,
+            "Wm": torch.empty_like(W), "dphi": torch.empty_like(phi),
+            "hard": torch.empty(roi.hard_words(rows, cols), dtype=torch.int32, device=dev)})
+    torch.cuda.synchronize()
+    stream = torch.cuda.Stream(device=dev)
+    states = {t["id"]: roi.NoiseState(0, 0, t["id"], 1.0, 0) for t in tensors}
+
+    def step(s, ev=None):
+        for t in tensors:
+            st = states[t["id"]]
+            st.step = s
+            if ev is not None:
+                ev[0].append(torch.cuda.Event(enable_timing=True))
+                ev[0][-1].record(stream)
+            roi.roi_mask_fwd_ex(t["phi"], t["W"], N, M, tau, st, t["Wm"], None, t["hard"], stream=stream)
+            if ev is not None:
+                ev[1].append(torch.cuda.Event(enable_timing=True))
+                ev[1][-1].record(stream)
+        for t in reversed(tensors):
+            st = states[t["id"]]
+            if ev is not None:
+                ev[2].append(torch.cuda.Event(enable_timing=True))
+                ev[2][-1].record(stream)
+            roi.roi_mask_bwd(t["phi"], t["W"], st, N, M, t["dWm"], tau, t["dphi"], None, stream=stream)
+            if ev is not None:
+                ev[3].append(torch.cuda.Event(enable_timing=True))
+                ev[3][-1].record(stream)
+
+    with torch.cuda.stream(stream):
+        for w in range(args.warmup):
+            step(w)
+    torch.cuda.synchronize()
+    roi.roi_device_status(stream)
+
+    # timed region: K steps, per-launch events for the per-kernel roofline
+    ev = ([], [], [], [])
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    launches0 = roi.roi_launch_count()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clocks:
+        start.record(stream)
+        for s in range(args.steps):
+            step(args.warmup + s, ev)
+        end.record(stream)
+        torch.cuda.synchronize()
+    launches = roi.roi_launch_count() - launches0
+    if world > 1:
+        dist.barrier()
+    roi.roi_device_status(stream)
+    elapsed = start.elapsed_time(end) / 1e3
+    fwd_t = sum(a.elapsed_time(b) for a, b in zip(ev[0], ev[1])) / 1e3
+    bwd_t = sum(a.elapsed_time(b) for a, b in zip(ev[2], ev[3])) / 1e3
+    if world > 1:
+        tt = torch.tensor([elapsed], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        elapsed = float(tt.item())
+
+    E = lset.elements
+    groups_all = world * (E // M) * args.steps
+    value = groups_all / elapsed
+    step_gbs = world * E * (FWD_BYTES + BWD_BYTES) * args.steps / elapsed / 1e9
+    peak, peak_kind = hbm_peak()
+    fwd_gbs = E * FWD_BYTES * args.steps / fwd_t / 1e9
+    bwd_gbs = E * BWD_BYTES * args.steps / bwd_t / 1e9
+    dom = "bwd" if bwd_t >= fwd_t else "fwd"
+    tag = f"roi_{dom}_kernel<{N},{M},{'tau1' if tau == 1.0 else 'tau'}>"
+    traffic = recorded_traffic(tag)
+    per_elem = BWD_BYTES if dom == "bwd" else FWD_BYTES
+    achieved = bwd_gbs if dom == "bwd" else fwd_gbs
+    launches_per_kernel = len(tensors)
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4),
+                "traffic": (None if traffic is None else traffic * E / launches_per_kernel),
+                "kernel": tag, "peak_kind": peak_kind,
+                "algorithmic_bytes_per_element": per_elem,
+                "units_per_launch": f"{E / launches_per_kernel:.0f} elements (mean over the {launches_per_kernel} tensors)",
+                "fwd_gbs": round(fwd_gbs, 1), "bwd_gbs": round(bwd_gbs, 1),
+                "fwd_ms_per_step": round(1e3 * fwd_t / args.steps, 3),
+                "bwd_ms_per_step": round(1e3 * bwd_t / args.steps, 3),
+                "step_gbs": round(step_gbs / world, 1), "step_frac": round(step_gbs / world / peak, 4)}
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, roi, tensors, lset, N, M, tau, dev, world)
+
+    if rank == 0:
+        out = {"metric": METRIC, "value": value, "unit": "groups/s", "n_gpus": world, "steps": args.steps,
+               "warmup": args.warmup, "ms_per_step": 1e3 * elapsed / args.steps, "higher_is_better": True,
+               "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": cfg,
+               "hbm_gbs": round(step_gbs, 1), "hbm_frac": round(step_gbs / world / peak, 4),
+               "roofline": roofline, "cpu_baseline": base, "e2e": e2e,
+               "gpu_launches": int(launches), "clocks": clocks.summary(),
+               "clocks_note": "sampled with nvidia-smi every 100 ms during the timed region"}
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_e2e(args, roi, tensors, lset, N, M, tau, dev, world):
+    """Same step through the C ABI with host buffers: per tensor, copy logits, W and
+    dWm from pinned host memory, run fwd + bwd, copy Wm, the hard bits and the logit
+    gradients back; two streams alternate so copies overlap compute."""
+    import torch
+    per_layer = [t for t in tensors if t["id"] < len(WL.PROJS)]  # one layer's shapes
+    host = {}
+    for t in per_layer:
+        p = t["id"]
+        host[p] = {
+            "phi": t["phi"].cpu().pin_memory(), "W": t["W"].cpu().pin_memory(), "dWm": t["dWm"].cpu().pin_memory(),
+            "Wm": torch.empty_like(t["Wm"], device="cpu").pin_memory(),
+            "hard": torch.empty_like(t["hard"], device="cpu").pin_memory(),
+            "dphi": torch.empty_like(t["dphi"], device="cpu").pin_memory()}
+    streams = [torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)]
+    h2d = sum(t["rows"] * t["cols"] * 8 for t in tensors)
+    d2h = sum(t["rows"] * t["cols"] * 6 + t["hard"].numel() * 4 for t in tensors)
+
+    def one(s):
+        for i, t in enumerate(tensors):
+            hs = host[t["id"] % len(WL.PROJS)]
+            stm = streams[i % 2]
+            st = roi.NoiseState(0, s, t["id"], 1.0, 0)
+            with torch.cuda.stream(stm):
+                t["phi"].copy_(hs["phi"], non_blocking=True)
+                t["W"].copy_(hs["W"], non_blocking=True)
+                t["dWm"].copy_(hs["dWm"], non_blocking=True)
+                roi.roi_mask_fwd_ex(t["phi"], t["W"], N, M, tau, st, t["Wm"], None, t["hard"], stream=stm)
+                roi.roi_mask_bwd(t["phi"], t["W"], st, N, M, t["dWm"], tau, t["dphi"], None, stream=stm)
+                hs["Wm"].copy_(t["Wm"], non_blocking=True)
+                hs["hard"].copy_(t["hard"], non_blocking=True)
+                hs["dphi"].copy_(t["dphi"], non_blocking=True)
+
+    one(10_000)
+    torch.cuda.synchronize()
+    steps = max(1, args.e2e_steps)
+    t0 = time.perf_counter()
+    for s in range(steps):
+        one(10_001 + s)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t0
+    if world > 1:
+        import torch.distributed as dist
+        tt = torch.tensor([wall], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        wall = float(tt.item())
+    groups = world * (lset.elements // M) * steps
+    return {"value": groups / wall, "unit": "groups/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "steps": steps, "ms_per_step": 1e3 * wall / steps,
+            "note": "host buffers: one layer's tensors in pinned memory, reused for all layers"}
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()
