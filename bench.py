@@ -50,7 +50,22 @@ def parse_args():
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--layers", type=int, default=None, help="only the first L layers (profiling cases)")
+    p.add_argument("--proj", default=None, help="comma-separated projections to keep, e.g. gate")
     return p.parse_args()
+
+
+def selected_tensors(args):
+    """[(layer, proj_index, rows, cols)] of the layer set, optionally restricted."""
+    lset = WL.LAYER_SETS[args.set]
+    keep = set(args.proj.split(",")) if args.proj else set(WL.PROJS)
+    out = []
+    for layer, p, rows, cols in lset.tensors():
+        if args.layers is not None and layer >= args.layers:
+            continue
+        if WL.PROJS[p] in keep:
+            out.append((layer, p, rows, cols))
+    return out
 
 
 def config_for(args):
@@ -58,14 +73,18 @@ def config_for(args):
     cfg = WL.CONFIGS[args.set]
     N, M = map(int, args.nm.split(":"))
     tau = args.tau if args.tau is not None else cfg.taus[0]
-    E = lset.elements
+    sel = selected_tensors(args)
+    E = sum(r * c for _, _, r, c in sel)
     h, kv, i = lset.hidden, lset.kv, lset.inter
+    layers = lset.layers if args.layers is None else min(args.layers, lset.layers)
+    projs = "{q,o %dx%d; k,v %dx%d; gate,up %dx%d; down %dx%d}" % (h, h, kv, h, i, h, h, i)
+    if args.proj:
+        projs = "{" + ",".join(f"{q} {'x'.join(map(str, lset.shape(q)))}" for q in args.proj.split(",")) + "}"
     return {
-        "workload": (f"{args.set}-shaped layer set, {N}:{M}, tau={tau}, {lset.layers} layers x "
-                     f"{{q,o {h}x{h}; k,v {kv}x{h}; gate,up {i}x{h}; down {h}x{i}}}, "
+        "workload": (f"{args.set}-shaped layer set, {N}:{M}, tau={tau}, {layers} layers x {projs}, "
                      f"logits {cfg.logits}, step-keyed noise"),
         "layer_set": args.set, "N": N, "M": M, "tau": tau, "lambda": 1.0,
-        "elements": E, "groups": E // M, "tensors": len(lset.tensors()),
+        "elements": E, "groups": E // M, "tensors": len(sel),
         "l2": "inputs larger than L2: every step streams the whole set (>90 GB for the 7B set)",
     }
 
@@ -297,7 +316,7 @@ def run_ours(args):
     lset = WL.LAYER_SETS[args.set]
     kind = WL.CONFIGS[args.set].logits
     tensors = []
-    for layer, p, rows, cols in lset.tensors():
+    for layer, p, rows, cols in selected_tensors(args):
         W, phi, dWm = WL.make_inputs(rows, cols, kind, WL.tensor_seed(layer, p) + 7919 * rank, device=dev)
         tensors.append({
             "id": layer * len(WL.PROJS) + p, "rows": rows, "cols": cols, "phi": phi, "W": W, "dWm": dWm,
@@ -359,7 +378,7 @@ def run_ours(args):
         dist.all_reduce(tt, op=dist.ReduceOp.MAX)
         elapsed = float(tt.item())
 
-    E = lset.elements
+    E = cfg["elements"]
     groups_all = world * (E // M) * args.steps
     value = groups_all / elapsed
     step_gbs = world * E * (FWD_BYTES + BWD_BYTES) * args.steps / elapsed / 1e9
@@ -405,10 +424,11 @@ def run_e2e(args, roi, tensors, lset, N, M, tau, dev, world):
     dWm from pinned host memory, run fwd + bwd, copy Wm, the hard bits and the logit
     gradients back; two streams alternate so copies overlap compute."""
     import torch
-    per_layer = [t for t in tensors if t["id"] < len(WL.PROJS)]  # one layer's shapes
     host = {}
-    for t in per_layer:
-        p = t["id"]
+    for t in tensors:
+        p = t["id"] % len(WL.PROJS)
+        if p in host:
+            continue
         host[p] = {
             "phi": t["phi"].cpu().pin_memory(), "W": t["W"].cpu().pin_memory(), "dWm": t["dWm"].cpu().pin_memory(),
             "Wm": torch.empty_like(t["Wm"], device="cpu").pin_memory(),
@@ -446,7 +466,7 @@ def run_e2e(args, roi, tensors, lset, N, M, tau, dev, world):
         tt = torch.tensor([wall], device=dev)
         dist.all_reduce(tt, op=dist.ReduceOp.MAX)
         wall = float(tt.item())
-    groups = world * (lset.elements // M) * steps
+    groups = world * (sum(t["rows"] * t["cols"] for t in tensors) // M) * steps
     return {"value": groups / wall, "unit": "groups/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
             "steps": steps, "ms_per_step": 1e3 * wall / steps,
             "note": "host buffers: one layer's tensors in pinned memory, reused for all layers"}

@@ -21,7 +21,8 @@
  *  - bfloat16 tensors are passed as their 16-bit patterns (roi_bf16).
  *  - Every tensor pointer is caller-owned DEVICE memory, 16-byte aligned, and
  *    must not alias any other tensor of the same call.  The library allocates
- *    no memory.
+ *    no memory.  With rows == 0 nothing is read or written and tensor pointers
+ *    may be NULL.
  *  - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
  *    stream).  Arguments are validated on the host before anything is
  *    launched; on any non-OK return nothing was launched and nothing written.
@@ -113,6 +114,17 @@ roi_status roi_mask_bwd(const float* logits, const roi_bf16* W, const roi_noise_
 roi_status roi_hard_mask_export(const float* logits, int N, int M, int64_t rows, int64_t cols,
                                 uint32_t* out_bits, const roi_bf16* W, roi_bf16* out_Wpruned,
                                 void* stream);
+
+/* The noise of a call, materialised (for inspecting or reproducing a sample; the
+ * mask calls never store it).  st->lambda is ignored; st->row_offset applies.
+ *  roi_noise_words: out_words[rows*cols] uint32, the Philox word x_e of element e.
+ *  roi_gumbel_noise: out_g[rows*cols] float32, g_e = -log(-log u_e) exactly as the
+ *    mask kernels form it (Algorithm 1, Gumbel lines): -log u through a range
+ *    reduction and the 2 atanh series (relative error about 2e-7), the outer log
+ *    through the hardware log2 (absolute error about 1e-7). */
+roi_status roi_noise_words(const roi_noise_state* st, int64_t rows, int64_t cols, uint32_t* out_words,
+                           void* stream);
+roi_status roi_gumbel_noise(const roi_noise_state* st, int64_t rows, int64_t cols, float* out_g, void* stream);
 
 /* Device-side status.  The kernels wait on their own asynchronous copies with
  * a time limit (about 2 s); a kernel that gives up records it in a per-device

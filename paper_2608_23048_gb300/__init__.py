@@ -15,7 +15,7 @@ import os
 __all__ = [
     "RoiError", "NoiseState", "lib", "roi_mask_fwd", "roi_mask_fwd_ex", "roi_mask_bwd",
     "roi_hard_mask_export", "roi_device_status", "roi_status_string", "roi_launch_count",
-    "library_path", "hard_words",
+    "library_path", "hard_words", "roi_noise_words", "roi_gumbel_noise",
 ]
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
@@ -57,11 +57,14 @@ def lib() -> ctypes.CDLL:
     L.roi_mask_bwd.argtypes = [_P, _P, ctypes.POINTER(NoiseState), i32, i32, _P, f32, i64, i64, _P, _P, _P]
     L.roi_hard_mask_export.argtypes = [_P, i32, i32, i64, i64, _P, _P, _P, _P]
     L.roi_device_status.argtypes = [_P]
+    L.roi_noise_words.argtypes = [ctypes.POINTER(NoiseState), i64, i64, _P, _P]
+    L.roi_gumbel_noise.argtypes = [ctypes.POINTER(NoiseState), i64, i64, _P, _P]
     L.roi_status_string.argtypes = [i32]
     L.roi_status_string.restype = ctypes.c_char_p
     L.roi_launch_count.argtypes = []
     L.roi_launch_count.restype = ctypes.c_uint64
-    for name in ("roi_mask_fwd", "roi_mask_fwd_ex", "roi_mask_bwd", "roi_hard_mask_export", "roi_device_status"):
+    for name in ("roi_mask_fwd", "roi_mask_fwd_ex", "roi_mask_bwd", "roi_hard_mask_export", "roi_device_status",
+                 "roi_noise_words", "roi_gumbel_noise"):
         getattr(L, name).restype = i32
     _LIB = L
     return L
@@ -169,6 +172,22 @@ def roi_hard_mask_export(logits, N, M, out_bits, W=None, out_Wpruned=None, strea
     s = lib().roi_hard_mask_export(_ptr(logits), int(N), int(M), rows, cols, _ptr(out_bits), _ptr(W),
                                    _ptr(out_Wpruned), _stream(stream))
     _raise(s, "roi_hard_mask_export")
+
+
+def roi_noise_words(state: NoiseState, rows, cols, out_words, stream=None):
+    """Philox words of every element of a [rows, cols] call (int32 tensor of rows*cols)."""
+    import torch
+    _check_tensor(out_words, "out_words", torch.int32, (rows * cols,))
+    st = state if isinstance(state, NoiseState) else NoiseState(*state)
+    _raise(lib().roi_noise_words(ctypes.byref(st), rows, cols, _ptr(out_words), _stream(stream)), "roi_noise_words")
+
+
+def roi_gumbel_noise(state: NoiseState, rows, cols, out_g, stream=None):
+    """Gumbel noise of every element of a [rows, cols] call (float32 tensor of rows*cols)."""
+    import torch
+    _check_tensor(out_g, "out_g", torch.float32, (rows * cols,))
+    st = state if isinstance(state, NoiseState) else NoiseState(*state)
+    _raise(lib().roi_gumbel_noise(ctypes.byref(st), rows, cols, _ptr(out_g), _stream(stream)), "roi_gumbel_noise")
 
 
 def roi_device_status(stream=None):

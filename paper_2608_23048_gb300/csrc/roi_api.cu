@@ -97,11 +97,13 @@ extern "C" {
 roi_status roi_mask_fwd_ex(const float* logits, const roi_bf16* W, int N, int M, float tau,
                            const roi_noise_state* st, int64_t rows, int64_t cols, roi_bf16* out_Wm,
                            float* out_soft, uint32_t* out_hard, void* stream) {
-  if (logits == nullptr || W == nullptr || out_Wm == nullptr || st == nullptr) return ROI_ERR_NULL;
+  if (st == nullptr) return ROI_ERR_NULL;
   roi_status s = check_common(N, M, tau, rows, cols);
   if (s != ROI_OK) return s;
   if (st->row_offset < 0) return ROI_ERR_SHAPE;
   if (!finite_positive(st->lambda)) return ROI_ERR_TAU;
+  if (rows == 0) return ROI_OK;  // nothing is read or written; pointers may be NULL
+  if (logits == nullptr || W == nullptr || out_Wm == nullptr) return ROI_ERR_NULL;
   if (!aligned16(logits) || !aligned16(W) || !aligned16(out_Wm) || !aligned16(out_soft) || !aligned16(out_hard))
     return ROI_ERR_ALIGN;
   const int64_t E = rows * cols;
@@ -141,12 +143,13 @@ roi_status roi_mask_fwd(const float* logits, const roi_bf16* W, int N, int M, fl
 roi_status roi_mask_bwd(const float* logits, const roi_bf16* W, const roi_noise_state* st, int N, int M,
                         const roi_bf16* dWm, float tau, int64_t rows, int64_t cols, float* out_dlogits,
                         roi_bf16* out_dW, void* stream) {
-  if (logits == nullptr || W == nullptr || st == nullptr || dWm == nullptr || out_dlogits == nullptr)
-    return ROI_ERR_NULL;
+  if (st == nullptr) return ROI_ERR_NULL;
   roi_status s = check_common(N, M, tau, rows, cols);
   if (s != ROI_OK) return s;
   if (st->row_offset < 0) return ROI_ERR_SHAPE;
   if (!finite_positive(st->lambda)) return ROI_ERR_TAU;
+  if (rows == 0) return ROI_OK;
+  if (logits == nullptr || W == nullptr || dWm == nullptr || out_dlogits == nullptr) return ROI_ERR_NULL;
   if (!aligned16(logits) || !aligned16(W) || !aligned16(dWm) || !aligned16(out_dlogits) || !aligned16(out_dW))
     return ROI_ERR_ALIGN;
   const int64_t E = rows * cols;
@@ -173,10 +176,11 @@ roi_status roi_mask_bwd(const float* logits, const roi_bf16* W, const roi_noise_
 
 roi_status roi_hard_mask_export(const float* logits, int N, int M, int64_t rows, int64_t cols, uint32_t* out_bits,
                                 const roi_bf16* W, roi_bf16* out_Wpruned, void* stream) {
-  if (logits == nullptr || out_bits == nullptr) return ROI_ERR_NULL;
-  if ((W == nullptr) != (out_Wpruned == nullptr)) return ROI_ERR_NULL;
   roi_status s = check_common(N, M, 1.0f, rows, cols);
   if (s != ROI_OK) return s;
+  if (rows == 0) return ROI_OK;
+  if (logits == nullptr || out_bits == nullptr) return ROI_ERR_NULL;
+  if ((W == nullptr) != (out_Wpruned == nullptr)) return ROI_ERR_NULL;
   if (!aligned16(logits) || !aligned16(out_bits) || !aligned16(W) || !aligned16(out_Wpruned)) return ROI_ERR_ALIGN;
   const int64_t E = rows * cols;
   const Range in[2] = {{logits, uint64_t(E) * 4}, {W, uint64_t(E) * 2}};
@@ -193,6 +197,27 @@ roi_status roi_hard_mask_export(const float* logits, int N, int M, int64_t rows,
   c.M = M;
   c.stream = static_cast<cudaStream_t>(stream);
   return finish(launch_export(c));
+}
+
+static roi_status noise_call(const roi_noise_state* st, int64_t rows, int64_t cols, uint32_t* words, float* g,
+                             void* stream) {
+  if (st == nullptr) return ROI_ERR_NULL;
+  if (rows < 0 || cols <= 0 || (rows > 0 && cols > INT64_MAX / 64 / rows) || st->row_offset < 0) return ROI_ERR_SHAPE;
+  if (rows == 0) return ROI_OK;
+  if (words == nullptr && g == nullptr) return ROI_ERR_NULL;
+  if (!aligned16(words) || !aligned16(g)) return ROI_ERR_ALIGN;
+  const int64_t E = rows * cols;
+  return finish(launch_noise(make_noise(*st, cols), E, words, g, static_cast<cudaStream_t>(stream)));
+}
+
+roi_status roi_noise_words(const roi_noise_state* st, int64_t rows, int64_t cols, uint32_t* out_words, void* stream) {
+  if (out_words == nullptr && rows > 0) return ROI_ERR_NULL;
+  return noise_call(st, rows, cols, out_words, nullptr, stream);
+}
+
+roi_status roi_gumbel_noise(const roi_noise_state* st, int64_t rows, int64_t cols, float* out_g, void* stream) {
+  if (out_g == nullptr && rows > 0) return ROI_ERR_NULL;
+  return noise_call(st, rows, cols, nullptr, out_g, stream);
 }
 
 roi_status roi_device_status(void* stream) {

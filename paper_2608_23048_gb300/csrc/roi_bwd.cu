@@ -9,8 +9,11 @@ namespace roi {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kTile = 4096;
-constexpr int kStages = 3;
+// Tiles of 512 M elements: two groups per thread per tile, relaxed in lockstep.
+template <int M>
+constexpr int kTile = 512 * M;
+template <int M>
+constexpr int kStages = M == 4 ? 3 : 2;
 
 struct BwdArgs {
   const float* phi;
@@ -25,7 +28,6 @@ struct BwdArgs {
   unsigned int* status;
 };
 
-template <int M>
 __device__ __forceinline__ void unpack4(uint2 q, float* out) {
   out[0] = bf16_bits_to_float(q.x & 0xffffu);
   out[1] = bf16_bits_to_float(q.x >> 16);
@@ -33,58 +35,114 @@ __device__ __forceinline__ void unpack4(uint2 q, float* out) {
   out[3] = bf16_bits_to_float(q.y >> 16);
 }
 
-template <int N, int M, bool TAU1>
-__device__ __forceinline__ void bwd_group(const float* phi_g, const uint16_t* W_g, const uint16_t* dWm_g,
-                                          int64_t e0, const BwdArgs& a) {
-  float ph[M], w[M], dw[M], kap[M], c[M];
-#pragma unroll
-  for (int s = 0; s < M / 4; ++s) {
-    const float4 p = reinterpret_cast<const float4*>(phi_g)[s];
-    ph[4 * s] = p.x, ph[4 * s + 1] = p.y, ph[4 * s + 2] = p.z, ph[4 * s + 3] = p.w;
-    unpack4<M>(reinterpret_cast<const uint2*>(W_g)[s], w + 4 * s);
-    unpack4<M>(reinterpret_cast<const uint2*>(dWm_g)[s], dw + 4 * s);
-  }
-#pragma unroll
-  for (int s = 0; s < M / 4; ++s) {
-    const uint4 x = noise_block(a.np, a.np.e_base + uint64_t(e0) + 4 * s);
-    kap[4 * s + 0] = fmaf(ph[4 * s + 0], a.np.inv_lam, gumbel_from_word(x.x));
-    kap[4 * s + 1] = fmaf(ph[4 * s + 1], a.np.inv_lam, gumbel_from_word(x.y));
-    kap[4 * s + 2] = fmaf(ph[4 * s + 2], a.np.inv_lam, gumbel_from_word(x.z));
-    kap[4 * s + 3] = fmaf(ph[4 * s + 3], a.np.inv_lam, gumbel_from_word(x.w));
-  }
-#pragma unroll
-  for (int l = 0; l < M; ++l) c[l] = dw[l] * w[l];
-
-  FastGroup<N, M, TAU1, true> fg;
-  fg.forward(kap, a.inv_tau);
-  float dk[M], S[M];
-  if (!fg.flag) {
-    fg.backward(c, a.inv_tau, dk);
-#pragma unroll
-    for (int l = 0; l < M; ++l) S[l] = fg.S[l];
+template <class V>
+__device__ __forceinline__ float lane_of(V v, int h) {
+  if constexpr (vlanes<V>() == 1) {
+    return v;
   } else {
-    ExactGroup<N, M> ex;
-    ex.forward(kap, N, M, a.tau, S);
-    ex.backward(c, N, M, a.tau, dk);
+    return h == 0 ? lo(v) : hi(v);
   }
+}
+
+// L groups (one per lane of V) in lockstep: regenerate keys and relaxation,
+// sweep back, write dL/dphi (and dW).
+template <int N, int M, bool TAU1, class V>
+__device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint16_t* const* W_g,
+                                           const uint16_t* const* dWm_g, const int64_t* e0, const BwdArgs& a) {
+  constexpr int L = vlanes<V>();
+  V kap[M], c[M];
+  {
+    float ph[L][M], w[L][M], dw[L][M];
+    uint32_t x[L][M];
 #pragma unroll
-  for (int s = 0; s < M / 4; ++s) {
-    reinterpret_cast<float4*>(a.dphi + e0)[s] =
-        make_float4(dk[4 * s] * a.np.inv_lam, dk[4 * s + 1] * a.np.inv_lam, dk[4 * s + 2] * a.np.inv_lam,
-                    dk[4 * s + 3] * a.np.inv_lam);
-    if (a.dW != nullptr) {
-      uint2 o;
-      o.x = pack_bf16x2(dw[4 * s] * S[4 * s], dw[4 * s + 1] * S[4 * s + 1]);
-      o.y = pack_bf16x2(dw[4 * s + 2] * S[4 * s + 2], dw[4 * s + 3] * S[4 * s + 3]);
-      reinterpret_cast<uint2*>(a.dW + e0)[s] = o;
+    for (int h = 0; h < L; ++h) {
+      const uint64_t q0 = (a.np.e_base + uint64_t(e0[h])) >> 2;
+#pragma unroll
+      for (int s = 0; s < M / 4; ++s) {
+        const float4 p = reinterpret_cast<const float4*>(phi_g[h])[s];
+        ph[h][4 * s] = p.x, ph[h][4 * s + 1] = p.y, ph[h][4 * s + 2] = p.z, ph[h][4 * s + 3] = p.w;
+        unpack4(reinterpret_cast<const uint2*>(W_g[h])[s], w[h] + 4 * s);
+        unpack4(reinterpret_cast<const uint2*>(dWm_g[h])[s], dw[h] + 4 * s);
+        const uint4 q = noise_block_q(a.np, q0 + s);
+        x[h][4 * s] = q.x, x[h][4 * s + 1] = q.y, x[h][4 * s + 2] = q.z, x[h][4 * s + 3] = q.w;
+      }
     }
+#pragma unroll
+    for (int l = 0; l < M; ++l) {
+      V one_plus, phv, wv, dwv;
+      if constexpr (L == 1) {
+        one_plus = __uint_as_float(0x3f800000u | (x[0][l] >> 9));
+        phv = ph[0][l], wv = w[0][l], dwv = dw[0][l];
+      } else {
+        one_plus =
+            f2(__uint_as_float(0x3f800000u | (x[0][l] >> 9)), __uint_as_float(0x3f800000u | (x[1][l] >> 9)));
+        phv = f2(ph[0][l], ph[1][l]), wv = f2(w[0][l], w[1][l]), dwv = f2(dw[0][l], dw[1][l]);
+      }
+      const V u = vsub(one_plus, vconst<V>(__uint_as_float(0x3f7fffffu)));
+      kap[l] = vfma(phv, vconst<V>(a.np.inv_lam), gumbel_from_u(u));
+      c[l] = vmul(dwv, wv);
+    }
+  }
+
+  FastGroup<N, M, TAU1, true, V> fg;
+  fg.forward(kap, a.inv_tau);
+  if (a.dW != nullptr) {
+    // dW = bf16(dWm * S) now, while mu is live anyway (dWm is re-read)
+#pragma unroll
+    for (int h = 0; h < L; ++h) {
+#pragma unroll
+      for (int s = 0; s < M / 4; ++s) {
+        float d[4];
+        unpack4(reinterpret_cast<const uint2*>(dWm_g[h])[s], d);
+        uint2 o;
+        o.x = pack_bf16x2(__fmul_rn(d[0], lane_of(fg.soft(4 * s), h)), __fmul_rn(d[1], lane_of(fg.soft(4 * s + 1), h)));
+        o.y = pack_bf16x2(__fmul_rn(d[2], lane_of(fg.soft(4 * s + 2), h)), __fmul_rn(d[3], lane_of(fg.soft(4 * s + 3), h)));
+        reinterpret_cast<uint2*>(a.dW + e0[h])[s] = o;
+      }
+    }
+  }
+  V dkv[M];
+  fg.backward(c, a.inv_tau, dkv);
+#pragma unroll
+  for (int h = 0; h < L; ++h) {
+    float dk[M];
+#pragma unroll
+    for (int l = 0; l < M; ++l) dk[l] = lane_of(dkv[l], h);
+    if ((fg.flag >> h) & 1u) {
+      float k[M], cc[M], S[M];
+#pragma unroll
+      for (int l = 0; l < M; ++l) {
+        k[l] = lane_of(kap[l], h);
+        cc[l] = lane_of(c[l], h);
+      }
+      ExactGroup<N, M> ex;
+      ex.forward(k, N, M, a.tau, S);
+      ex.backward(cc, N, M, a.tau, dk);
+      if (a.dW != nullptr) {
+#pragma unroll
+        for (int s = 0; s < M / 4; ++s) {
+          float d[4];
+          unpack4(reinterpret_cast<const uint2*>(dWm_g[h])[s], d);
+          uint2 o;
+          o.x = pack_bf16x2(__fmul_rn(d[0], S[4 * s]), __fmul_rn(d[1], S[4 * s + 1]));
+          o.y = pack_bf16x2(__fmul_rn(d[2], S[4 * s + 2]), __fmul_rn(d[3], S[4 * s + 3]));
+          reinterpret_cast<uint2*>(a.dW + e0[h])[s] = o;
+        }
+      }
+    }
+#pragma unroll
+    for (int s = 0; s < M / 4; ++s)
+      reinterpret_cast<float4*>(a.dphi + e0[h])[s] =
+          make_float4(dk[4 * s] * a.np.inv_lam, dk[4 * s + 1] * a.np.inv_lam, dk[4 * s + 2] * a.np.inv_lam,
+                      dk[4 * s + 3] * a.np.inv_lam);
   }
 }
 
 template <int N, int M, bool TAU1>
-__global__ void __launch_bounds__(kThreads) roi_bwd_kernel(BwdArgs a) {
+__global__ void __launch_bounds__(kThreads, M == 4 ? 4 : 2) roi_bwd_kernel(BwdArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
-  constexpr int kGroupsPerThread = kTile / M / kThreads;
+  constexpr int kT = kTile<M>;
+  static_assert(kT / M == 2 * kThreads, "two groups per thread per tile");
   TileSrc<3> src;
   src.ptr[0] = reinterpret_cast<const uint8_t*>(a.phi);
   src.esize[0] = 4;
@@ -93,25 +151,31 @@ __global__ void __launch_bounds__(kThreads) roi_bwd_kernel(BwdArgs a) {
   src.ptr[2] = reinterpret_cast<const uint8_t*>(a.dWm);
   src.esize[2] = 2;
 
-  const bool ok = run_tiles<kThreads, kTile, kStages, 3>(
+  const bool ok = run_tiles<kThreads, kT, kStages<M>, 3>(
       smem, src, a.full_tiles, a.status, [&](const uint8_t* const* stage, int64_t tile) {
         const float* sphi = reinterpret_cast<const float*>(stage[0]);
         const uint16_t* sW = reinterpret_cast<const uint16_t*>(stage[1]);
         const uint16_t* sdW = reinterpret_cast<const uint16_t*>(stage[2]);
-        const int64_t base = tile * kTile;
-#pragma unroll 1
-        for (int j = 0; j < kGroupsPerThread; ++j) {
-          const int gi = threadIdx.x + j * kThreads;
-          bwd_group<N, M, TAU1>(sphi + gi * M, sW + gi * M, sdW + gi * M, base + gi * M, a);
-        }
+        const int64_t base = tile * kT;
+        const int g0 = threadIdx.x, g1 = threadIdx.x + kThreads;
+        const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
+        const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
+        const uint16_t* pd[2] = {sdW + g0 * M, sdW + g1 * M};
+        const int64_t e0[2] = {base + g0 * M, base + g1 * M};
+        bwd_groups<N, M, TAU1, F2>(pp, pw, pd, e0, a);
       });
   if (!ok) return;
 
   if (blockIdx.x == gridDim.x - 1) {
-    const int64_t t0 = a.full_tiles * kTile;
+    const int64_t t0 = a.full_tiles * kT;
     const int64_t tail_groups = (a.E - t0) / M;
-    for (int64_t gi = threadIdx.x; gi < tail_groups; gi += kThreads)
-      bwd_group<N, M, TAU1>(a.phi + t0 + gi * M, a.W + t0 + gi * M, a.dWm + t0 + gi * M, t0 + gi * M, a);
+    for (int64_t gi = threadIdx.x; gi < tail_groups; gi += kThreads) {
+      const float* pp[1] = {a.phi + t0 + gi * M};
+      const uint16_t* pw[1] = {a.W + t0 + gi * M};
+      const uint16_t* pd[1] = {a.dWm + t0 + gi * M};
+      const int64_t e0[1] = {t0 + gi * M};
+      bwd_groups<N, M, TAU1, float>(pp, pw, pd, e0, a);
+    }
   }
 }
 
@@ -144,7 +208,7 @@ struct LaunchCache {
 template <int N, int M, bool TAU1>
 int launch_tiles(const BwdArgs& a, cudaStream_t stream) {
   auto kern = roi_bwd_kernel<N, M, TAU1>;
-  const size_t smem = size_t(kStages) * kTile * 8 + 8 * kStages + 8;
+  const size_t smem = tile_smem_bytes<kTile<M>, kStages<M>>(8);
   static LaunchCache cache;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return -1;
@@ -176,7 +240,7 @@ int launch_bwd(const BwdCall& c) {
   a.dphi = c.dphi;
   a.dW = c.dW;
   a.E = c.E;
-  a.full_tiles = c.E / kTile;
+  a.full_tiles = c.E / (c.M == 8 ? kTile<8> : kTile<4>);
   a.tau = c.tau;
   a.inv_tau = 1.0f / c.tau;
   a.np = c.np;

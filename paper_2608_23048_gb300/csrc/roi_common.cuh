@@ -13,6 +13,8 @@
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 
+#include "roi_vec.cuh"
+
 namespace roi {
 
 // ---------------------------------------------------------------------------
@@ -64,8 +66,11 @@ constexpr uint32_t kPhiloxW1 = 0xBB67AE85u;
 __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
 #pragma unroll
   for (int r = 0; r < 10; ++r) {
-    const uint32_t hi0 = __umulhi(kPhiloxM0, c.x), lo0 = kPhiloxM0 * c.x;
-    const uint32_t hi1 = __umulhi(kPhiloxM1, c.z), lo1 = kPhiloxM1 * c.z;
+    // one 32x32 -> 64-bit product per multiplier gives both (hi, lo) words
+    const uint64_t p0 = uint64_t(kPhiloxM0) * c.x;
+    const uint64_t p1 = uint64_t(kPhiloxM1) * c.z;
+    const uint32_t hi0 = uint32_t(p0 >> 32), lo0 = uint32_t(p0);
+    const uint32_t hi1 = uint32_t(p1 >> 32), lo1 = uint32_t(p1);
     c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
     k0 += kPhiloxW0;
     k1 += kPhiloxW1;
@@ -80,11 +85,13 @@ struct NoiseParams {
   uint64_t e_base;       // row_offset * cols: flat index of this call's element 0
 };
 
+// The four noise words of block q (elements 4q .. 4q+3).
+__device__ __forceinline__ uint4 noise_block_q(const NoiseParams& np, uint64_t q) {
+  return philox4x32_10(make_uint4(uint32_t(q), uint32_t(q >> 32), np.step, np.tensor_id), np.k0, np.k1);
+}
 // Four consecutive noise words for elements e4 .. e4+3 (e4 % 4 == 0).
 __device__ __forceinline__ uint4 noise_block(const NoiseParams& np, uint64_t e4) {
-  const uint64_t q = e4 >> 2;
-  return philox4x32_10(make_uint4(uint32_t(q), uint32_t(q >> 32), np.step, np.tensor_id),
-                       np.k0, np.k1);
+  return noise_block_q(np, e4 >> 2);
 }
 // The word of a single element (any e).
 __device__ __forceinline__ uint32_t noise_word(const NoiseParams& np, uint64_t e) {
@@ -99,10 +106,52 @@ __device__ __forceinline__ float uniform_from_word(uint32_t x) {
   return __uint_as_float(0x3f800000u | (x >> 9)) - __uint_as_float(0x3f7fffffu);
 }
 
-// Gumbel(0,1) sample from a word: -log(-log u) (Algorithm 1), accurate logf.
+// E = -ln(u) for u in [2^-24, 1) with a small relative error everywhere,
+// including u -> 1 where E -> 0 (the hardware log2 has an absolute error floor
+// there).  Method: u = 2^e m with m in [sqrt(1/2), sqrt(2)), so
+// ln u = e ln2 + ln m and ln m = 2 atanh(s), s = (m - 1) / (m + 1), |s| < 0.1716,
+// 2 atanh(s) = 2s + (2/3)s^3 + (2/5)s^5 + (2/7)s^7 + (2/9)s^9 + O(s^11)
+// (truncation below 2^-28 relative).  m - 1 is exact (Sterbenz).  The Horner
+// chain runs on negated coefficients so the result needs no final negation.
+__device__ __forceinline__ void unit_split(float u, float& m, float& ef) {
+  const uint32_t b = __float_as_uint(u);
+  const int32_t e = int32_t(b - 0x3f3504f3u) >> 23;  // 0x3f3504f3 = sqrt(1/2)
+  m = __uint_as_float(b - (uint32_t(e) << 23));
+  // e in [-25, 0] -> float without a conversion instruction (1.5 * 2^23 trick)
+  ef = __int_as_float(0x4b400000 + e) - 12582912.0f;
+}
+template <class V>
+__device__ __forceinline__ V neg_log_unit(V u) {
+  V m, ef;
+  if constexpr (vlanes<V>() == 1) {
+    unit_split(u, m, ef);
+  } else {
+    float m0, m1, e0, e1;
+    unit_split(lo(u), m0, e0);
+    unit_split(hi(u), m1, e1);
+    m = f2(m0, m1);
+    ef = f2(e0, e1);
+  }
+  const V one = vconst<V>(1.0f);
+  const V f = vsub(m, one);
+  const V s = vmul(f, vmap(vadd(m, one), rcp_approx));
+  const V s2 = vmul(s, s);
+  V q = vfma(s2, vconst<V>(-0.22222222f), vconst<V>(-0.28571429f));
+  q = vfma(s2, q, vconst<V>(-0.4f));
+  q = vfma(s2, q, vconst<V>(-0.66666667f));
+  const V nlnm = vfma(vmul(s, s2), q, vmul(s, vconst<V>(-2.0f)));  // -ln m
+  return vfma(ef, vconst<V>(-kLn2), nlnm);
+}
+
+// Gumbel(0,1) samples from words: g = -log(-log u) (Algorithm 1).  The outer
+// log only needs absolute accuracy (g enters the keys additively) and uses the
+// hardware log2.
+template <class V>
+__device__ __forceinline__ V gumbel_from_u(V u) {
+  return vmul(vmap(neg_log_unit(u), lg2_approx), vconst<V>(-kLn2));
+}
 __device__ __forceinline__ float gumbel_from_word(uint32_t x) {
-  const float u = uniform_from_word(x);
-  return -logf(-logf(u));
+  return gumbel_from_u(uniform_from_word(x));
 }
 
 // ---------------------------------------------------------------------------
@@ -131,6 +180,23 @@ __device__ __forceinline__ uint32_t topn_bits(const float (&kap)[M], int N) {
 #pragma unroll
   for (int l = 0; l < M; ++l) bits |= uint32_t(rank[l] < N) << l;
   return bits;
+}
+
+// M = 4: l is selected iff it beats at least 4 - N of the other three keys.
+__device__ __forceinline__ uint32_t topn_bits4(const float (&kap)[4], int N) {
+  const float k0 = fmaxf(kap[0], -INFINITY), k1 = fmaxf(kap[1], -INFINITY);
+  const float k2 = fmaxf(kap[2], -INFINITY), k3 = fmaxf(kap[3], -INFINITY);
+  // tij: i beats j (i < j, ties to the lower index)
+  const bool t01 = k0 >= k1, t02 = k0 >= k2, t03 = k0 >= k3;
+  const bool t12 = k1 >= k2, t13 = k1 >= k3, t23 = k2 >= k3;
+  const bool w0[3] = {t01, t02, t03}, w1[3] = {!t01, t12, t13};
+  const bool w2[3] = {!t02, !t12, t23}, w3[3] = {!t03, !t13, !t23};
+  auto pick = [N](const bool (&w)[3]) -> uint32_t {
+    if (N == 2) return uint32_t((w[0] & w[1]) | (w[0] & w[2]) | (w[1] & w[2]));
+    if (N == 1) return uint32_t(w[0] & w[1] & w[2]);
+    return uint32_t(w[0] | w[1] | w[2]);
+  };
+  return pick(w0) | (pick(w1) << 1) | (pick(w2) << 2) | (pick(w3) << 3);
 }
 
 // Runtime-M version for the generic path (M <= 32).
@@ -163,8 +229,8 @@ __device__ __forceinline__ float lse_excluding(const float* z, int M, int skip) 
   if (m == -INFINITY) return -INFINITY;
   float s = 0.f;
   for (int i = 0; i < M; ++i)
-    if (i != skip) s += expf(z[i] - m);
-  return m + logf(s);
+    if (i != skip) s = __fadd_rn(s, expf(__fsub_rn(z[i], m)));
+  return __fadd_rn(m, logf(s));
 }
 
 template <int NMAX, int MMAX>
@@ -175,16 +241,16 @@ struct ExactGroup {
   __device__ __forceinline__ void forward(const float* kap, int N, int M, float tau, float* S) {
     float z[MMAX];
     for (int l = 0; l < M; ++l) {
-      z[l] = kap[l] / tau;
+      z[l] = __fdiv_rn(kap[l], tau);
       S[l] = 0.f;
     }
     for (int k = 0; k < N; ++k) {
       for (int l = 0; l < M; ++l) zh[k][l] = z[l];
       const float lt = lse_excluding(z, M, -1);
-      for (int l = 0; l < M; ++l) S[l] += expf(z[l] - lt);
+      for (int l = 0; l < M; ++l) S[l] = __fadd_rn(S[l], expf(__fsub_rn(z[l], lt)));
       if (k + 1 < N) {
         float zn[MMAX];
-        for (int l = 0; l < M; ++l) zn[l] = z[l] + (lse_excluding(z, M, l) - lt) / tau;
+        for (int l = 0; l < M; ++l) zn[l] = __fadd_rn(z[l], __fdiv_rn(__fsub_rn(lse_excluding(z, M, l), lt), tau));
         for (int l = 0; l < M; ++l) z[l] = zn[l];
       }
     }
@@ -220,7 +286,8 @@ struct ExactGroup {
 };
 
 // ---------------------------------------------------------------------------
-// Fast register-resident relaxation of one group held by one thread (M <= 8).
+// Fast register-resident relaxation of one group (V = float) or of two groups in
+// lockstep (V = F2, one per half), M <= 8, held by one thread.
 //
 // State: per step the normalised weights mu(k) and, for k < N, the exact
 // complements om(k) = 1 - mu(k), each formed as a sum of the other members
@@ -229,130 +296,146 @@ struct ExactGroup {
 //    softmax is mu' = mu om / sum(mu om).
 //  - otherwise keys are kept as log2 offsets d from the group maximum:
 //    d += log2(om) / tau, renormalised to max 0 each step.
-// `flag` is raised when an exclusive sum drops below 2^-100 (a key gap of ~69
-// natural-log units); the caller then recomputes the group with ExactGroup.
+// The relaxation is a fixed sequence of explicitly rounded operations; the
+// backward kernel recomputes it from the same keys and agrees with the forward's
+// S to within fp32 rounding (packed products may be fused into FMAs by the
+// compiler, see roi_vec.cuh).  The fallback decision depends only on sums of
+// exp2 outputs and is therefore the same in both kernels.
+// `flag` (one bit per lane) is raised when an exclusive sum drops below 2^-100
+// (a key gap of ~69 natural-log units); the caller then recomputes that group
+// with ExactGroup.
 // ---------------------------------------------------------------------------
-template <int M>
-__device__ __forceinline__ void exclusive_sums(const float (&x)[M], float (&ex)[M]) {
+template <int M, class V>
+__device__ __forceinline__ void exclusive_sums(const V (&x)[M], V (&ex)[M]) {
   static_assert(M == 4 || M == 8, "tree exclusive sums for M = 4, 8");
   if constexpr (M == 4) {
-    const float p01 = x[0] + x[1], p23 = x[2] + x[3];
-    ex[0] = x[1] + p23;
-    ex[1] = x[0] + p23;
-    ex[2] = p01 + x[3];
-    ex[3] = p01 + x[2];
+    const V p01 = vadd(x[0], x[1]), p23 = vadd(x[2], x[3]);
+    ex[0] = vadd(x[1], p23);
+    ex[1] = vadd(x[0], p23);
+    ex[2] = vadd(p01, x[3]);
+    ex[3] = vadd(p01, x[2]);
   } else {
-    const float p01 = x[0] + x[1], p23 = x[2] + x[3], p45 = x[4] + x[5], p67 = x[6] + x[7];
-    const float q0 = p01 + p23, q1 = p45 + p67;
-    ex[0] = (x[1] + p23) + q1;
-    ex[1] = (x[0] + p23) + q1;
-    ex[2] = (p01 + x[3]) + q1;
-    ex[3] = (p01 + x[2]) + q1;
-    ex[4] = (x[5] + p67) + q0;
-    ex[5] = (x[4] + p67) + q0;
-    ex[6] = (p45 + x[7]) + q0;
-    ex[7] = (p45 + x[6]) + q0;
+    const V p01 = vadd(x[0], x[1]), p23 = vadd(x[2], x[3]), p45 = vadd(x[4], x[5]), p67 = vadd(x[6], x[7]);
+    const V q0 = vadd(p01, p23), q1 = vadd(p45, p67);
+    ex[0] = vadd(vadd(x[1], p23), q1);
+    ex[1] = vadd(vadd(x[0], p23), q1);
+    ex[2] = vadd(vadd(p01, x[3]), q1);
+    ex[3] = vadd(vadd(p01, x[2]), q1);
+    ex[4] = vadd(vadd(x[5], p67), q0);
+    ex[5] = vadd(vadd(x[4], p67), q0);
+    ex[6] = vadd(vadd(p45, x[7]), q0);
+    ex[7] = vadd(vadd(p45, x[6]), q0);
   }
 }
 
-template <int M>
-__device__ __forceinline__ float sum_of(const float (&x)[M]) {
+template <int M, class V>
+__device__ __forceinline__ V sum_of(const V (&x)[M]) {
   if constexpr (M == 4) {
-    return (x[0] + x[1]) + (x[2] + x[3]);
+    return vadd(vadd(x[0], x[1]), vadd(x[2], x[3]));
   } else {
-    return ((x[0] + x[1]) + (x[2] + x[3])) + ((x[4] + x[5]) + (x[6] + x[7]));
+    return vadd(vadd(vadd(x[0], x[1]), vadd(x[2], x[3])), vadd(vadd(x[4], x[5]), vadd(x[6], x[7])));
   }
 }
 
-template <int M>
-__device__ __forceinline__ float max_of(const float (&x)[M]) {
-  float m = x[0];
+template <int M, class V>
+__device__ __forceinline__ V max_of(const V (&x)[M]) {
+  V m = x[0];
 #pragma unroll
-  for (int l = 1; l < M; ++l) m = fmaxf(m, x[l]);
+  for (int l = 1; l < M; ++l) m = vmax(m, x[l]);
   return m;
 }
 
-template <int M>
-__device__ __forceinline__ float min_of(const float (&x)[M]) {
-  float m = x[0];
+template <int M, class V>
+__device__ __forceinline__ V min_of(const V (&x)[M]) {
+  V m = x[0];
 #pragma unroll
-  for (int l = 1; l < M; ++l) m = fminf(m, x[l]);
+  for (int l = 1; l < M; ++l) m = vmin(m, x[l]);
   return m;
 }
 
-template <int N, int M, bool TAU1, bool KEEP>
+template <int N, int M, bool TAU1, bool KEEP, class V = float>
 struct FastGroup {
-  // KEEP: store mu / om of every step for a backward sweep.
-  float mu[KEEP ? N : 1][M];
-  float om[(KEEP && N > 1) ? N - 1 : 1][M];
-  float S[M];
-  bool flag;
+  // KEEP: store mu of every step for a backward sweep (S is then re-summed from
+  // mu on demand, in the same order, instead of being kept live).
+  V mu[KEEP ? N : 1][M];
+  V S[KEEP ? 1 : M];
+  uint32_t flag;
 
-  __device__ __forceinline__ void forward(const float (&kap)[M], float inv_tau) {
-    const float kmax = max_of(kap);
-    float cur[M];
+  // S_l of a KEEP run, summed exactly as forward() accumulates it.
+  __device__ __forceinline__ V soft(int l) const {
+    V s = mu[0][l];
 #pragma unroll
-    for (int l = 0; l < M; ++l) S[l] = 0.f;
-    flag = false;
+    for (int k = 1; k < N; ++k) s = vadd(s, mu[KEEP ? k : 0][l]);
+    return s;
+  }
+
+  __device__ __forceinline__ void forward(const V (&kap)[M], float inv_tau) {
+    V cur[M];
+    flag = 0;
     if constexpr (TAU1) {
-      float e[M];
+      // Weights relative to the group's first key (any reference works: they are
+      // normalised next); a group whose weights leave [2^-100, 2^100] (a key gap
+      // of ~69), or that holds a non-finite key, goes to the exact routine.
+      V e[M];
 #pragma unroll
-      for (int l = 0; l < M; ++l) e[l] = ex2_approx((kap[l] - kmax) * kLog2e);
-      flag = !(min_of(e) >= kTinyExcl);  // also catches NaN
-      const float r = rcp_approx(sum_of(e));
+      for (int l = 0; l < M; ++l) e[l] = vmap(vmul(vsub(kap[l], kap[0]), vconst<V>(kLog2e)), ex2_approx);
+      const V tot = sum_of(e);
+      flag = vbelow(min_of(e), kTinyExcl) | vbelow(vsub(vconst<V>(1.0f / kTinyExcl), tot), 0.0f);
+      const V r = vmap(tot, rcp_approx);
 #pragma unroll
-      for (int l = 0; l < M; ++l) cur[l] = e[l] * r;
+      for (int l = 0; l < M; ++l) cur[l] = vmul(e[l], r);
 #pragma unroll
       for (int k = 0; k < N; ++k) {
 #pragma unroll
         for (int l = 0; l < M; ++l) {
-          S[l] += cur[l];
-          if constexpr (KEEP) mu[k][l] = cur[l];
+          if constexpr (KEEP) {
+            mu[k][l] = cur[l];
+          } else {
+            S[l] = k == 0 ? cur[l] : vadd(S[l], cur[l]);
+          }
         }
         if (k + 1 < N) {
-          float o[M], v[M];
+          V o[M], v[M];
           exclusive_sums(cur, o);
 #pragma unroll
-          for (int l = 0; l < M; ++l) {
-            if constexpr (KEEP) om[k < N - 1 ? k : 0][l] = o[l];
-            v[l] = cur[l] * o[l];
-          }
-          const float rt = rcp_approx(sum_of(v));
+          for (int l = 0; l < M; ++l) v[l] = vmul(cur[l], o[l]);
+          const V rt = vmap(sum_of(v), rcp_approx);
 #pragma unroll
-          for (int l = 0; l < M; ++l) cur[l] = v[l] * rt;
+          for (int l = 0; l < M; ++l) cur[l] = vmul(v[l], rt);
         }
       }
     } else {
-      const float sc = inv_tau * kLog2e;
-      float d[M];
+      const V kmax = max_of(kap);
+      const V sc = vconst<V>(inv_tau * kLog2e);
+      const V itau = vconst<V>(inv_tau);
+      V d[M];
 #pragma unroll
-      for (int l = 0; l < M; ++l) d[l] = (kap[l] - kmax) * sc;
-      if (!(kmax > -INFINITY && kmax < INFINITY)) flag = true;
+      for (int l = 0; l < M; ++l) d[l] = vmul(vsub(kap[l], kmax), sc);
+      flag = vbelow(vsub(kmax, kmax), 0.0f);  // non-finite maximum
 #pragma unroll
       for (int k = 0; k < N; ++k) {
-        float e[M];
+        V e[M];
 #pragma unroll
-        for (int l = 0; l < M; ++l) e[l] = ex2_approx(d[l]);
-        const float r = rcp_approx(sum_of(e));
+        for (int l = 0; l < M; ++l) e[l] = vmap(d[l], ex2_approx);
+        const V r = vmap(sum_of(e), rcp_approx);
 #pragma unroll
         for (int l = 0; l < M; ++l) {
-          cur[l] = e[l] * r;
-          S[l] += cur[l];
-          if constexpr (KEEP) mu[k][l] = cur[l];
+          cur[l] = vmul(e[l], r);
+          if constexpr (KEEP) {
+            mu[k][l] = cur[l];
+          } else {
+            S[l] = k == 0 ? cur[l] : vadd(S[l], cur[l]);
+          }
         }
         if (k + 1 < N) {
-          float ex[M];
+          V ex[M];
           exclusive_sums(e, ex);
-          flag |= !(min_of(ex) >= kTinyExcl);
+          flag |= vbelow(min_of(ex), kTinyExcl);
 #pragma unroll
-          for (int l = 0; l < M; ++l) {
-            const float o = ex[l] * r;
-            if constexpr (KEEP) om[k < N - 1 ? k : 0][l] = o;
-            d[l] += lg2_approx(o) * inv_tau;
-          }
-          const float dm = max_of(d);
+          for (int l = 0; l < M; ++l) d[l] = vfma(vmap(vmul(ex[l], r), lg2_approx), itau, d[l]);
+          const V dm = max_of(d);
 #pragma unroll
-          for (int l = 0; l < M; ++l) d[l] -= dm;
+          for (int l = 0; l < M; ++l) d[l] = vsub(d[l], dm);
         }
       }
     }
@@ -360,31 +443,35 @@ struct FastGroup {
 
   // Reverse sweep (requires KEEP): dk = dL/dkappa for c = dL/dS.
   //   abar_l = b_l + (mu_l / tau) (c_l - <c, mu> + H_l - B),
-  //   H_l = sum_{i != l} b_i / om_i,  B = sum_i b_i.
-  __device__ __forceinline__ void backward(const float (&c)[M], float inv_tau, float (&dk)[M]) const {
+  //   H_l = sum_{i != l} b_i / om_i,  B = sum_i b_i,
+  // with om_i = 1 - mu_i formed as the sum of the other members' mu.
+  __device__ __forceinline__ void backward(const V (&c)[M], float inv_tau, V (&dk)[M]) const {
     static_assert(KEEP, "backward needs the stored steps");
-    float b[M];
+    const V itau = vconst<V>(inv_tau);
+    V b[M];
     {
-      float cm[M];
+      V cm[M];
 #pragma unroll
-      for (int l = 0; l < M; ++l) cm[l] = c[l] * mu[N - 1][l];
-      const float cmu = sum_of(cm);
+      for (int l = 0; l < M; ++l) cm[l] = vmul(c[l], mu[N - 1][l]);
+      const V cmu = sum_of(cm);
 #pragma unroll
-      for (int l = 0; l < M; ++l) b[l] = mu[N - 1][l] * inv_tau * (c[l] - cmu);
+      for (int l = 0; l < M; ++l) b[l] = vmul(vmul(mu[N - 1][l], itau), vsub(c[l], cmu));
     }
 #pragma unroll
     for (int k = N - 2; k >= 0; --k) {
-      float cm[M], h[M], H[M];
+      V cm[M], h[M], H[M], om[M];
+      exclusive_sums(mu[k], om);
 #pragma unroll
       for (int l = 0; l < M; ++l) {
-        cm[l] = c[l] * mu[k][l];
-        h[l] = b[l] * rcp_approx(om[k][l]);
+        cm[l] = vmul(c[l], mu[k][l]);
+        h[l] = vmul(b[l], vmap(om[l], rcp_approx));
       }
-      const float cmu = sum_of(cm);
-      const float B = sum_of(b);
+      const V cmu = sum_of(cm);
+      const V B = sum_of(b);
       exclusive_sums(h, H);
 #pragma unroll
-      for (int l = 0; l < M; ++l) b[l] += mu[k][l] * inv_tau * (((c[l] - cmu) + H[l]) - B);
+      for (int l = 0; l < M; ++l)
+        b[l] = vfma(vmul(mu[k][l], itau), vsub(vadd(vsub(c[l], cmu), H[l]), B), b[l]);
     }
 #pragma unroll
     for (int l = 0; l < M; ++l) dk[l] = b[l];

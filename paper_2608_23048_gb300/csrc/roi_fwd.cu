@@ -9,8 +9,12 @@ namespace roi {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kTile = 4096;    // elements per tile (16 KB of logits)
-constexpr int kStages = 4;
+// Tiles of 512 M elements give every thread two groups per tile, relaxed in
+// lockstep on packed FP32 (F2).  Stages: 48 KB (M = 4) or 48 KB (M = 8, two).
+template <int M>
+constexpr int kTile = 512 * M;
+template <int M>
+constexpr int kStages = M == 4 ? 4 : 2;
 
 struct FwdArgs {
   const float* phi;
@@ -24,20 +28,6 @@ struct FwdArgs {
   NoiseParams np;
   unsigned int* status;
 };
-
-// Perturbed keys of one group of M (M % 4 == 0) starting at call-flat index e0.
-template <int M>
-__device__ __forceinline__ void group_keys(const float (&ph)[M], uint64_t e0, const NoiseParams& np,
-                                           float (&kap)[M]) {
-#pragma unroll
-  for (int s = 0; s < M / 4; ++s) {
-    const uint4 x = noise_block(np, np.e_base + e0 + 4 * s);
-    kap[4 * s + 0] = fmaf(ph[4 * s + 0], np.inv_lam, gumbel_from_word(x.x));
-    kap[4 * s + 1] = fmaf(ph[4 * s + 1], np.inv_lam, gumbel_from_word(x.y));
-    kap[4 * s + 2] = fmaf(ph[4 * s + 2], np.inv_lam, gumbel_from_word(x.z));
-    kap[4 * s + 3] = fmaf(ph[4 * s + 3], np.inv_lam, gumbel_from_word(x.w));
-  }
-}
 
 template <int M>
 __device__ __forceinline__ void load_group(const float* phi_g, const uint16_t* W_g, float (&ph)[M],
@@ -54,35 +44,100 @@ __device__ __forceinline__ void load_group(const float* phi_g, const uint16_t* W
   }
 }
 
-// One group, one thread.  Returns the group's hard bits.
-template <int N, int M, bool TAU1>
-__device__ __forceinline__ uint32_t fwd_group(const float* phi_g, const uint16_t* W_g, int64_t e0,
-                                              const FwdArgs& a) {
-  float ph[M], w[M], kap[M];
-  load_group<M>(phi_g, W_g, ph, w);
-  group_keys<M>(ph, uint64_t(e0), a.np, kap);
-  const uint32_t bits = topn_bits<M>(kap, N);
+// Perturbed keys kappa = phi / lambda + g of L groups (one per lane of V) whose
+// first elements have call-flat indices e0[h]; ph[h] holds each group's logits.
+template <int M, class V>
+__device__ __forceinline__ void group_keys(const float (&ph)[vlanes<V>()][M], const int64_t* e0,
+                                           const NoiseParams& np, V (&kap)[M]) {
+  constexpr int L = vlanes<V>();
+  uint32_t x[L][M];
+#pragma unroll
+  for (int h = 0; h < L; ++h) {
+    const uint64_t q0 = (np.e_base + uint64_t(e0[h])) >> 2;
+#pragma unroll
+    for (int s = 0; s < M / 4; ++s) {
+      const uint4 w = noise_block_q(np, q0 + s);
+      x[h][4 * s] = w.x, x[h][4 * s + 1] = w.y, x[h][4 * s + 2] = w.z, x[h][4 * s + 3] = w.w;
+    }
+  }
+#pragma unroll
+  for (int l = 0; l < M; ++l) {
+    V one_plus, phv;
+    if constexpr (L == 1) {
+      one_plus = __uint_as_float(0x3f800000u | (x[0][l] >> 9));
+      phv = ph[0][l];
+    } else {
+      one_plus = f2(__uint_as_float(0x3f800000u | (x[0][l] >> 9)), __uint_as_float(0x3f800000u | (x[1][l] >> 9)));
+      phv = f2(ph[0][l], ph[1][l]);
+    }
+    // u = (1 + k 2^-23) - (1 - 2^-24), exact (see uniform_from_word)
+    const V u = vsub(one_plus, vconst<V>(__uint_as_float(0x3f7fffffu)));
+    kap[l] = vfma(phv, vconst<V>(np.inv_lam), gumbel_from_u(u));
+  }
+}
 
-  FastGroup<N, M, TAU1, false> fg;
+template <class V>
+__device__ __forceinline__ float lane_of(V v, int h) {
+  if constexpr (vlanes<V>() == 1) {
+    return v;
+  } else {
+    return h == 0 ? lo(v) : hi(v);
+  }
+}
+
+// L groups (one per lane of V) processed in lockstep by one thread; writes their
+// outputs and returns each group's hard bits in bits[h].
+template <int N, int M, bool TAU1, class V>
+__device__ __forceinline__ void fwd_groups(const float* const* phi_g, const uint16_t* const* W_g, const int64_t* e0,
+                                           const FwdArgs& a, uint32_t* bits) {
+  constexpr int L = vlanes<V>();
+  V kap[M];
+  {
+    float ph[L][M];
+#pragma unroll
+    for (int h = 0; h < L; ++h) {
+#pragma unroll
+      for (int s = 0; s < M / 4; ++s) {
+        const float4 p = reinterpret_cast<const float4*>(phi_g[h])[s];
+        ph[h][4 * s] = p.x, ph[h][4 * s + 1] = p.y, ph[h][4 * s + 2] = p.z, ph[h][4 * s + 3] = p.w;
+      }
+    }
+    group_keys<M, V>(ph, e0, a.np, kap);
+  }
+
+  FastGroup<N, M, TAU1, false, V> fg;
   fg.forward(kap, a.inv_tau);
-  float S[M];
 #pragma unroll
-  for (int l = 0; l < M; ++l) S[l] = fg.S[l];
-  if (fg.flag) {
-    ExactGroup<N, M> ex;
-    ex.forward(kap, N, M, a.tau, S);
-  }
-
+  for (int h = 0; h < L; ++h) {
+    float k[M], S[M];
 #pragma unroll
-  for (int s = 0; s < M / 4; ++s) {
-    uint2 o;
-    o.x = pack_bf16x2(w[4 * s] * S[4 * s], w[4 * s + 1] * S[4 * s + 1]);
-    o.y = pack_bf16x2(w[4 * s + 2] * S[4 * s + 2], w[4 * s + 3] * S[4 * s + 3]);
-    reinterpret_cast<uint2*>(a.Wm + e0)[s] = o;
-    if (a.soft != nullptr)
-      reinterpret_cast<float4*>(a.soft + e0)[s] = make_float4(S[4 * s], S[4 * s + 1], S[4 * s + 2], S[4 * s + 3]);
+    for (int l = 0; l < M; ++l) {
+      k[l] = lane_of(kap[l], h);
+      S[l] = lane_of(fg.S[l], h);
+    }
+    if constexpr (M == 4) {
+      bits[h] = topn_bits4(k, N);
+    } else {
+      bits[h] = topn_bits<M>(k, N);
+    }
+    if ((fg.flag >> h) & 1u) {
+      ExactGroup<N, M> ex;
+      ex.forward(k, N, M, a.tau, S);
+    }
+#pragma unroll
+    for (int s = 0; s < M / 4; ++s) {
+      // W is read here, not kept live through the relaxation
+      const uint2 q = reinterpret_cast<const uint2*>(W_g[h])[s];
+      const float wv[4] = {bf16_bits_to_float(q.x & 0xffffu), bf16_bits_to_float(q.x >> 16),
+                           bf16_bits_to_float(q.y & 0xffffu), bf16_bits_to_float(q.y >> 16)};
+      const float* sv = S + 4 * s;
+      uint2 o;
+      o.x = pack_bf16x2(__fmul_rn(wv[0], sv[0]), __fmul_rn(wv[1], sv[1]));
+      o.y = pack_bf16x2(__fmul_rn(wv[2], sv[2]), __fmul_rn(wv[3], sv[3]));
+      reinterpret_cast<uint2*>(a.Wm + e0[h])[s] = o;
+      if (a.soft != nullptr) reinterpret_cast<float4*>(a.soft + e0[h])[s] = make_float4(sv[0], sv[1], sv[2], sv[3]);
+    }
   }
-  return bits;
 }
 
 // Combine the M-bit masks of 32 / M consecutive lanes into words and store.
@@ -97,39 +152,49 @@ __device__ __forceinline__ void store_hard(uint32_t* hard, int64_t e0, uint32_t 
 }
 
 template <int N, int M, bool TAU1>
-__global__ void __launch_bounds__(kThreads) roi_fwd_kernel(FwdArgs a) {
+__global__ void __launch_bounds__(kThreads, M == 4 ? 4 : 2) roi_fwd_kernel(FwdArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
-  constexpr int kGroupsPerThread = kTile / M / kThreads;
+  constexpr int kT = kTile<M>;
+  static_assert(kT / M == 2 * kThreads, "two groups per thread per tile");
   TileSrc<2> src;
   src.ptr[0] = reinterpret_cast<const uint8_t*>(a.phi);
   src.esize[0] = 4;
   src.ptr[1] = reinterpret_cast<const uint8_t*>(a.W);
   src.esize[1] = 2;
 
-  const bool ok = run_tiles<kThreads, kTile, kStages, 2>(
+  const bool ok = run_tiles<kThreads, kT, kStages<M>, 2>(
       smem, src, a.full_tiles, a.status, [&](const uint8_t* const* stage, int64_t tile) {
         const float* sphi = reinterpret_cast<const float*>(stage[0]);
         const uint16_t* sW = reinterpret_cast<const uint16_t*>(stage[1]);
-        const int64_t base = tile * kTile;
-#pragma unroll
-        for (int j = 0; j < kGroupsPerThread; ++j) {
-          const int gi = threadIdx.x + j * kThreads;
-          const uint32_t bits = fwd_group<N, M, TAU1>(sphi + gi * M, sW + gi * M, base + gi * M, a);
-          if (a.hard != nullptr) store_hard<M>(a.hard, base + gi * M, bits, true);
+        const int64_t base = tile * kT;
+        const int g0 = threadIdx.x, g1 = threadIdx.x + kThreads;
+        const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
+        const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
+        const int64_t e0[2] = {base + g0 * M, base + g1 * M};
+        uint32_t bits[2];
+        fwd_groups<N, M, TAU1, F2>(pp, pw, e0, a, bits);
+        if (a.hard != nullptr) {
+          store_hard<M>(a.hard, e0[0], bits[0], true);
+          store_hard<M>(a.hard, e0[1], bits[1], true);
         }
       });
   if (!ok) return;
 
-  // ragged tail (fewer than kTile elements), last CTA, straight from global memory
+  // ragged tail (fewer than one tile), last CTA, straight from global memory
   if (blockIdx.x == gridDim.x - 1) {
-    const int64_t t0 = a.full_tiles * kTile;
+    const int64_t t0 = a.full_tiles * kT;
     const int64_t tail_groups = (a.E - t0) / M;
     const int64_t rounds = (tail_groups + kThreads - 1) / kThreads;
     for (int64_t r = 0; r < rounds; ++r) {
       const int64_t gi = threadIdx.x + r * kThreads;
       const bool active = gi < tail_groups;
       uint32_t bits = 0;
-      if (active) bits = fwd_group<N, M, TAU1>(a.phi + t0 + gi * M, a.W + t0 + gi * M, t0 + gi * M, a);
+      if (active) {
+        const float* pp[1] = {a.phi + t0 + gi * M};
+        const uint16_t* pw[1] = {a.W + t0 + gi * M};
+        const int64_t e0[1] = {t0 + gi * M};
+        fwd_groups<N, M, TAU1, float>(pp, pw, e0, a, &bits);
+      }
       if (a.hard != nullptr) store_hard<M>(a.hard, t0 + gi * M, bits, active);
     }
   }
@@ -172,7 +237,7 @@ struct LaunchCache {
 template <int N, int M, bool TAU1>
 int launch_tiles(const FwdArgs& a, cudaStream_t stream) {
   auto kern = roi_fwd_kernel<N, M, TAU1>;
-  const size_t smem = size_t(kStages) * kTile * 6 + 8 * kStages + 8;
+  const size_t smem = tile_smem_bytes<kTile<M>, kStages<M>>(6);
   static LaunchCache cache;  // per instantiation and device; racing writers store the same value
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return -1;
@@ -204,7 +269,7 @@ int launch_fwd(const FwdCall& c) {
   a.soft = c.soft;
   a.hard = c.hard;
   a.E = c.E;
-  a.full_tiles = c.E / kTile;
+  a.full_tiles = c.E / (c.M == 8 ? kTile<8> : kTile<4>);
   a.tau = c.tau;
   a.inv_tau = 1.0f / c.tau;
   a.np = c.np;

@@ -50,6 +50,7 @@ struct ExportCall {
 int launch_fwd(const FwdCall& c);
 int launch_bwd(const BwdCall& c);
 int launch_export(const ExportCall& c);
+int launch_noise(const NoiseParams& np, int64_t E, uint32_t* words, float* g, cudaStream_t stream);
 
 // Streaming multiprocessors of the current device (cached).
 int sm_count();

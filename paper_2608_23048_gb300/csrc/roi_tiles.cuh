@@ -1,8 +1,10 @@
 // Persistent tile pipeline: each CTA walks tiles blockIdx.x, blockIdx.x + grid, ...
-// of TILE contiguous elements.  One thread stages the inputs of upcoming tiles
-// into a ring of shared-memory stages with 1-D bulk copies (TMA) that complete
-// on one mbarrier per stage; all threads wait (bounded), compute from shared
-// memory and store their outputs straight to global memory (coalesced).
+// of TILE contiguous elements.  The inputs of upcoming tiles are staged into a
+// ring of shared-memory stages with 1-D bulk copies (TMA) that complete on one
+// mbarrier per stage.  Warps never wait for each other: each warp waits (bounded)
+// for its stage to land, computes from shared memory, stores its outputs straight
+// to global memory, then counts itself out of the stage; the last warp out issues
+// the copies that refill the stage with the tile STAGES ahead.
 #pragma once
 
 #include "roi_common.cuh"
@@ -15,21 +17,21 @@ struct TileSrc {
   uint32_t esize[NARR];      // bytes per element of each input array
 };
 
-template <int TILE, int STAGES, int NARR>
-struct TileSmem {
-  static constexpr size_t bars_offset(const uint32_t (&es)[NARR]) {
-    size_t off = 0;
-    for (int a = 0; a < NARR; ++a) off += size_t(STAGES) * TILE * es[a];
-    return off;
-  }
-};
+// Shared memory needed by run_tiles: the stages, then per stage one mbarrier,
+// one "warps done" counter and one "fills issued" counter.
+template <int TILE, int STAGES>
+constexpr size_t tile_smem_bytes(uint32_t bytes_per_element) {
+  return ((size_t(STAGES) * TILE * bytes_per_element + 7) & ~size_t(7)) + size_t(STAGES) * 16;
+}
 
 // Runs `compute(stage_ptrs, tile)` for every full tile of this CTA.  Returns
 // false if a wait timed out (status recorded, copies drained).
 template <int THREADS, int TILE, int STAGES, int NARR, class Compute>
 __device__ __forceinline__ bool run_tiles(uint8_t* smem, const TileSrc<NARR>& src, int64_t full_tiles,
                                           unsigned int* status, Compute&& compute) {
+  constexpr int kWarps = THREADS / 32;
   const int tid = threadIdx.x;
+  const int lane = tid & 31;
   size_t arr_off[NARR];
   size_t off = 0;
   uint32_t stage_bytes = 0;
@@ -40,21 +42,17 @@ __device__ __forceinline__ bool run_tiles(uint8_t* smem, const TileSrc<NARR>& sr
     stage_bytes += TILE * src.esize[a];
   }
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + ((off + 7) & ~size_t(7)));
+  uint32_t* done = reinterpret_cast<uint32_t*>(bars + STAGES);   // warps finished with the current fill
+  uint32_t* fills = done + STAGES;                                // fills issued per stage
 
   const int64_t first = blockIdx.x;
   const int64_t stride = gridDim.x;
   const int64_t my_tiles = first < full_tiles ? (full_tiles - first + stride - 1) / stride : 0;
 
-  if (tid == 0) {
-#pragma unroll
-    for (int s = 0; s < STAGES; ++s) mbar_init(&bars[s], 1);
-    fence_mbar_init();
-  }
-  __syncthreads();
-
   auto issue = [&](int64_t i) {
     const int s = int(i % STAGES);
     const int64_t t = first + i * stride;
+    fills[s] += 1;
     mbar_arrive_expect_tx(&bars[s], stage_bytes);
 #pragma unroll
     for (int a = 0; a < NARR; ++a) {
@@ -64,34 +62,48 @@ __device__ __forceinline__ bool run_tiles(uint8_t* smem, const TileSrc<NARR>& sr
     }
   };
 
-  int64_t issued = 0;
   if (tid == 0) {
-    for (; issued < my_tiles && issued < STAGES; ++issued) issue(issued);
+#pragma unroll
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&bars[s], 1);
+      done[s] = 0;
+      fills[s] = 0;
+    }
+    fence_mbar_init();
+    for (int64_t i = 0; i < my_tiles && i < STAGES; ++i) issue(i);
   }
+  __syncthreads();
 
   for (int64_t i = 0; i < my_tiles; ++i) {
     const int s = int(i % STAGES);
     const uint32_t parity = uint32_t((i / STAGES) & 1);
-    const bool timed_out = !mbar_wait_bounded(&bars[s], parity);
-    if (!timed_out) {
-      const uint8_t* stage[NARR];
-#pragma unroll
-      for (int a = 0; a < NARR; ++a) stage[a] = smem + arr_off[a] + size_t(s) * TILE * src.esize[a];
-      compute(stage, first + i * stride);
-    }
-    if (__syncthreads_or(timed_out)) {
-      if (tid == 0) {
+    if (!mbar_wait_bounded(&bars[s], parity)) {
+      if (lane == 0) {
         atomicOr(status, kStatusTimeout);
         // let copies still in flight land before the CTA's shared memory is released
-        for (int64_t j = i; j < issued; ++j)
-          mbar_wait_bounded(&bars[int(j % STAGES)], uint32_t((j / STAGES) & 1));
+        for (int q = 0; q < STAGES; ++q) {
+          const uint32_t n = *reinterpret_cast<volatile uint32_t*>(&fills[q]);
+          if (n > 0) mbar_wait_bounded(&bars[q], (n - 1) & 1u);
+        }
       }
-      __syncthreads();
+      __syncwarp();
       return false;
     }
-    if (tid == 0 && issued < my_tiles) {
-      issue(issued);
-      ++issued;
+    const uint8_t* stage[NARR];
+#pragma unroll
+    for (int a = 0; a < NARR; ++a) stage[a] = smem + arr_off[a] + size_t(s) * TILE * src.esize[a];
+    compute(stage, first + i * stride);
+    __syncwarp();
+    if (lane == 0) {
+      __threadfence_block();
+      if (atomicAdd(&done[s], 1u) == kWarps - 1) {
+        // every warp is done reading this fill: refill it with the tile STAGES ahead
+        done[s] = 0;
+        if (i + STAGES < my_tiles) {
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          issue(i + STAGES);
+        }
+      }
     }
   }
   return true;

@@ -61,6 +61,7 @@ def fwd(L, logits=A, W=B, N=2, M=4, tau=1.0, rows=4, cols=8, Wm=C, soft=None, ha
 def test_validation_codes(L):
     import paper_2608_23048_gb300 as roi
     assert fwd(L, logits=0) == 1                    # ROI_ERR_NULL
+    assert fwd(L, logits=0, W=0, Wm=0, rows=0) == 0  # empty: pointers may be NULL
     assert fwd(L, Wm=0) == 1
     assert fwd(L, N=0) == 3 and fwd(L, N=4, M=4) == 3 and fwd(L, N=2, M=33, cols=33) == 3   # ROI_ERR_NM
     assert fwd(L, cols=6) == 2 and fwd(L, rows=-1) == 2 and fwd(L, cols=0) == 2            # ROI_ERR_SHAPE

@@ -76,10 +76,12 @@ def check_against_oracle(got, phi, Wb, dWb, N, M, tau, seed, step, tid, lam, row
     Wabs = np.abs(O.bf16_to_f32(Wb).astype(np.float64)).ravel()
     dWabs = np.abs(O.bf16_to_f32(dWb).astype(np.float64)).ravel()
     if "soft" in got:
-        # the library's bf16 outputs are exactly bf16_rne(fp32(x * S)) of its own S
+        # Wm is exactly bf16_rne(fp32(W * S)) of the forward's own S; the backward
+        # recomputes S in another kernel, where the compiler may fuse packed products
+        # into FMAs differently, so dW agrees with bf16(dWm * S_fwd) to one bf16 ulp
         assert np.array_equal(got["Wm"].ravel(), O.bf16_product(Wb.ravel(), got["soft"].ravel())), "Wm != bf16(W*S)"
         if "dW" in got:
-            assert np.array_equal(got["dW"].ravel(), O.bf16_product(dWb.ravel(), got["soft"].ravel()))
+            assert C.bf16_violations(got["dW"].ravel(), O.bf16_product(dWb.ravel(), got["soft"].ravel())) == 0
     for ref, tag in ((f64, "f64"), (f32, "f32")):
         if "soft" in got:
             n, worst = C.soft_violations(got["soft"], ref["soft"], keys, N, M, tau)
@@ -290,3 +292,29 @@ def test_launches_are_counted(roi):
     W, phi, dWm, *_ = make(4, 64, "normal")
     gpu_run(roi, phi, W, dWm, 2, 4, 1.0, roi.NoiseState(0, 0, 0, 1.0, 0))
     assert roi.roi_launch_count() >= before + 2
+
+
+def test_noise_words_bit_exact(roi):
+    """The library's Philox-4x32-10 stream equals the oracle's, word for word."""
+    import torch
+    rows, cols, r0 = 37, 1000, 3
+    st = roi.NoiseState(2 ** 33 + 7, 11, 5, 1.0, r0)
+    out = torch.empty(rows * cols, dtype=torch.int32, device="cuda")
+    roi.roi_noise_words(st, rows, cols, out)
+    torch.cuda.synchronize()
+    want = O.noise_words(2 ** 33 + 7, 11, 5, O.element_indices(rows, cols, r0))
+    assert np.array_equal(out.cpu().numpy().view(np.uint32), want)
+
+
+def test_gumbel_noise_error_bound(roi):
+    """g = -log(-log u) as the kernels form it: within 5e-7 + 2^-22 |g| of float64."""
+    import torch
+    rows, cols = 2048, 4096
+    st = roi.NoiseState(99, 1, 0, 1.0, 0)
+    out = torch.empty(rows * cols, dtype=torch.float32, device="cuda")
+    roi.roi_gumbel_noise(st, rows, cols, out)
+    torch.cuda.synchronize()
+    g = out.cpu().numpy().astype(np.float64)
+    want = O.gumbel_noise(99, 1, 0, rows, cols)
+    err = np.abs(g - want)
+    assert np.all(err <= 5e-7 + 2.0 ** -22 * np.abs(want)), float(np.max(err))
