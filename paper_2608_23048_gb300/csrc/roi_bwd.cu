@@ -71,11 +71,11 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
     for (int l = 0; l < M; ++l) {
       V one_plus, phv, wv, dwv;
       if constexpr (L == 1) {
-        one_plus = __uint_as_float(0x3f800000u | (x[0][l] >> 9));
+        one_plus = one_plus_from_word(x[0][l]);
         phv = ph[0][l], wv = w[0][l], dwv = dw[0][l];
       } else {
         one_plus =
-            f2(__uint_as_float(0x3f800000u | (x[0][l] >> 9)), __uint_as_float(0x3f800000u | (x[1][l] >> 9)));
+            f2(one_plus_from_word(x[0][l]), one_plus_from_word(x[1][l]));
         phv = f2(ph[0][l], ph[1][l]), wv = f2(w[0][l], w[1][l]), dwv = f2(dw[0][l], dw[1][l]);
       }
       const V u = vsub(one_plus, vconst<V>(__uint_as_float(0x3f7fffffu)));
@@ -162,7 +162,13 @@ __global__ void __launch_bounds__(kThreads, M == 4 ? 4 : 2) roi_bwd_kernel(BwdAr
         const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
         const uint16_t* pd[2] = {sdW + g0 * M, sdW + g1 * M};
         const int64_t e0[2] = {base + g0 * M, base + g1 * M};
-        bwd_groups<N, M, TAU1, F2>(pp, pw, pd, e0, a);
+        if constexpr (M == 4) {
+          bwd_groups<N, M, TAU1, F2>(pp, pw, pd, e0, a);
+        } else {
+          // M = 8: the paired step history does not fit the register file; one group at a time
+#pragma unroll 1
+          for (int h = 0; h < 2; ++h) bwd_groups<N, M, TAU1, float>(pp + h, pw + h, pd + h, e0 + h, a);
+        }
       });
   if (!ok) return;
 

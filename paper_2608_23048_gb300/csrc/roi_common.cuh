@@ -100,10 +100,15 @@ __device__ __forceinline__ uint32_t noise_word(const NoiseParams& np, uint64_t e
   return s == 0 ? w.x : s == 1 ? w.y : s == 2 ? w.z : w.w;
 }
 
+// The bits of 1 + k 2^-23 with k = x >> 9: (x >> 9) | 0x3f800000 is one funnel
+// shift of the 64-bit pair {127 : x} right by 9 (127 << 23 == 0x3f800000).
+__device__ __forceinline__ float one_plus_from_word(uint32_t x) {
+  return __uint_as_float(__funnelshift_r(x, 127u, 9));
+}
 // u = ((x >> 9) + 1/2) * 2^-23, exactly: (1 + k 2^-23) - (1 - 2^-24) is exact
 // by Sterbenz's lemma and equals (2k + 1) 2^-24.
 __device__ __forceinline__ float uniform_from_word(uint32_t x) {
-  return __uint_as_float(0x3f800000u | (x >> 9)) - __uint_as_float(0x3f7fffffu);
+  return __fsub_rn(one_plus_from_word(x), __uint_as_float(0x3f7fffffu));
 }
 
 // E = -ln(u) for u in [2^-24, 1) with a small relative error everywhere,
@@ -359,6 +364,7 @@ struct FastGroup {
   // mu on demand, in the same order, instead of being kept live).
   V mu[KEEP ? N : 1][M];
   V S[KEEP ? 1 : M];
+  V rt_last;  // tau = 1, KEEP: 1 / sum(mu om) of step N-2 (mu(N-1) = mu(N-2) om rt_last)
   uint32_t flag;
 
   // S_l of a KEEP run, summed exactly as forward() accumulates it.
@@ -400,6 +406,9 @@ struct FastGroup {
 #pragma unroll
           for (int l = 0; l < M; ++l) v[l] = vmul(cur[l], o[l]);
           const V rt = vmap(sum_of(v), rcp_approx);
+          if constexpr (KEEP) {
+            if (k == N - 2) rt_last = rt;
+          }
 #pragma unroll
           for (int l = 0; l < M; ++l) cur[l] = vmul(v[l], rt);
         }
@@ -448,24 +457,34 @@ struct FastGroup {
   __device__ __forceinline__ void backward(const V (&c)[M], float inv_tau, V (&dk)[M]) const {
     static_assert(KEEP, "backward needs the stored steps");
     const V itau = vconst<V>(inv_tau);
-    V b[M];
+    V b[M], hl[M];
     {
       V cm[M];
 #pragma unroll
       for (int l = 0; l < M; ++l) cm[l] = vmul(c[l], mu[N - 1][l]);
       const V cmu = sum_of(cm);
 #pragma unroll
-      for (int l = 0; l < M; ++l) b[l] = vmul(vmul(mu[N - 1][l], itau), vsub(c[l], cmu));
+      for (int l = 0; l < M; ++l) {
+        const V t = vmul(itau, vsub(c[l], cmu));
+        b[l] = vmul(mu[N - 1][l], t);
+        // tau = 1: b / om(N-2) = mu(N-2) rt_last (c - <c, mu(N-1)>) / tau, no division
+        if constexpr (TAU1 && N >= 2) hl[l] = vmul(vmul(mu[N - 2][l], rt_last), t);
+      }
     }
 #pragma unroll
     for (int k = N - 2; k >= 0; --k) {
-      V cm[M], h[M], H[M], om[M];
-      exclusive_sums(mu[k], om);
+      V cm[M], h[M], H[M];
+      if (!TAU1 || k != N - 2) {
+        V om[M];
+        exclusive_sums(mu[k], om);
 #pragma unroll
-      for (int l = 0; l < M; ++l) {
-        cm[l] = vmul(c[l], mu[k][l]);
-        h[l] = vmul(b[l], vmap(om[l], rcp_approx));
+        for (int l = 0; l < M; ++l) h[l] = vmul(b[l], vmap(om[l], rcp_approx));
+      } else {
+#pragma unroll
+        for (int l = 0; l < M; ++l) h[l] = hl[l];
       }
+#pragma unroll
+      for (int l = 0; l < M; ++l) cm[l] = vmul(c[l], mu[k][l]);
       const V cmu = sum_of(cm);
       const V B = sum_of(b);
       exclusive_sums(h, H);

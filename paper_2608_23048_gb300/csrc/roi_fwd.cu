@@ -64,10 +64,10 @@ __device__ __forceinline__ void group_keys(const float (&ph)[vlanes<V>()][M], co
   for (int l = 0; l < M; ++l) {
     V one_plus, phv;
     if constexpr (L == 1) {
-      one_plus = __uint_as_float(0x3f800000u | (x[0][l] >> 9));
+      one_plus = one_plus_from_word(x[0][l]);
       phv = ph[0][l];
     } else {
-      one_plus = f2(__uint_as_float(0x3f800000u | (x[0][l] >> 9)), __uint_as_float(0x3f800000u | (x[1][l] >> 9)));
+      one_plus = f2(one_plus_from_word(x[0][l]), one_plus_from_word(x[1][l]));
       phv = f2(ph[0][l], ph[1][l]);
     }
     // u = (1 + k 2^-23) - (1 - 2^-24), exact (see uniform_from_word)
