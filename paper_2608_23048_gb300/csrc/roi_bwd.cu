@@ -254,6 +254,7 @@ int launch_bwd(const BwdCall& c) {
   if (c.N == 2 && c.M == 4) return launch_nm<2, 4>(a, c.stream);
   if (c.N == 4 && c.M == 8) return launch_nm<4, 8>(a, c.stream);
   if (c.N == 2 && c.M == 8) return launch_nm<2, 8>(a, c.stream);
+  if (slice_supported(c.N, c.M)) return launch_slice_bwd(c);
   const int64_t groups = c.E / c.M;
   int64_t blocks = (groups + 127) / 128;
   const int64_t cap = int64_t(sm_count()) * 16;

@@ -255,8 +255,18 @@ struct ExactGroup {
       for (int l = 0; l < M; ++l) S[l] = __fadd_rn(S[l], expf(__fsub_rn(z[l], lt)));
       if (k + 1 < N) {
         float zn[MMAX];
-        for (int l = 0; l < M; ++l) zn[l] = __fadd_rn(z[l], __fdiv_rn(__fsub_rn(lse_excluding(z, M, l), lt), tau));
-        for (int l = 0; l < M; ++l) z[l] = zn[l];
+        float zmax = -INFINITY;
+        for (int l = 0; l < M; ++l) {
+          zn[l] = __fadd_rn(z[l], __fdiv_rn(__fsub_rn(lse_excluding(z, M, l), lt), tau));
+          zmax = fmaxf(zmax, zn[l]);
+        }
+        // shift so the largest key is 0 (softmax and log(1 - mu) are shift-invariant):
+        // keeps the rounding of the keys that matter small over many steps
+        if (zmax > -INFINITY && zmax < INFINITY) {
+          for (int l = 0; l < M; ++l) z[l] = __fsub_rn(zn[l], zmax);
+        } else {
+          for (int l = 0; l < M; ++l) z[l] = zn[l];
+        }
       }
     }
   }

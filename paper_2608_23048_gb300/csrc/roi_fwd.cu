@@ -277,6 +277,7 @@ int launch_fwd(const FwdCall& c) {
   if (c.N == 2 && c.M == 4) return launch_nm<2, 4>(a, c.stream);
   if (c.N == 4 && c.M == 8) return launch_nm<4, 8>(a, c.stream);
   if (c.N == 2 && c.M == 8) return launch_nm<2, 8>(a, c.stream);
+  if (slice_supported(c.N, c.M)) return launch_slice_fwd(c);
   // generic path
   int launched = 0;
   if (c.hard != nullptr) {

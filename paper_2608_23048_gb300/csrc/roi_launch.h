@@ -50,6 +50,10 @@ struct ExportCall {
 int launch_fwd(const FwdCall& c);
 int launch_bwd(const BwdCall& c);
 int launch_export(const ExportCall& c);
+// Warp-slice kernels for M = 16, 32 (roi_slice.cu).
+bool slice_supported(int N, int M);
+int launch_slice_fwd(const FwdCall& c);
+int launch_slice_bwd(const BwdCall& c);
 int launch_noise(const NoiseParams& np, int64_t E, uint32_t* words, float* g, cudaStream_t stream);
 
 // Streaming multiprocessors of the current device (cached).

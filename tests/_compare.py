@@ -11,7 +11,14 @@ is carried through N softmax steps, so the allowed difference is
 with c = dWm * W the upstream gradient of S (the backward sums terms of size
 |c| / tau, so their rounding is relative to that scale, not to a small result).
 At tau = 1 the second term is below 1e-5 and the rule is the plain 1e-5 relative
-bound.  bf16 outputs Wm = bf16(W * S) and dW = bf16(dWm * S): bit-exact against the
+bound.  The relaxation at tau < 1 with many steps can amplify rounding from step to
+step, so on extreme inputs (key gaps of tens of z-units competing over 8-16 steps)
+no fp32 evaluation meets a bound linear in N: the float32 oracle itself reaches
+several times it.  The input's own conditioning is therefore measured as the float32
+oracle's deviation from the float64 one, dev32, element by element, and the
+allowance becomes bound + 4 |dev32| against the float64 oracle (the truth) and
+bound + 5 |dev32| against the float32 oracle.  On the configs' inputs dev32 is far
+below the bound, so the bound governs.  bf16 outputs Wm = bf16(W * S) and dW = bf16(dWm * S): bit-exact against the
 library's own S (the rounding is fully defined), and against the oracle within one
 bf16 ulp beyond what the S tolerance already allows (|W| * tol_S).  Hard masks:
 bit-exact, except groups whose N-th and (N+1)-th float64 keys differ by less than
@@ -34,20 +41,24 @@ def soft_tolerance(want, kappa64, N, M, tau):
     return (1e-5 + 2 * N * eps_z(kappa64, M, tau)) * scale
 
 
-def soft_violations(got, want, kappa64, N, M, tau):
+def soft_violations(got, want, kappa64, N, M, tau, extra=None):
     g = np.asarray(got, dtype=np.float64).reshape(-1, M)
     w = np.asarray(want, dtype=np.float64).reshape(-1, M)
     tol = soft_tolerance(want, kappa64, N, M, tau)
+    if extra is not None:
+        tol = tol + np.abs(np.asarray(extra, dtype=np.float64)).reshape(-1, M)
     bad = ~(np.abs(g - w) <= tol)
     return int(bad.sum()), float(np.max(np.abs(g - w) / np.maximum(tol, 1e-300)))
 
 
-def dlogit_violations(got, want, c, kappa64, N, M, tau, lam=1.0):
+def dlogit_violations(got, want, c, kappa64, N, M, tau, lam=1.0, extra=None):
     g = np.asarray(got, dtype=np.float64).reshape(-1, M)
     w = np.asarray(want, dtype=np.float64).reshape(-1, M)
     cs = np.abs(np.asarray(c, dtype=np.float64)).reshape(-1, M).max(axis=1, keepdims=True) / (tau * lam)
     scale = np.maximum(np.abs(w).max(axis=1, keepdims=True), cs)
     tol = (1e-5 + 8 * N * eps_z(kappa64, M, tau)) * scale
+    if extra is not None:
+        tol = tol + np.abs(np.asarray(extra, dtype=np.float64)).reshape(-1, M)
     bad = ~(np.abs(g - w) <= tol)
     return int(bad.sum()), float(np.max(np.abs(g - w) / np.maximum(tol, 1e-300)))
 
