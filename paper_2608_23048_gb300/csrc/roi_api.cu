@@ -64,6 +64,7 @@ NoiseParams make_noise(const roi_noise_state& st, int64_t cols) {
   np.step = st.step;
   np.tensor_id = st.tensor_id;
   np.inv_lam = 1.0f / st.lambda;
+  np.l2e_inv_lam = static_cast<float>(1.4426950408889634 / static_cast<double>(st.lambda));
   np.e_base = static_cast<uint64_t>(st.row_offset) * static_cast<uint64_t>(cols);
   return np;
 }

@@ -79,7 +79,7 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
         phv = f2(ph[0][l], ph[1][l]), wv = f2(w[0][l], w[1][l]), dwv = f2(dw[0][l], dw[1][l]);
       }
       const V u = vsub(one_plus, vconst<V>(__uint_as_float(0x3f7fffffu)));
-      kap[l] = vfma(phv, vconst<V>(a.np.inv_lam), gumbel_from_u(u));
+      kap[l] = key_log2(phv, u, a.np.l2e_inv_lam);  // log2 units
       c[l] = vmul(dwv, wv);
     }
   }
@@ -112,7 +112,7 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
       float k[M], cc[M], S[M];
 #pragma unroll
       for (int l = 0; l < M; ++l) {
-        k[l] = lane_of(kap[l], h);
+        k[l] = lane_of(kap[l], h) * kLn2;  // natural-log keys
         cc[l] = lane_of(c[l], h);
       }
       ExactGroup<N, M> ex;

@@ -82,6 +82,7 @@ struct NoiseParams {
   uint32_t k0, k1;       // seed words
   uint32_t step, tensor_id;
   float inv_lam;         // 1 / lambda
+  float l2e_inv_lam;     // log2(e) / lambda: keys in log2 units, t = phi log2(e) / lambda - log2(E)
   uint64_t e_base;       // row_offset * cols: flat index of this call's element 0
 };
 
@@ -113,30 +114,23 @@ __device__ __forceinline__ float uniform_from_word(uint32_t x) {
 
 // E = -ln(u) for u in [2^-24, 1) with a small relative error everywhere,
 // including u -> 1 where E -> 0 (the hardware log2 has an absolute error floor
-// there).  Method: u = 2^e m with m in [sqrt(1/2), sqrt(2)), so
-// ln u = e ln2 + ln m and ln m = 2 atanh(s), s = (m - 1) / (m + 1), |s| < 0.1716,
+// there).  Method: u = 2^e m with e = rint(log2 u) and m = u 2^-e in
+// [sqrt(1/2), sqrt(2)], so ln u = e ln2 + ln m; ln m = 2 atanh(s),
+// s = (m - 1) / (m + 1), |s| < 0.172,
 // 2 atanh(s) = 2s + (2/3)s^3 + (2/5)s^5 + (2/7)s^7 + (2/9)s^9 + O(s^11)
-// (truncation below 2^-28 relative).  m - 1 is exact (Sterbenz).  The Horner
+// (truncation below 2^-28 relative).  e comes from the hardware log2 rounded to
+// the nearest integer (its error only moves m across the boundary of the
+// interval when log2 u is within 2^-22 of a half-integer, which the series
+// tolerates); 2^-e from the hardware exp2, exact on integers (verified on the
+// GPU for all integers in [-100, 127]); m - 1 is exact (Sterbenz).  The Horner
 // chain runs on negated coefficients so the result needs no final negation.
-__device__ __forceinline__ void unit_split(float u, float& m, float& ef) {
-  const uint32_t b = __float_as_uint(u);
-  const int32_t e = int32_t(b - 0x3f3504f3u) >> 23;  // 0x3f3504f3 = sqrt(1/2)
-  m = __uint_as_float(b - (uint32_t(e) << 23));
-  // e in [-25, 0] -> float without a conversion instruction (1.5 * 2^23 trick)
-  ef = __int_as_float(0x4b400000 + e) - 12582912.0f;
-}
 template <class V>
 __device__ __forceinline__ V neg_log_unit(V u) {
-  V m, ef;
-  if constexpr (vlanes<V>() == 1) {
-    unit_split(u, m, ef);
-  } else {
-    float m0, m1, e0, e1;
-    unit_split(lo(u), m0, e0);
-    unit_split(hi(u), m1, e1);
-    m = f2(m0, m1);
-    ef = f2(e0, e1);
-  }
+  const V y = vmap(u, lg2_approx);
+  const V tt = vadd(y, vconst<V>(12582912.0f));               // 1.5 * 2^23: rounds y to an integer
+  const V ef = vsub(tt, vconst<V>(12582912.0f));              // e = rint(log2 u)
+  const V p2 = vmap(vsub(vconst<V>(12582912.0f), tt), ex2_approx);  // 2^-e, exact
+  const V m = vmul(u, p2);                                     // exact power-of-two scaling
   const V one = vconst<V>(1.0f);
   const V f = vsub(m, one);
   const V s = vmul(f, vmap(vadd(m, one), rcp_approx));
@@ -148,12 +142,24 @@ __device__ __forceinline__ V neg_log_unit(V u) {
   return vfma(ef, vconst<V>(-kLn2), nlnm);
 }
 
-// Gumbel(0,1) samples from words: g = -log(-log u) (Algorithm 1).  The outer
-// log only needs absolute accuracy (g enters the keys additively) and uses the
+// log2 of E = -ln u.  The keys the fast kernels rank and relax are kept in log2
+// units, t = kappa log2(e) = phi log2(e) / lambda - log2(E) (Eq. 10 with
+// g = -ln E), so exp2 of key differences needs no further scaling.  The outer
+// log only needs absolute accuracy (it enters the key additively) and uses the
 // hardware log2.
 template <class V>
+__device__ __forceinline__ V log2_neg_log_unit(V u) {
+  return vmap(neg_log_unit(u), lg2_approx);
+}
+// Key in log2 units from the logit and the uniform.
+template <class V>
+__device__ __forceinline__ V key_log2(V phi, V u, float l2e_inv_lam) {
+  return vsub(vmul(phi, vconst<V>(l2e_inv_lam)), log2_neg_log_unit(u));
+}
+// Gumbel(0,1) sample g = -log(-log u) (Algorithm 1) in natural units.
+template <class V>
 __device__ __forceinline__ V gumbel_from_u(V u) {
-  return vmul(vmap(neg_log_unit(u), lg2_approx), vconst<V>(-kLn2));
+  return vmul(log2_neg_log_unit(u), vconst<V>(-kLn2));
 }
 __device__ __forceinline__ float gumbel_from_word(uint32_t x) {
   return gumbel_from_u(uniform_from_word(x));
@@ -385,18 +391,26 @@ struct FastGroup {
     return s;
   }
 
+  // kap: the keys in log2 units (t = kappa log2 e).
   __device__ __forceinline__ void forward(const V (&kap)[M], float inv_tau) {
     V cur[M];
     flag = 0;
     if constexpr (TAU1) {
       // Weights relative to the group's first key (any reference works: they are
-      // normalised next); a group whose weights leave [2^-100, 2^100] (a key gap
-      // of ~69), or that holds a non-finite key, goes to the exact routine.
-      V e[M];
+      // normalised next).  A group with a key more than 100 (log2 units, ~69
+      // natural) from the first one, or with a non-finite key, goes to the exact
+      // routine: the squared offsets are summed on the FMA pipe and compared once.
+      V e[M], x[M];
 #pragma unroll
-      for (int l = 0; l < M; ++l) e[l] = vmap(vmul(vsub(kap[l], kap[0]), vconst<V>(kLog2e)), ex2_approx);
+      for (int l = 0; l < M; ++l) {
+        x[l] = vsub(kap[l], kap[0]);
+        e[l] = vmap(x[l], ex2_approx);
+      }
+      V sq = vmul(x[1], x[1]);
+#pragma unroll
+      for (int l = 2; l < M; ++l) sq = vfma(x[l], x[l], sq);
+      flag = vbelow(vsub(vconst<V>(1.0e4f), sq), 0.0f);
       const V tot = sum_of(e);
-      flag = vbelow(min_of(e), kTinyExcl) | vbelow(vsub(vconst<V>(1.0f / kTinyExcl), tot), 0.0f);
       const V r = vmap(tot, rcp_approx);
 #pragma unroll
       for (int l = 0; l < M; ++l) cur[l] = vmul(e[l], r);
@@ -425,7 +439,7 @@ struct FastGroup {
       }
     } else {
       const V kmax = max_of(kap);
-      const V sc = vconst<V>(inv_tau * kLog2e);
+      const V sc = vconst<V>(inv_tau);
       const V itau = vconst<V>(inv_tau);
       V d[M];
 #pragma unroll

@@ -44,8 +44,9 @@ __device__ __forceinline__ void load_group(const float* phi_g, const uint16_t* W
   }
 }
 
-// Perturbed keys kappa = phi / lambda + g of L groups (one per lane of V) whose
-// first elements have call-flat indices e0[h]; ph[h] holds each group's logits.
+// Perturbed keys of L groups (one per lane of V), in log2 units
+// (t = (phi / lambda + g) log2 e), whose first elements have call-flat indices
+// e0[h]; ph[h] holds each group's logits.
 template <int M, class V>
 __device__ __forceinline__ void group_keys(const float (&ph)[vlanes<V>()][M], const int64_t* e0,
                                            const NoiseParams& np, V (&kap)[M]) {
@@ -72,7 +73,7 @@ __device__ __forceinline__ void group_keys(const float (&ph)[vlanes<V>()][M], co
     }
     // u = (1 + k 2^-23) - (1 - 2^-24), exact (see uniform_from_word)
     const V u = vsub(one_plus, vconst<V>(__uint_as_float(0x3f7fffffu)));
-    kap[l] = vfma(phv, vconst<V>(np.inv_lam), gumbel_from_u(u));
+    kap[l] = key_log2(phv, u, np.l2e_inv_lam);
   }
 }
 
@@ -115,14 +116,18 @@ __device__ __forceinline__ void fwd_groups(const float* const* phi_g, const uint
       k[l] = lane_of(kap[l], h);
       S[l] = lane_of(fg.S[l], h);
     }
+    // ranking the log2-unit keys ranks kappa
     if constexpr (M == 4) {
       bits[h] = topn_bits4(k, N);
     } else {
       bits[h] = topn_bits<M>(k, N);
     }
     if ((fg.flag >> h) & 1u) {
+      float kn[M];
+#pragma unroll
+      for (int l = 0; l < M; ++l) kn[l] = k[l] * kLn2;  // natural-log keys
       ExactGroup<N, M> ex;
-      ex.forward(k, N, M, a.tau, S);
+      ex.forward(kn, N, M, a.tau, S);
     }
 #pragma unroll
     for (int s = 0; s < M / 4; ++s) {

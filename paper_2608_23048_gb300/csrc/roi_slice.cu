@@ -79,14 +79,15 @@ struct SliceArgs {
   unsigned int* status;
 };
 
-// Keys of one four-element slot starting at call-flat index e0.
+// Keys of one four-element slot starting at call-flat index e0, in log2 units
+// (t = kappa log2 e).
 __device__ __forceinline__ void slot_keys(const float* phi4, int64_t e0, const NoiseParams& np, float (&kap)[4]) {
   const float4 p = *reinterpret_cast<const float4*>(phi4);
   const uint4 x = noise_block_q(np, (np.e_base + uint64_t(e0)) >> 2);
-  kap[0] = fmaf(p.x, np.inv_lam, gumbel_from_word(x.x));
-  kap[1] = fmaf(p.y, np.inv_lam, gumbel_from_word(x.y));
-  kap[2] = fmaf(p.z, np.inv_lam, gumbel_from_word(x.z));
-  kap[3] = fmaf(p.w, np.inv_lam, gumbel_from_word(x.w));
+  kap[0] = key_log2(p.x, uniform_from_word(x.x), np.l2e_inv_lam);
+  kap[1] = key_log2(p.y, uniform_from_word(x.y), np.l2e_inv_lam);
+  kap[2] = key_log2(p.z, uniform_from_word(x.z), np.l2e_inv_lam);
+  kap[3] = key_log2(p.w, uniform_from_word(x.w), np.l2e_inv_lam);
 }
 
 // Forward relaxation of the group held by this slice; mu of every step kept if
@@ -105,7 +106,7 @@ struct SliceRelax {
       const float kref = __shfl_sync(0xffffffffu, kap[0], base_lane);
       float e[4];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) e[j] = ex2_approx(__fmul_rn(__fsub_rn(kap[j], kref), kLog2e));
+      for (int j = 0; j < 4; ++j) e[j] = ex2_approx(__fsub_rn(kap[j], kref));
       float tot;
       Slice<SL>::others(sum4(e), tot);
       flag = (!(min4(e) >= kTinyExcl) || !(tot <= 1.0f / kTinyExcl)) ? 1u : 0u;
@@ -133,7 +134,7 @@ struct SliceRelax {
       }
     } else {
       const float kmax = Slice<SL>::max(max4(kap));
-      const float sc = inv_tau * kLog2e;
+      const float sc = inv_tau;
       float d[4];
 #pragma unroll
       for (int j = 0; j < 4; ++j) d[j] = __fmul_rn(__fsub_rn(kap[j], kmax), sc);
@@ -238,8 +239,8 @@ __device__ __forceinline__ uint32_t slice_topn_bits(const float (&kap)[4], int N
   return bits;
 }
 
-// Exact fallback for the whole group, run by one lane: keys of all M elements
-// from logits at phi_g (call-flat index g0).
+// Exact fallback for the whole group, run by one lane: natural-log keys of all
+// M elements from logits at phi_g (call-flat index g0).
 template <int N, int M>
 __device__ __forceinline__ void group_keys_all(const float* phi_g, int64_t g0, const NoiseParams& np, float (&k)[M]) {
 #pragma unroll 1
@@ -247,7 +248,7 @@ __device__ __forceinline__ void group_keys_all(const float* phi_g, int64_t g0, c
     float k4[4];
     slot_keys(phi_g + 4 * s, g0 + 4 * s, np, k4);
 #pragma unroll
-    for (int j = 0; j < 4; ++j) k[4 * s + j] = k4[j];
+    for (int j = 0; j < 4; ++j) k[4 * s + j] = k4[j] * kLn2;
   }
 }
 
