@@ -8,12 +8,17 @@
 namespace roi {
 namespace {
 
-constexpr int kThreads = 256;
-// Tiles of 512 M elements: two groups per thread per tile, relaxed in lockstep.
+// Launch shape per group size M: threads per CTA, pairs of groups per thread per
+// tile (relaxed in lockstep on packed FP32 for M = 4, one after the other for
+// M = 8), shared-memory stages, and the CTAs per SM the register budget is sized for.
 template <int M>
-constexpr int kTile = 512 * M;
-template <int M>
-constexpr int kStages = M == 4 ? 3 : 2;
+struct Cfg {
+  static constexpr int kThreads = 256;
+  static constexpr int kPairs = 1;
+  static constexpr int kStages = M == 4 ? 3 : 2;
+  static constexpr int kMinBlocks = M == 4 ? 4 : 2;
+  static constexpr int kTile = 2 * kPairs * kThreads * M;  // elements
+};
 
 struct BwdArgs {
   const float* phi;
@@ -89,20 +94,34 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
   if (a.dW != nullptr) {
     // dW = bf16(dWm * S) now, while mu is live anyway (dWm is re-read)
 #pragma unroll
-    for (int h = 0; h < L; ++h) {
-#pragma unroll
-      for (int s = 0; s < M / 4; ++s) {
+    for (int s = 0; s < M / 4; ++s) {
+      if constexpr (L == 2) {
+        // both groups' products of member l in one packed multiply
+        const uint2 qa = reinterpret_cast<const uint2*>(dWm_g[0])[s];
+        const uint2 qb = reinterpret_cast<const uint2*>(dWm_g[1])[s];
+        const F2 p0 = f2(__uint_as_float(qa.x << 16), __uint_as_float(qb.x << 16)) * fg.soft(4 * s);
+        const F2 p1 = f2(__uint_as_float(qa.x & 0xffff0000u), __uint_as_float(qb.x & 0xffff0000u)) * fg.soft(4 * s + 1);
+        const F2 p2 = f2(__uint_as_float(qa.y << 16), __uint_as_float(qb.y << 16)) * fg.soft(4 * s + 2);
+        const F2 p3 = f2(__uint_as_float(qa.y & 0xffff0000u), __uint_as_float(qb.y & 0xffff0000u)) * fg.soft(4 * s + 3);
+        reinterpret_cast<uint2*>(a.dW + e0[0])[s] =
+            make_uint2(pack_bf16x2(lo(p0), lo(p1)), pack_bf16x2(lo(p2), lo(p3)));
+        reinterpret_cast<uint2*>(a.dW + e0[1])[s] =
+            make_uint2(pack_bf16x2(hi(p0), hi(p1)), pack_bf16x2(hi(p2), hi(p3)));
+      } else {
         float d[4];
-        unpack4(reinterpret_cast<const uint2*>(dWm_g[h])[s], d);
+        unpack4(reinterpret_cast<const uint2*>(dWm_g[0])[s], d);
         uint2 o;
-        o.x = pack_bf16x2(__fmul_rn(d[0], lane_of(fg.soft(4 * s), h)), __fmul_rn(d[1], lane_of(fg.soft(4 * s + 1), h)));
-        o.y = pack_bf16x2(__fmul_rn(d[2], lane_of(fg.soft(4 * s + 2), h)), __fmul_rn(d[3], lane_of(fg.soft(4 * s + 3), h)));
-        reinterpret_cast<uint2*>(a.dW + e0[h])[s] = o;
+        o.x = pack_bf16x2(__fmul_rn(d[0], fg.soft(4 * s)), __fmul_rn(d[1], fg.soft(4 * s + 1)));
+        o.y = pack_bf16x2(__fmul_rn(d[2], fg.soft(4 * s + 2)), __fmul_rn(d[3], fg.soft(4 * s + 3)));
+        reinterpret_cast<uint2*>(a.dW + e0[0])[s] = o;
       }
     }
   }
   V dkv[M];
   fg.backward(c, a.inv_tau, dkv);
+  // dL/dphi = dL/dkappa / lambda
+#pragma unroll
+  for (int l = 0; l < M; ++l) dkv[l] = vmul(dkv[l], vconst<V>(a.np.inv_lam));
 #pragma unroll
   for (int h = 0; h < L; ++h) {
     float dk[M];
@@ -118,6 +137,8 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
       ExactGroup<N, M> ex;
       ex.forward(k, N, M, a.tau, S);
       ex.backward(cc, N, M, a.tau, dk);
+#pragma unroll
+      for (int l = 0; l < M; ++l) dk[l] = __fmul_rn(dk[l], a.np.inv_lam);
       if (a.dW != nullptr) {
 #pragma unroll
         for (int s = 0; s < M / 4; ++s) {
@@ -132,17 +153,15 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
     }
 #pragma unroll
     for (int s = 0; s < M / 4; ++s)
-      reinterpret_cast<float4*>(a.dphi + e0[h])[s] =
-          make_float4(dk[4 * s] * a.np.inv_lam, dk[4 * s + 1] * a.np.inv_lam, dk[4 * s + 2] * a.np.inv_lam,
-                      dk[4 * s + 3] * a.np.inv_lam);
+      reinterpret_cast<float4*>(a.dphi + e0[h])[s] = make_float4(dk[4 * s], dk[4 * s + 1], dk[4 * s + 2], dk[4 * s + 3]);
   }
 }
 
 template <int N, int M, bool TAU1>
-__global__ void __launch_bounds__(kThreads, M == 4 ? 4 : 2) roi_bwd_kernel(BwdArgs a) {
+__global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_kernel(BwdArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
-  constexpr int kT = kTile<M>;
-  static_assert(kT / M == 2 * kThreads, "two groups per thread per tile");
+  using C = Cfg<M>;
+  constexpr int kT = C::kTile;
   TileSrc<3> src;
   src.ptr[0] = reinterpret_cast<const uint8_t*>(a.phi);
   src.esize[0] = 4;
@@ -151,23 +170,26 @@ __global__ void __launch_bounds__(kThreads, M == 4 ? 4 : 2) roi_bwd_kernel(BwdAr
   src.ptr[2] = reinterpret_cast<const uint8_t*>(a.dWm);
   src.esize[2] = 2;
 
-  const bool ok = run_tiles<kThreads, kT, kStages<M>, 3>(
+  const bool ok = run_tiles<C::kThreads, kT, C::kStages, 3>(
       smem, src, a.full_tiles, a.status, [&](const uint8_t* const* stage, int64_t tile) {
         const float* sphi = reinterpret_cast<const float*>(stage[0]);
         const uint16_t* sW = reinterpret_cast<const uint16_t*>(stage[1]);
         const uint16_t* sdW = reinterpret_cast<const uint16_t*>(stage[2]);
         const int64_t base = tile * kT;
-        const int g0 = threadIdx.x, g1 = threadIdx.x + kThreads;
-        const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
-        const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
-        const uint16_t* pd[2] = {sdW + g0 * M, sdW + g1 * M};
-        const int64_t e0[2] = {base + g0 * M, base + g1 * M};
-        if constexpr (M == 4) {
-          bwd_groups<N, M, TAU1, F2>(pp, pw, pd, e0, a);
-        } else {
-          // M = 8: the paired step history does not fit the register file; one group at a time
+#pragma unroll
+        for (int p = 0; p < C::kPairs; ++p) {
+          const int g0 = threadIdx.x + 2 * p * C::kThreads, g1 = g0 + C::kThreads;
+          const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
+          const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
+          const uint16_t* pd[2] = {sdW + g0 * M, sdW + g1 * M};
+          const int64_t e0[2] = {base + g0 * M, base + g1 * M};
+          if constexpr (M == 4) {
+            bwd_groups<N, M, TAU1, F2>(pp, pw, pd, e0, a);
+          } else {
+            // M = 8: the paired step history does not fit the register file; one group at a time
 #pragma unroll 1
-          for (int h = 0; h < 2; ++h) bwd_groups<N, M, TAU1, float>(pp + h, pw + h, pd + h, e0 + h, a);
+            for (int h = 0; h < 2; ++h) bwd_groups<N, M, TAU1, float>(pp + h, pw + h, pd + h, e0 + h, a);
+          }
         }
       });
   if (!ok) return;
@@ -175,7 +197,7 @@ __global__ void __launch_bounds__(kThreads, M == 4 ? 4 : 2) roi_bwd_kernel(BwdAr
   if (blockIdx.x == gridDim.x - 1) {
     const int64_t t0 = a.full_tiles * kT;
     const int64_t tail_groups = (a.E - t0) / M;
-    for (int64_t gi = threadIdx.x; gi < tail_groups; gi += kThreads) {
+    for (int64_t gi = threadIdx.x; gi < tail_groups; gi += C::kThreads) {
       const float* pp[1] = {a.phi + t0 + gi * M};
       const uint16_t* pw[1] = {a.W + t0 + gi * M};
       const uint16_t* pd[1] = {a.dWm + t0 + gi * M};
@@ -213,8 +235,9 @@ struct LaunchCache {
 
 template <int N, int M, bool TAU1>
 int launch_tiles(const BwdArgs& a, cudaStream_t stream) {
+  using C = Cfg<M>;
   auto kern = roi_bwd_kernel<N, M, TAU1>;
-  const size_t smem = tile_smem_bytes<kTile<M>, kStages<M>>(8);
+  const size_t smem = tile_smem_bytes<C::kTile, C::kStages>(8);
   static LaunchCache cache;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return -1;
@@ -222,12 +245,12 @@ int launch_tiles(const BwdArgs& a, cudaStream_t stream) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem)) != cudaSuccess)
       return -1;
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem) != cudaSuccess) return -1;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, C::kThreads, smem) != cudaSuccess) return -1;
     cache.per_sm[dev] = per_sm < 1 ? 1 : per_sm;
   }
   const int64_t cap = int64_t(sm_count()) * cache.per_sm[dev];
   const int grid = int(a.full_tiles < 1 ? 1 : (a.full_tiles < cap ? a.full_tiles : cap));
-  kern<<<grid, kThreads, smem, stream>>>(a);
+  kern<<<grid, C::kThreads, smem, stream>>>(a);
   return cudaGetLastError() == cudaSuccess ? 1 : -1;
 }
 
@@ -246,7 +269,7 @@ int launch_bwd(const BwdCall& c) {
   a.dphi = c.dphi;
   a.dW = c.dW;
   a.E = c.E;
-  a.full_tiles = c.E / (c.M == 8 ? kTile<8> : kTile<4>);
+  a.full_tiles = c.E / (c.M == 8 ? Cfg<8>::kTile : Cfg<4>::kTile);
   a.tau = c.tau;
   a.inv_tau = 1.0f / c.tau;
   a.np = c.np;

@@ -210,6 +210,43 @@ __device__ __forceinline__ uint32_t topn_bits4(const float (&kap)[4], int N) {
   return pick(w0) | (pick(w1) << 1) | (pick(w2) << 2) | (pick(w3) << 3);
 }
 
+// M = 4, two groups at once (one per lane of F2), for groups whose four keys are
+// all finite: the sign bit of k_i - k_j is set iff k_i < k_j, i.e. iff j outranks
+// i (equal keys give +0, so the lower index wins, as above).  The six pairwise
+// differences of both groups take six packed subtractions; each member's
+// selection is then one 3-input logic function of its three signs (majority for
+// N = 2, AND for N = 1, OR for N = 3).  Differences are exact in sign: no
+// flush-to-zero, and x - y == 0 only for x == y.
+__device__ __forceinline__ void topn_bits4_signs(const F2 (&k)[4], int N, uint32_t (&bits)[2]) {
+  const F2 d01 = k[0] - k[1], d02 = k[0] - k[2], d03 = k[0] - k[3];
+  const F2 d12 = k[1] - k[2], d13 = k[1] - k[3], d23 = k[2] - k[3];
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    auto sg = [h](F2 d) { return __float_as_uint(h == 0 ? lo(d) : hi(d)); };
+    const uint32_t s01 = sg(d01), s02 = sg(d02), s03 = sg(d03), s12 = sg(d12), s13 = sg(d13), s23 = sg(d23);
+    // member l wins against j < l when s_jl is set, against j > l when s_lj is clear
+    uint32_t w0, w1, w2, w3;
+    if (N == 2) {
+      auto maj = [](uint32_t a, uint32_t b, uint32_t c) { return (a & b) | (a & c) | (b & c); };
+      w0 = ~maj(s01, s02, s03);
+      w1 = maj(s01, ~s12, ~s13);
+      w2 = maj(s02, s12, ~s23);
+      w3 = maj(s03, s13, s23);
+    } else if (N == 1) {
+      w0 = ~(s01 | s02 | s03);
+      w1 = s01 & ~s12 & ~s13;
+      w2 = s02 & s12 & ~s23;
+      w3 = s03 & s13 & s23;
+    } else {
+      w0 = ~(s01 & s02 & s03);
+      w1 = s01 | ~s12 | ~s13;
+      w2 = s02 | s12 | ~s23;
+      w3 = s03 | s13 | s23;
+    }
+    bits[h] = (w0 >> 31) | ((w1 >> 31) << 1) | ((w2 >> 31) << 2) | ((w3 >> 31) << 3);
+  }
+}
+
 // Runtime-M version for the generic path (M <= 32).
 __device__ __forceinline__ uint32_t topn_bits_dyn(const float* kap, int N, int M) {
   uint32_t bits = 0;
@@ -237,7 +274,8 @@ __device__ __forceinline__ float lse_excluding(const float* z, int M, int skip) 
   float m = -INFINITY;
   for (int i = 0; i < M; ++i)
     if (i != skip) m = fmaxf(m, z[i]);
-  if (m == -INFINITY) return -INFINITY;
+  if (m == -INFINITY) return -INFINITY;  // every member -inf
+  if (m == INFINITY) return INFINITY;     // a +inf member
   float s = 0.f;
   for (int i = 0; i < M; ++i)
     if (i != skip) s = __fadd_rn(s, expf(__fsub_rn(z[i], m)));
@@ -322,9 +360,11 @@ struct ExactGroup {
 // S to within fp32 rounding (packed products may be fused into FMAs by the
 // compiler, see roi_vec.cuh).  The fallback decision depends only on sums of
 // exp2 outputs and is therefore the same in both kernels.
-// `flag` (one bit per lane) is raised when an exclusive sum drops below 2^-100
-// (a key gap of ~69 natural-log units); the caller then recomputes that group
-// with ExactGroup.
+// `flag` (one bit per lane) is raised when a key is not finite and, depending on
+// tau, when a key lies more than 100 log2 units from the first one (tau = 1) or
+// an exclusive sum drops below 2^-100 (a key gap of ~69 natural-log units); the
+// caller then recomputes that group with ExactGroup (and re-ranks it with the
+// comparison-based top-N, which orders NaN as -inf).
 // ---------------------------------------------------------------------------
 template <int M, class V>
 __device__ __forceinline__ void exclusive_sums(const V (&x)[M], V (&ex)[M]) {
@@ -444,7 +484,8 @@ struct FastGroup {
       V d[M];
 #pragma unroll
       for (int l = 0; l < M; ++l) d[l] = vmul(vsub(kap[l], kmax), sc);
-      flag = vbelow(vsub(kmax, kmax), 0.0f);  // non-finite maximum
+      const V ksum = sum_of(kap);
+      flag = vbelow(vsub(ksum, ksum), 0.0f);  // a non-finite key (or a sum beyond the float range)
 #pragma unroll
       for (int k = 0; k < N; ++k) {
         V e[M];

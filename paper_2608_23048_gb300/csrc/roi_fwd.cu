@@ -8,13 +8,17 @@
 namespace roi {
 namespace {
 
-constexpr int kThreads = 256;
-// Tiles of 512 M elements give every thread two groups per tile, relaxed in
-// lockstep on packed FP32 (F2).  Stages: 48 KB (M = 4) or 48 KB (M = 8, two).
+// Launch shape per group size M: threads per CTA, pairs of groups per thread per
+// tile (the two groups of a pair are relaxed in lockstep on packed FP32, F2),
+// shared-memory stages, and the CTAs per SM the register budget is sized for.
 template <int M>
-constexpr int kTile = 512 * M;
-template <int M>
-constexpr int kStages = M == 4 ? 4 : 2;
+struct Cfg {
+  static constexpr int kThreads = 256;
+  static constexpr int kPairs = M == 4 ? 2 : 1;
+  static constexpr int kStages = 2;  // 48 KB per CTA (M = 4) or 48 KB (M = 8)
+  static constexpr int kMinBlocks = M == 4 ? 4 : 2;
+  static constexpr int kTile = 2 * kPairs * kThreads * M;  // elements
+};
 
 struct FwdArgs {
   const float* phi;
@@ -108,39 +112,78 @@ __device__ __forceinline__ void fwd_groups(const float* const* phi_g, const uint
 
   FastGroup<N, M, TAU1, false, V> fg;
   fg.forward(kap, a.inv_tau);
+  float S[L][M];
 #pragma unroll
-  for (int h = 0; h < L; ++h) {
-    float k[M], S[M];
+  for (int h = 0; h < L; ++h)
 #pragma unroll
-    for (int l = 0; l < M; ++l) {
-      k[l] = lane_of(kap[l], h);
-      S[l] = lane_of(fg.S[l], h);
+    for (int l = 0; l < M; ++l) S[h][l] = lane_of(fg.S[l], h);
+  // ranking the log2-unit keys ranks kappa
+  constexpr bool kSigns = M == 4 && L == 2;
+  if constexpr (kSigns) {
+    uint32_t b2[2];
+    topn_bits4_signs(kap, N, b2);  // finite keys; flagged groups are re-ranked below
+    bits[0] = b2[0], bits[1] = b2[1];
+  } else {
+#pragma unroll
+    for (int h = 0; h < L; ++h) {
+      float k[M];
+#pragma unroll
+      for (int l = 0; l < M; ++l) k[l] = lane_of(kap[l], h);
+      if constexpr (M == 4) {
+        bits[h] = topn_bits4(k, N);
+      } else {
+        bits[h] = topn_bits<M>(k, N);
+      }
     }
-    // ranking the log2-unit keys ranks kappa
-    if constexpr (M == 4) {
-      bits[h] = topn_bits4(k, N);
+  }
+  if (fg.flag != 0u) {
+#pragma unroll
+    for (int h = 0; h < L; ++h) {
+      if ((fg.flag >> h) & 1u) {
+        float k[M], kn[M];
+#pragma unroll
+        for (int l = 0; l < M; ++l) {
+          k[l] = lane_of(kap[l], h);
+          kn[l] = k[l] * kLn2;  // natural-log keys
+        }
+        if constexpr (kSigns) bits[h] = topn_bits4(k, N);
+        ExactGroup<N, M> ex;
+        ex.forward(kn, N, M, a.tau, S[h]);
+      }
+    }
+  }
+  // Wm = bf16(W * S); W is read here, not kept live through the relaxation
+#pragma unroll
+  for (int s = 0; s < M / 4; ++s) {
+    const float* sa = S[0] + 4 * s;
+    if constexpr (L == 2) {
+      // both groups' products of member l in one packed multiply
+      const float* sb = S[1] + 4 * s;
+      const uint2 qa = reinterpret_cast<const uint2*>(W_g[0])[s];
+      const uint2 qb = reinterpret_cast<const uint2*>(W_g[1])[s];
+      const F2 p0 = f2(__uint_as_float(qa.x << 16), __uint_as_float(qb.x << 16)) * f2(sa[0], sb[0]);
+      const F2 p1 = f2(__uint_as_float(qa.x & 0xffff0000u), __uint_as_float(qb.x & 0xffff0000u)) * f2(sa[1], sb[1]);
+      const F2 p2 = f2(__uint_as_float(qa.y << 16), __uint_as_float(qb.y << 16)) * f2(sa[2], sb[2]);
+      const F2 p3 = f2(__uint_as_float(qa.y & 0xffff0000u), __uint_as_float(qb.y & 0xffff0000u)) * f2(sa[3], sb[3]);
+      reinterpret_cast<uint2*>(a.Wm + e0[0])[s] =
+          make_uint2(pack_bf16x2(lo(p0), lo(p1)), pack_bf16x2(lo(p2), lo(p3)));
+      reinterpret_cast<uint2*>(a.Wm + e0[1])[s] =
+          make_uint2(pack_bf16x2(hi(p0), hi(p1)), pack_bf16x2(hi(p2), hi(p3)));
     } else {
-      bits[h] = topn_bits<M>(k, N);
-    }
-    if ((fg.flag >> h) & 1u) {
-      float kn[M];
-#pragma unroll
-      for (int l = 0; l < M; ++l) kn[l] = k[l] * kLn2;  // natural-log keys
-      ExactGroup<N, M> ex;
-      ex.forward(kn, N, M, a.tau, S);
-    }
-#pragma unroll
-    for (int s = 0; s < M / 4; ++s) {
-      // W is read here, not kept live through the relaxation
-      const uint2 q = reinterpret_cast<const uint2*>(W_g[h])[s];
+      const uint2 q = reinterpret_cast<const uint2*>(W_g[0])[s];
       const float wv[4] = {bf16_bits_to_float(q.x & 0xffffu), bf16_bits_to_float(q.x >> 16),
                            bf16_bits_to_float(q.y & 0xffffu), bf16_bits_to_float(q.y >> 16)};
-      const float* sv = S + 4 * s;
       uint2 o;
-      o.x = pack_bf16x2(__fmul_rn(wv[0], sv[0]), __fmul_rn(wv[1], sv[1]));
-      o.y = pack_bf16x2(__fmul_rn(wv[2], sv[2]), __fmul_rn(wv[3], sv[3]));
-      reinterpret_cast<uint2*>(a.Wm + e0[h])[s] = o;
-      if (a.soft != nullptr) reinterpret_cast<float4*>(a.soft + e0[h])[s] = make_float4(sv[0], sv[1], sv[2], sv[3]);
+      o.x = pack_bf16x2(__fmul_rn(wv[0], sa[0]), __fmul_rn(wv[1], sa[1]));
+      o.y = pack_bf16x2(__fmul_rn(wv[2], sa[2]), __fmul_rn(wv[3], sa[3]));
+      reinterpret_cast<uint2*>(a.Wm + e0[0])[s] = o;
+    }
+    if (a.soft != nullptr) {
+#pragma unroll
+      for (int h = 0; h < L; ++h) {
+        const float* sh = S[h] + 4 * s;
+        reinterpret_cast<float4*>(a.soft + e0[h])[s] = make_float4(sh[0], sh[1], sh[2], sh[3]);
+      }
     }
   }
 }
@@ -156,31 +199,55 @@ __device__ __forceinline__ void store_hard(uint32_t* hard, int64_t e0, uint32_t 
   if (active && (lane % kLanesPerWord) == 0) hard[e0 >> 5] = v;
 }
 
+// The same for a tile's two groups per thread (first elements e0a, e0b; all
+// lanes active).  Both masks travel in one register, the first group's in the
+// low half-word and the second's in the high one; the shuffles OR the masks of
+// the 16 / M lanes that fill a half-word, then one exchange between the two
+// halves of each word's lane range completes the first group's word on the
+// leader of the first half and the second group's word on the leader of the
+// second half.
+template <int M>
+__device__ __forceinline__ void store_hard_pair(uint32_t* hard, int64_t e0a, int64_t e0b, uint32_t bits_a,
+                                                uint32_t bits_b) {
+  constexpr int kHalf = 16 / M;  // lanes per half-word
+  const int lane = threadIdx.x & 31;
+  const int sh = (lane % kHalf) * M;
+  uint32_t v = (bits_a << sh) | (bits_b << (16 + sh));
+#pragma unroll
+  for (int o = 1; o < kHalf; o <<= 1) v |= __shfl_xor_sync(0xffffffffu, v, o);
+  const uint32_t w = __shfl_xor_sync(0xffffffffu, v, kHalf);
+  const bool upper = (lane & kHalf) != 0;
+  // lower leader: {own low half, partner's low half}; upper leader: {partner's high half, own high half}
+  const uint32_t word = __byte_perm(v, w, upper ? 0x3276u : 0x5410u);
+  if (lane % kHalf == 0) hard[(upper ? e0b : e0a) >> 5] = word;
+}
+
 template <int N, int M, bool TAU1>
-__global__ void __launch_bounds__(kThreads, M == 4 ? 4 : 2) roi_fwd_kernel(FwdArgs a) {
+__global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_fwd_kernel(FwdArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
-  constexpr int kT = kTile<M>;
-  static_assert(kT / M == 2 * kThreads, "two groups per thread per tile");
+  using C = Cfg<M>;
+  constexpr int kT = C::kTile;
   TileSrc<2> src;
   src.ptr[0] = reinterpret_cast<const uint8_t*>(a.phi);
   src.esize[0] = 4;
   src.ptr[1] = reinterpret_cast<const uint8_t*>(a.W);
   src.esize[1] = 2;
 
-  const bool ok = run_tiles<kThreads, kT, kStages<M>, 2>(
+  const bool ok = run_tiles<C::kThreads, kT, C::kStages, 2>(
       smem, src, a.full_tiles, a.status, [&](const uint8_t* const* stage, int64_t tile) {
         const float* sphi = reinterpret_cast<const float*>(stage[0]);
         const uint16_t* sW = reinterpret_cast<const uint16_t*>(stage[1]);
         const int64_t base = tile * kT;
-        const int g0 = threadIdx.x, g1 = threadIdx.x + kThreads;
-        const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
-        const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
-        const int64_t e0[2] = {base + g0 * M, base + g1 * M};
-        uint32_t bits[2];
-        fwd_groups<N, M, TAU1, F2>(pp, pw, e0, a, bits);
-        if (a.hard != nullptr) {
-          store_hard<M>(a.hard, e0[0], bits[0], true);
-          store_hard<M>(a.hard, e0[1], bits[1], true);
+#pragma unroll
+        for (int p = 0; p < C::kPairs; ++p) {
+          // pair p: groups t and t + kThreads of the p-th block of 2 kThreads groups
+          const int g0 = threadIdx.x + 2 * p * C::kThreads, g1 = g0 + C::kThreads;
+          const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
+          const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
+          const int64_t e0[2] = {base + g0 * M, base + g1 * M};
+          uint32_t bits[2];
+          fwd_groups<N, M, TAU1, F2>(pp, pw, e0, a, bits);
+          if (a.hard != nullptr) store_hard_pair<M>(a.hard, e0[0], e0[1], bits[0], bits[1]);
         }
       });
   if (!ok) return;
@@ -189,9 +256,9 @@ __global__ void __launch_bounds__(kThreads, M == 4 ? 4 : 2) roi_fwd_kernel(FwdAr
   if (blockIdx.x == gridDim.x - 1) {
     const int64_t t0 = a.full_tiles * kT;
     const int64_t tail_groups = (a.E - t0) / M;
-    const int64_t rounds = (tail_groups + kThreads - 1) / kThreads;
+    const int64_t rounds = (tail_groups + C::kThreads - 1) / C::kThreads;
     for (int64_t r = 0; r < rounds; ++r) {
-      const int64_t gi = threadIdx.x + r * kThreads;
+      const int64_t gi = threadIdx.x + r * C::kThreads;
       const bool active = gi < tail_groups;
       uint32_t bits = 0;
       if (active) {
@@ -241,8 +308,9 @@ struct LaunchCache {
 
 template <int N, int M, bool TAU1>
 int launch_tiles(const FwdArgs& a, cudaStream_t stream) {
+  using C = Cfg<M>;
   auto kern = roi_fwd_kernel<N, M, TAU1>;
-  const size_t smem = tile_smem_bytes<kTile<M>, kStages<M>>(6);
+  const size_t smem = tile_smem_bytes<C::kTile, C::kStages>(6);
   static LaunchCache cache;  // per instantiation and device; racing writers store the same value
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return -1;
@@ -250,12 +318,12 @@ int launch_tiles(const FwdArgs& a, cudaStream_t stream) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem)) != cudaSuccess)
       return -1;
     int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem) != cudaSuccess) return -1;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, C::kThreads, smem) != cudaSuccess) return -1;
     cache.per_sm[dev] = per_sm < 1 ? 1 : per_sm;
   }
   const int64_t cap = int64_t(sm_count()) * cache.per_sm[dev];
   const int grid = int(a.full_tiles < 1 ? 1 : (a.full_tiles < cap ? a.full_tiles : cap));
-  kern<<<grid, kThreads, smem, stream>>>(a);
+  kern<<<grid, C::kThreads, smem, stream>>>(a);
   return cudaGetLastError() == cudaSuccess ? 1 : -1;
 }
 
@@ -274,7 +342,7 @@ int launch_fwd(const FwdCall& c) {
   a.soft = c.soft;
   a.hard = c.hard;
   a.E = c.E;
-  a.full_tiles = c.E / (c.M == 8 ? kTile<8> : kTile<4>);
+  a.full_tiles = c.E / (c.M == 8 ? Cfg<8>::kTile : Cfg<4>::kTile);
   a.tau = c.tau;
   a.inv_tau = 1.0f / c.tau;
   a.np = c.np;

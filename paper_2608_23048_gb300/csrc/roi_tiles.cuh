@@ -49,9 +49,8 @@ __device__ __forceinline__ bool run_tiles(uint8_t* smem, const TileSrc<NARR>& sr
   const int64_t stride = gridDim.x;
   const int64_t my_tiles = first < full_tiles ? (full_tiles - first + stride - 1) / stride : 0;
 
-  auto issue = [&](int64_t i) {
-    const int s = int(i % STAGES);
-    const int64_t t = first + i * stride;
+  // fill stage s with tile t
+  auto issue = [&](int s, int64_t t) {
     fills[s] += 1;
     mbar_arrive_expect_tx(&bars[s], stage_bytes);
 #pragma unroll
@@ -70,13 +69,15 @@ __device__ __forceinline__ bool run_tiles(uint8_t* smem, const TileSrc<NARR>& sr
       fills[s] = 0;
     }
     fence_mbar_init();
-    for (int64_t i = 0; i < my_tiles && i < STAGES; ++i) issue(i);
+    for (int i = 0; i < STAGES && i < my_tiles; ++i) issue(i, first + i * stride);
   }
   __syncthreads();
 
-  for (int64_t i = 0; i < my_tiles; ++i) {
-    const int s = int(i % STAGES);
-    const uint32_t parity = uint32_t((i / STAGES) & 1);
+  // stage index and mbarrier phase advance incrementally (no 64-bit division)
+  int s = 0;
+  uint32_t parity = 0;
+  int64_t tile = first;
+  for (int64_t i = 0; i < my_tiles; ++i, tile += stride) {
     if (!mbar_wait_bounded(&bars[s], parity)) {
       if (lane == 0) {
         atomicOr(status, kStatusTimeout);
@@ -92,7 +93,7 @@ __device__ __forceinline__ bool run_tiles(uint8_t* smem, const TileSrc<NARR>& sr
     const uint8_t* stage[NARR];
 #pragma unroll
     for (int a = 0; a < NARR; ++a) stage[a] = smem + arr_off[a] + size_t(s) * TILE * src.esize[a];
-    compute(stage, first + i * stride);
+    compute(stage, tile);
     __syncwarp();
     if (lane == 0) {
       __threadfence_block();
@@ -101,9 +102,13 @@ __device__ __forceinline__ bool run_tiles(uint8_t* smem, const TileSrc<NARR>& sr
         done[s] = 0;
         if (i + STAGES < my_tiles) {
           asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-          issue(i + STAGES);
+          issue(s, tile + STAGES * stride);
         }
       }
+    }
+    if (++s == STAGES) {
+      s = 0;
+      parity ^= 1u;
     }
   }
   return true;

@@ -209,21 +209,37 @@ def test_wide_key_gaps_take_exact_path(roi, N, M, tau):
     check_against_oracle(got, phi.numpy(), WL.bf16_bits(W), WL.bf16_bits(dWm), N, M, tau, 3, 0, 0, 1.0, 0)
 
 
-def test_non_finite_logits_propagate(roi):
-    import torch
-    W, phi, dWm, *_ = make(4, 64, "normal", data_seed=9)
+@pytest.mark.parametrize("rows,cols", [(4, 64), (8, 2112)])
+def test_non_finite_logits_propagate(roi, rows, cols):
+    """NaN / +inf logits make their group's outputs NaN (for N = 1 a +inf member
+    alone, as in the oracle), -inf ranks last with zero weight; the 8 x 2112 case
+    puts them in full tiles and in the ragged tail."""
+    W, phi, dWm, *_ = make(rows, cols, "normal", data_seed=9)
     phi = phi.clone()
     phi[0, 1] = float("nan")
     phi[1, 5] = float("inf")
     phi[2, 8] = float("-inf")
+    if cols > 64:
+        phi[3, 1000] = float("-inf")
+        phi[4, 2000] = float("nan")
+        phi[5, 33] = float("inf")
+        phi[rows - 1, cols - 3] = float("-inf")  # ragged tail
     st = roi.NoiseState(0, 0, 0, 1.0, 0)
-    for N, M, tau in ((2, 4, 1.0), (2, 4, 0.5), (4, 8, 1.0), (3, 4, 1.0)):
+    Wb, dWb = WL.bf16_bits(W), WL.bf16_bits(dWm)
+    for N, M, tau in ((2, 4, 1.0), (2, 4, 0.5), (4, 8, 1.0), (4, 8, 0.5), (3, 4, 1.0), (1, 4, 0.7),
+                      (8, 16, 0.5), (16, 32, 1.0)):
         got = gpu_run(roi, phi, W, dWm, N, M, tau, st)
-        ref = O.mask_fwd(phi.numpy(), WL.bf16_bits(W), N, M, tau, 0, 0)
+        with np.errstate(all="ignore"):
+            ref = O.mask_fwd(phi.numpy(), Wb, N, M, tau, 0, 0)
+            refb = O.mask_bwd(phi.numpy(), Wb, dWb, N, M, tau, 0, 0)
         assert np.array_equal(np.isnan(got["soft"]), np.isnan(ref["soft"])), (N, M, tau)
         fin = ~np.isnan(ref["soft"])
         assert np.allclose(got["soft"][fin], ref["soft"][fin], atol=1e-5)
         assert np.array_equal(got["hard_bits"], ref["hard_bits"]), (N, M, tau)
+        assert np.array_equal(np.isnan(got["dlogits"]), np.isnan(refb["dlogits"])), (N, M, tau)
+        fin = ~np.isnan(refb["dlogits"])
+        scale = np.abs(refb["dlogits"][fin]).max()
+        assert np.allclose(got["dlogits"][fin], refb["dlogits"][fin], rtol=0, atol=1e-4 * scale), (N, M, tau)
 
 
 @pytest.mark.parametrize("rows,cols,N,M", [(37, 1000, 2, 4), (29, 1536, 4, 8), (13, 960, 3, 4),
