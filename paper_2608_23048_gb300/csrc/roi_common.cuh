@@ -247,6 +247,56 @@ __device__ __forceinline__ void topn_bits4_signs(const F2 (&k)[4], int N, uint32
   }
 }
 
+// M = 8, two groups at once, for groups whose keys are all finite: the N-th
+// largest key of each group comes out of a sorting network (Batcher's odd-even
+// merge sort, 19 compare-exchanges), and member l is selected iff its key is at
+// least that threshold, read off the sign bit of the packed difference.  When
+// the threshold is tied with another member more than N members pass; such a
+// group gets 0xffffffff and the caller re-ranks it with topn_bits<8>.
+template <int N>
+__device__ __forceinline__ void topn_bits8_threshold(const F2 (&k)[8], uint32_t (&bits)[2]) {
+  static_assert(N >= 1 && N < 8, "1 <= N < 8");
+  float thr[2];
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    float s[8];
+#pragma unroll
+    for (int l = 0; l < 8; ++l) s[l] = h == 0 ? lo(k[l]) : hi(k[l]);
+    // descending: after a compare-exchange (a, b), s[a] >= s[b]
+    auto ce = [&s](int a, int b) {
+      const float x = s[a], y = s[b];
+      s[a] = fmaxf(x, y);
+      s[b] = fminf(x, y);
+    };
+    ce(0, 1), ce(2, 3), ce(4, 5), ce(6, 7);
+    ce(0, 2), ce(1, 3), ce(4, 6), ce(5, 7);
+    ce(1, 2), ce(5, 6);
+    ce(0, 4), ce(1, 5), ce(2, 6), ce(3, 7);
+    ce(2, 4), ce(3, 5);
+    ce(1, 2), ce(3, 4), ce(5, 6);
+    thr[h] = s[N - 1];
+  }
+  const F2 t = f2(thr[0], thr[1]);
+  uint32_t sg[2][8];
+#pragma unroll
+  for (int l = 0; l < 8; ++l) {
+    const F2 d = k[l] - t;  // >= 0 (sign bit clear) iff member l passes
+    sg[0][l] = __float_as_uint(lo(d));
+    sg[1][l] = __float_as_uint(hi(d));
+  }
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    // the sign bytes of members 0-3 and 4-7 into two words; their four top bits
+    // (7, 15, 23, 31) land in bits 28-31 of the product with 2^21 + 2^14 + 2^7 + 1
+    const uint32_t a = __byte_perm(__byte_perm(sg[h][0], sg[h][1], 0x0073u), __byte_perm(sg[h][2], sg[h][3], 0x0073u), 0x5410u);
+    const uint32_t b = __byte_perm(__byte_perm(sg[h][4], sg[h][5], 0x0073u), __byte_perm(sg[h][6], sg[h][7], 0x0073u), 0x5410u);
+    const uint32_t pa = ((~a & 0x80808080u) * 0x00204081u) >> 28;
+    const uint32_t pb = ((~b & 0x80808080u) * 0x00204081u) >> 28;
+    const uint32_t v = pa | (pb << 4);
+    bits[h] = __popc(v) == N ? v : 0xffffffffu;
+  }
+}
+
 // Runtime-M version for the generic path (M <= 32).
 __device__ __forceinline__ uint32_t topn_bits_dyn(const float* kap, int N, int M) {
   uint32_t bits = 0;

@@ -45,15 +45,50 @@ __global__ void __launch_bounds__(256) roi_export_vec_kernel(const float* __rest
        wi += int64_t(gridDim.x) * blockDim.x) {
     const float4* p = reinterpret_cast<const float4*>(phi + wi * 32);
     uint32_t word = 0;
+    if constexpr (M == 8) {
+      // two groups at a time: threshold ranking, with the comparison-based
+      // routine for non-finite keys and tied thresholds
 #pragma unroll
-    for (int g = 0; g < 32 / M; ++g) {
-      float k[M];
+      for (int gp = 0; gp < 2; ++gp) {
+        float k[2][8];
 #pragma unroll
-      for (int s = 0; s < M / 4; ++s) {
-        const float4 v = p[g * (M / 4) + s];
-        k[4 * s] = v.x, k[4 * s + 1] = v.y, k[4 * s + 2] = v.z, k[4 * s + 3] = v.w;
+        for (int h = 0; h < 2; ++h) {
+          const float4 v0 = p[(2 * gp + h) * 2], v1 = p[(2 * gp + h) * 2 + 1];
+          k[h][0] = v0.x, k[h][1] = v0.y, k[h][2] = v0.z, k[h][3] = v0.w;
+          k[h][4] = v1.x, k[h][5] = v1.y, k[h][6] = v1.z, k[h][7] = v1.w;
+        }
+        F2 kk[8];
+#pragma unroll
+        for (int l = 0; l < 8; ++l) kk[l] = f2(k[0][l], k[1][l]);
+        const F2 ks = sum_of(kk);
+        const uint32_t bad = vbelow(ks - ks, 0.0f);  // a non-finite key
+        uint32_t b2[2];
+        switch (N) {
+          case 1: topn_bits8_threshold<1>(kk, b2); break;
+          case 2: topn_bits8_threshold<2>(kk, b2); break;
+          case 3: topn_bits8_threshold<3>(kk, b2); break;
+          case 4: topn_bits8_threshold<4>(kk, b2); break;
+          case 5: topn_bits8_threshold<5>(kk, b2); break;
+          case 6: topn_bits8_threshold<6>(kk, b2); break;
+          default: topn_bits8_threshold<7>(kk, b2); break;
+        }
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          if (((bad >> h) & 1u) || b2[h] == 0xffffffffu) b2[h] = topn_bits<8>(k[h], N);
+          word |= b2[h] << ((2 * gp + h) * 8);
+        }
       }
-      word |= topn_bits<M>(k, N) << (g * M);
+    } else {
+#pragma unroll
+      for (int g = 0; g < 32 / M; ++g) {
+        float k[M];
+#pragma unroll
+        for (int s = 0; s < M / 4; ++s) {
+          const float4 v = p[g * (M / 4) + s];
+          k[4 * s] = v.x, k[4 * s + 1] = v.y, k[4 * s + 2] = v.z, k[4 * s + 3] = v.w;
+        }
+        word |= topn_bits<M>(k, N) << (g * M);
+      }
     }
     bits[wi] = word;
     if (Wp != nullptr) {

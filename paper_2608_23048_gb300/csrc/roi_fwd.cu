@@ -118,11 +118,27 @@ __device__ __forceinline__ void fwd_groups(const float* const* phi_g, const uint
 #pragma unroll
     for (int l = 0; l < M; ++l) S[h][l] = lane_of(fg.S[l], h);
   // ranking the log2-unit keys ranks kappa
-  constexpr bool kSigns = M == 4 && L == 2;
-  if constexpr (kSigns) {
+  constexpr bool kFastTopn = (M == 4 || M == 8) && L == 2;
+  if constexpr (kFastTopn) {
+    // finite keys only: flagged groups are re-ranked below
     uint32_t b2[2];
-    topn_bits4_signs(kap, N, b2);  // finite keys; flagged groups are re-ranked below
+    if constexpr (M == 4) {
+      topn_bits4_signs(kap, N, b2);
+    } else {
+      topn_bits8_threshold<N>(kap, b2);
+    }
     bits[0] = b2[0], bits[1] = b2[1];
+    if constexpr (M == 8) {
+#pragma unroll
+      for (int h = 0; h < L; ++h) {
+        if (bits[h] == 0xffffffffu) {  // threshold tied with another member
+          float k[M];
+#pragma unroll
+          for (int l = 0; l < M; ++l) k[l] = lane_of(kap[l], h);
+          bits[h] = topn_bits<M>(k, N);
+        }
+      }
+    }
   } else {
 #pragma unroll
     for (int h = 0; h < L; ++h) {
@@ -146,7 +162,13 @@ __device__ __forceinline__ void fwd_groups(const float* const* phi_g, const uint
           k[l] = lane_of(kap[l], h);
           kn[l] = k[l] * kLn2;  // natural-log keys
         }
-        if constexpr (kSigns) bits[h] = topn_bits4(k, N);
+        if constexpr (kFastTopn) {
+          if constexpr (M == 4) {
+            bits[h] = topn_bits4(k, N);
+          } else {
+            bits[h] = topn_bits<M>(k, N);
+          }
+        }
         ExactGroup<N, M> ex;
         ex.forward(kn, N, M, a.tau, S[h]);
       }

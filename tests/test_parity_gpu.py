@@ -243,12 +243,19 @@ def test_non_finite_logits_propagate(roi, rows, cols):
 
 
 @pytest.mark.parametrize("rows,cols,N,M", [(37, 1000, 2, 4), (29, 1536, 4, 8), (13, 960, 3, 4),
-                                           (11, 1001, 3, 7), (1, 36, 2, 4), (3, 40, 4, 8), (2, 96, 16, 32)])
+                                           (11, 1001, 3, 7), (1, 36, 2, 4), (3, 40, 4, 8), (2, 96, 16, 32),
+                                           (9, 1024, 1, 8), (9, 1024, 2, 8), (9, 1024, 6, 8), (9, 1024, 7, 8)])
 def test_export_bit_exact(roi, rows, cols, N, M):
     import torch
     W, phi, *_ = make(rows, cols, "normal", data_seed=rows + cols)
     phi = phi.clone()
     phi[0, :4] = 0.5  # exact ties
+    if rows >= 3 and cols >= 32:
+        phi[1, :8] = 0.25  # a whole group tied
+        phi[2, 8:16] = torch.tensor([3.0, 1.0, 1.0, 0.0, 2.0, 2.0, -1.0, 2.0])  # ties at several ranks
+        phi[2, 16] = float("nan")
+        phi[2, 25] = float("inf")
+        phi[2, 30] = float("-inf")
     dev = torch.device("cuda")
     bits = torch.empty(roi.hard_words(rows, cols), dtype=torch.int32, device=dev)
     Wp = torch.empty(rows, cols, dtype=torch.bfloat16, device=dev)
