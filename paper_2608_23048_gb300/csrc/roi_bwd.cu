@@ -2,6 +2,8 @@
 // registers, then sweep the N steps in reverse to turn dL/dS = dWm * W into
 // dL/dphi (Sec. 3.2: the map from logits to the soft N-hot vector is
 // differentiable; Sec. 4.2.2 Eq. 11-12).  Optionally dW = bf16(dWm * S).
+#include <type_traits>
+
 #include "roi_launch.h"
 #include "roi_tiles.cuh"
 
@@ -9,16 +11,23 @@ namespace roi {
 namespace {
 
 // Launch shape per group size M: threads per CTA, pairs of groups per thread per
-// tile (relaxed in lockstep on packed FP32 for M = 4, one after the other for
-// M = 8), shared-memory stages, and the CTAs per SM the register budget is sized for.
+// tile (the two groups of a pair are relaxed in lockstep on packed FP32),
+// shared-memory stages, and the CTAs per SM the register budget is sized for.
 template <int M>
 struct Cfg {
-  static constexpr int kThreads = 256;
+  // M = 8: the paired sweep needs ~170 registers; 128 threads x 3 CTAs per SM
+  static constexpr int kThreads = M == 4 ? 256 : 128;
   static constexpr int kPairs = 1;
   static constexpr int kStages = M == 4 ? 3 : 2;
-  static constexpr int kMinBlocks = M == 4 ? 4 : 2;
+  static constexpr int kMinBlocks = M == 4 ? 4 : 3;
   static constexpr int kTile = 2 * kPairs * kThreads * M;  // elements
 };
+// Byte offset of the shared-memory step history (M = 8) behind the tile ring,
+// and its size: steps 0 .. N-2 of two groups (one F2 per member) per thread.
+template <int M>
+constexpr size_t kHistOffset = (tile_smem_bytes<Cfg<M>::kTile, Cfg<M>::kStages>(8) + 15) & ~size_t(15);
+template <int N, int M>
+constexpr size_t kHistBytes = M == 8 ? size_t(N - 1) * M * Cfg<M>::kThreads * sizeof(F2) : 0;
 
 struct BwdArgs {
   const float* phi;
@@ -49,50 +58,123 @@ __device__ __forceinline__ float lane_of(V v, int h) {
   }
 }
 
-// L groups (one per lane of V) in lockstep: regenerate keys and relaxation,
-// sweep back, write dL/dphi (and dW).
-template <int N, int M, bool TAU1, class V>
-__device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint16_t* const* W_g,
-                                           const uint16_t* const* dWm_g, const int64_t* e0, const BwdArgs& a) {
+// Keys (log2 units) of L groups (one per lane of V): logits from the tile stage,
+// noise regenerated four members (one Philox block) at a time.
+template <int M, class V>
+__device__ __forceinline__ void bwd_keys(const float* const* phi_g, const int64_t* e0, const NoiseParams& np,
+                                         V (&kap)[M]) {
   constexpr int L = vlanes<V>();
-  V kap[M], c[M];
-  {
-    float ph[L][M], w[L][M], dw[L][M];
-    uint32_t x[L][M];
+#pragma unroll
+  for (int s = 0; s < M / 4; ++s) {
+    float ph[L][4];
+    uint32_t x[L][4];
 #pragma unroll
     for (int h = 0; h < L; ++h) {
-      const uint64_t q0 = (a.np.e_base + uint64_t(e0[h])) >> 2;
-#pragma unroll
-      for (int s = 0; s < M / 4; ++s) {
-        const float4 p = reinterpret_cast<const float4*>(phi_g[h])[s];
-        ph[h][4 * s] = p.x, ph[h][4 * s + 1] = p.y, ph[h][4 * s + 2] = p.z, ph[h][4 * s + 3] = p.w;
-        unpack4(reinterpret_cast<const uint2*>(W_g[h])[s], w[h] + 4 * s);
-        unpack4(reinterpret_cast<const uint2*>(dWm_g[h])[s], dw[h] + 4 * s);
-        const uint4 q = noise_block_q(a.np, q0 + s);
-        x[h][4 * s] = q.x, x[h][4 * s + 1] = q.y, x[h][4 * s + 2] = q.z, x[h][4 * s + 3] = q.w;
-      }
+      const float4 p = reinterpret_cast<const float4*>(phi_g[h])[s];
+      ph[h][0] = p.x, ph[h][1] = p.y, ph[h][2] = p.z, ph[h][3] = p.w;
+      const uint4 q = noise_block_q(np, ((np.e_base + uint64_t(e0[h])) >> 2) + s);
+      x[h][0] = q.x, x[h][1] = q.y, x[h][2] = q.z, x[h][3] = q.w;
     }
 #pragma unroll
-    for (int l = 0; l < M; ++l) {
-      V one_plus, phv, wv, dwv;
+    for (int j = 0; j < 4; ++j) {
+      V one_plus, phv;
       if constexpr (L == 1) {
-        one_plus = one_plus_from_word(x[0][l]);
-        phv = ph[0][l], wv = w[0][l], dwv = dw[0][l];
+        one_plus = one_plus_from_word(x[0][j]);
+        phv = ph[0][j];
       } else {
-        one_plus =
-            f2(one_plus_from_word(x[0][l]), one_plus_from_word(x[1][l]));
-        phv = f2(ph[0][l], ph[1][l]), wv = f2(w[0][l], w[1][l]), dwv = f2(dw[0][l], dw[1][l]);
+        one_plus = f2(one_plus_from_word(x[0][j]), one_plus_from_word(x[1][j]));
+        phv = f2(ph[0][j], ph[1][j]);
       }
       const V u = vsub(one_plus, vconst<V>(__uint_as_float(0x3f7fffffu)));
-      kap[l] = key_log2(phv, u, a.np.l2e_inv_lam);  // log2 units
-      c[l] = vmul(dwv, wv);
+      kap[4 * s + j] = key_log2(phv, u, np.l2e_inv_lam);
     }
   }
+}
 
-  FastGroup<N, M, TAU1, true, V> fg;
-  fg.forward(kap, a.inv_tau);
+// dL/dS = dWm * W of L groups (the rounding of Wm treated as identity).
+template <int M, class V>
+__device__ __forceinline__ void bwd_upstream(const uint16_t* const* W_g, const uint16_t* const* dWm_g, V (&c)[M]) {
+  constexpr int L = vlanes<V>();
+#pragma unroll
+  for (int s = 0; s < M / 4; ++s) {
+    float w[L][4], dw[L][4];
+#pragma unroll
+    for (int h = 0; h < L; ++h) {
+      unpack4(reinterpret_cast<const uint2*>(W_g[h])[s], w[h]);
+      unpack4(reinterpret_cast<const uint2*>(dWm_g[h])[s], dw[h]);
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      if constexpr (L == 1) {
+        c[4 * s + j] = vmul(dw[0][j], w[0][j]);
+      } else {
+        c[4 * s + j] = vmul(f2(dw[0][j], dw[1][j]), f2(w[0][j], w[1][j]));
+      }
+    }
+  }
+}
+
+// Keys and upstream gradients together, reading each stage word once.
+template <int M, class V>
+__device__ __forceinline__ void bwd_inputs(const float* const* phi_g, const uint16_t* const* W_g,
+                                           const uint16_t* const* dWm_g, const int64_t* e0, const NoiseParams& np,
+                                           V (&kap)[M], V (&c)[M]) {
+  constexpr int L = vlanes<V>();
+#pragma unroll
+  for (int s = 0; s < M / 4; ++s) {
+    float ph[L][4], w[L][4], dw[L][4];
+    uint32_t x[L][4];
+#pragma unroll
+    for (int h = 0; h < L; ++h) {
+      const float4 p = reinterpret_cast<const float4*>(phi_g[h])[s];
+      ph[h][0] = p.x, ph[h][1] = p.y, ph[h][2] = p.z, ph[h][3] = p.w;
+      unpack4(reinterpret_cast<const uint2*>(W_g[h])[s], w[h]);
+      unpack4(reinterpret_cast<const uint2*>(dWm_g[h])[s], dw[h]);
+      const uint4 q = noise_block_q(np, ((np.e_base + uint64_t(e0[h])) >> 2) + s);
+      x[h][0] = q.x, x[h][1] = q.y, x[h][2] = q.z, x[h][3] = q.w;
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      V one_plus, phv, wv, dwv;
+      if constexpr (L == 1) {
+        one_plus = one_plus_from_word(x[0][j]);
+        phv = ph[0][j], wv = w[0][j], dwv = dw[0][j];
+      } else {
+        one_plus = f2(one_plus_from_word(x[0][j]), one_plus_from_word(x[1][j]));
+        phv = f2(ph[0][j], ph[1][j]), wv = f2(w[0][j], w[1][j]), dwv = f2(dw[0][j], dw[1][j]);
+      }
+      const V u = vsub(one_plus, vconst<V>(__uint_as_float(0x3f7fffffu)));
+      kap[4 * s + j] = key_log2(phv, u, np.l2e_inv_lam);
+      c[4 * s + j] = vmul(dwv, wv);
+    }
+  }
+}
+
+// L groups (one per lane of V) in lockstep: regenerate keys and relaxation,
+// sweep back, write dL/dphi (and dW).  `hist` (shared memory, this thread's
+// slot) holds steps 0 .. N-2 of the relaxation when HIST is set; otherwise the
+// whole history stays in registers.  With HIST (M = 8) registers are tight:
+// the keys die after the forward relaxation (a flagged group re-forms them) and
+// the upstream gradients are formed only for the sweep.
+template <int N, int M, bool TAU1, class V, bool HIST = false>
+__device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint16_t* const* W_g,
+                                           const uint16_t* const* dWm_g, const int64_t* e0, const BwdArgs& a,
+                                           V* hist = nullptr) {
+  constexpr int L = vlanes<V>();
+  using Steps = typename std::conditional<HIST, SmemSteps<N, M, V, Cfg<M>::kThreads>, RegSteps<N, M, V>>::type;
+  FastGroup<N, M, TAU1, true, V, Steps> fg;
+  if constexpr (HIST) fg.st.at = hist;
+  V kap[HIST ? 1 : M], c[M], dkv[M];
+  if constexpr (HIST) {
+    V k[M];
+    bwd_keys<M, V>(phi_g, e0, a.np, k);
+    fg.forward(k, a.inv_tau);
+  } else {
+    bwd_inputs<M, V>(phi_g, W_g, dWm_g, e0, a.np, kap, c);
+    fg.forward(kap, a.inv_tau);
+  }
   if (a.dW != nullptr) {
-    // dW = bf16(dWm * S) now, while mu is live anyway (dWm is re-read)
+    // dW = bf16(dWm * S) now, while the relaxation is live anyway (dWm is re-read)
 #pragma unroll
     for (int s = 0; s < M / 4; ++s) {
       if constexpr (L == 2) {
@@ -117,7 +199,7 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
       }
     }
   }
-  V dkv[M];
+  if constexpr (HIST) bwd_upstream<M, V>(W_g, dWm_g, c);
   fg.backward(c, a.inv_tau, dkv);
   // dL/dphi = dL/dkappa / lambda
 #pragma unroll
@@ -128,10 +210,21 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
 #pragma unroll
     for (int l = 0; l < M; ++l) dk[l] = lane_of(dkv[l], h);
     if ((fg.flag >> h) & 1u) {
+      // rare: the exact routine (with HIST from re-formed keys of this group; the
+      // opaque copy of the parameters keeps the compiler from holding the first
+      // keys live)
       float k[M], cc[M], S[M];
+      if constexpr (HIST) {
+        NoiseParams np = a.np;
+        asm volatile("" : "+r"(np.k0));
+        bwd_keys<M, float>(phi_g + h, e0 + h, np, k);
+      } else {
+#pragma unroll
+        for (int l = 0; l < M; ++l) k[l] = lane_of(kap[l], h);
+      }
 #pragma unroll
       for (int l = 0; l < M; ++l) {
-        k[l] = lane_of(kap[l], h) * kLn2;  // natural-log keys
+        k[l] *= kLn2;  // natural-log keys
         cc[l] = lane_of(c[l], h);
       }
       ExactGroup<N, M> ex;
@@ -186,9 +279,10 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_
           if constexpr (M == 4) {
             bwd_groups<N, M, TAU1, F2>(pp, pw, pd, e0, a);
           } else {
-            // M = 8: the paired step history does not fit the register file; one group at a time
-#pragma unroll 1
-            for (int h = 0; h < 2; ++h) bwd_groups<N, M, TAU1, float>(pp + h, pw + h, pd + h, e0 + h, a);
+            // M = 8: the paired step history does not fit the register file; steps
+            // 0 .. N-2 go to shared memory behind the tile ring
+            F2* hist = reinterpret_cast<F2*>(smem + kHistOffset<M>) + threadIdx.x;
+            bwd_groups<N, M, TAU1, F2, true>(pp, pw, pd, e0, a, hist);
           }
         }
       });
@@ -237,7 +331,7 @@ template <int N, int M, bool TAU1>
 int launch_tiles(const BwdArgs& a, cudaStream_t stream) {
   using C = Cfg<M>;
   auto kern = roi_bwd_kernel<N, M, TAU1>;
-  const size_t smem = tile_smem_bytes<C::kTile, C::kStages>(8);
+  const size_t smem = kHistBytes<N, M> > 0 ? kHistOffset<M> + kHistBytes<N, M> : tile_smem_bytes<C::kTile, C::kStages>(8);
   static LaunchCache cache;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return -1;

@@ -464,21 +464,58 @@ __device__ __forceinline__ V min_of(const V (&x)[M]) {
   return m;
 }
 
-template <int N, int M, bool TAU1, bool KEEP, class V = float>
+// Step history mu(k), k = 0 .. N-1, of a relaxation kept for the backward sweep:
+// in registers ...
+template <int N, int M, class V>
+struct RegSteps {
+  static constexpr bool kSmem = false;
+  V mu[N][M];
+  __device__ __forceinline__ void put(int k, int l, V v) { mu[k][l] = v; }
+  __device__ __forceinline__ V get(int k, int l) const { return mu[k][l]; }
+};
+// ... or steps 0 .. N-2 in shared memory and the last one in registers.  Slot
+// (k, l) of a thread is at[(k M + l) STRIDE]; with `at` = base + threadIdx.x and
+// STRIDE = threads per CTA a warp touches consecutive words.
+template <int N, int M, class V, int STRIDE>
+struct SmemSteps {
+  static constexpr bool kSmem = true;
+  V* at;
+  V last[M];
+  __device__ __forceinline__ void put(int k, int l, V v) {
+    if (k == N - 1) {
+      last[l] = v;
+    } else {
+      at[(k * M + l) * STRIDE] = v;
+    }
+  }
+  __device__ __forceinline__ V get(int k, int l) const {
+    return k == N - 1 ? last[l] : at[(k * M + l) * STRIDE];
+  }
+};
+
+template <int N, int M, bool TAU1, bool KEEP, class V = float,
+          class Steps = RegSteps<KEEP ? N : 1, KEEP ? M : 1, V>>
 struct FastGroup {
-  // KEEP: store mu of every step for a backward sweep (S is then re-summed from
-  // mu on demand, in the same order, instead of being kept live).
-  V mu[KEEP ? N : 1][M];
-  V S[KEEP ? 1 : M];
+  // KEEP: store mu of every step for a backward sweep.  With the history in
+  // registers S is re-summed from it on demand (in the order forward()
+  // accumulates it) instead of being kept live; with a shared-memory history S
+  // is accumulated as without KEEP.
+  static constexpr bool kSumS = !KEEP || Steps::kSmem;
+  Steps st;
+  V S[kSumS ? M : 1];
   V rt_last;  // tau = 1, KEEP: 1 / sum(mu om) of step N-2 (mu(N-1) = mu(N-2) om rt_last)
   uint32_t flag;
 
   // S_l of a KEEP run, summed exactly as forward() accumulates it.
   __device__ __forceinline__ V soft(int l) const {
-    V s = mu[0][l];
+    if constexpr (kSumS) {
+      return S[l];
+    } else {
+      V s = st.get(0, l);
 #pragma unroll
-    for (int k = 1; k < N; ++k) s = vadd(s, mu[KEEP ? k : 0][l]);
-    return s;
+      for (int k = 1; k < N; ++k) s = vadd(s, st.get(k, l));
+      return s;
+    }
   }
 
   // kap: the keys in log2 units (t = kappa log2 e).
@@ -508,11 +545,8 @@ struct FastGroup {
       for (int k = 0; k < N; ++k) {
 #pragma unroll
         for (int l = 0; l < M; ++l) {
-          if constexpr (KEEP) {
-            mu[k][l] = cur[l];
-          } else {
-            S[l] = k == 0 ? cur[l] : vadd(S[l], cur[l]);
-          }
+          if constexpr (KEEP) st.put(k, l, cur[l]);
+          if constexpr (kSumS) S[l] = k == 0 ? cur[l] : vadd(S[l], cur[l]);
         }
         if (k + 1 < N) {
           V o[M], v[M];
@@ -545,11 +579,8 @@ struct FastGroup {
 #pragma unroll
         for (int l = 0; l < M; ++l) {
           cur[l] = vmul(e[l], r);
-          if constexpr (KEEP) {
-            mu[k][l] = cur[l];
-          } else {
-            S[l] = k == 0 ? cur[l] : vadd(S[l], cur[l]);
-          }
+          if constexpr (KEEP) st.put(k, l, cur[l]);
+          if constexpr (kSumS) S[l] = k == 0 ? cur[l] : vadd(S[l], cur[l]);
         }
         if (k + 1 < N) {
           V ex[M];
@@ -576,22 +607,25 @@ struct FastGroup {
     {
       V cm[M];
 #pragma unroll
-      for (int l = 0; l < M; ++l) cm[l] = vmul(c[l], mu[N - 1][l]);
+      for (int l = 0; l < M; ++l) cm[l] = vmul(c[l], st.get(N - 1, l));
       const V cmu = sum_of(cm);
 #pragma unroll
       for (int l = 0; l < M; ++l) {
-        const V t = vmul(itau, vsub(c[l], cmu));
-        b[l] = vmul(mu[N - 1][l], t);
-        // tau = 1: b / om(N-2) = mu(N-2) rt_last (c - <c, mu(N-1)>) / tau, no division
-        if constexpr (TAU1 && N >= 2) hl[l] = vmul(vmul(mu[N - 2][l], rt_last), t);
+        V t = vsub(c[l], cmu);
+        if constexpr (!TAU1) t = vmul(itau, t);
+        b[l] = vmul(st.get(N - 1, l), t);
+        // tau = 1: b / om(N-2) = mu(N-2) rt_last (c - <c, mu(N-1)>), no division
+        if constexpr (TAU1 && N >= 2) hl[l] = vmul(vmul(st.get(N - 2, l), rt_last), t);
       }
     }
 #pragma unroll
     for (int k = N - 2; k >= 0; --k) {
-      V cm[M], h[M], H[M];
+      V mk[M], cm[M], h[M], H[M];
+#pragma unroll
+      for (int l = 0; l < M; ++l) mk[l] = st.get(k, l);
       if (!TAU1 || k != N - 2) {
         V om[M];
-        exclusive_sums(mu[k], om);
+        exclusive_sums(mk, om);
 #pragma unroll
         for (int l = 0; l < M; ++l) h[l] = vmul(b[l], vmap(om[l], rcp_approx));
       } else {
@@ -599,13 +633,15 @@ struct FastGroup {
         for (int l = 0; l < M; ++l) h[l] = hl[l];
       }
 #pragma unroll
-      for (int l = 0; l < M; ++l) cm[l] = vmul(c[l], mu[k][l]);
-      const V cmu = sum_of(cm);
-      const V B = sum_of(b);
+      for (int l = 0; l < M; ++l) cm[l] = vmul(c[l], mk[l]);
+      // c_l - <c, mu> + H_l - B as (c_l + H_l) - (<c, mu> + B)
+      const V K = vadd(sum_of(cm), sum_of(b));
       exclusive_sums(h, H);
 #pragma unroll
-      for (int l = 0; l < M; ++l)
-        b[l] = vfma(vmul(mu[k][l], itau), vsub(vadd(vsub(c[l], cmu), H[l]), B), b[l]);
+      for (int l = 0; l < M; ++l) {
+        const V mu_l = TAU1 ? mk[l] : vmul(mk[l], itau);
+        b[l] = vfma(mu_l, vsub(vadd(c[l], H[l]), K), b[l]);
+      }
     }
 #pragma unroll
     for (int l = 0; l < M; ++l) dk[l] = b[l];
