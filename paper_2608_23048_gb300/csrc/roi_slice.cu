@@ -1,10 +1,12 @@
 // Wide groups (M = 16, 32: the 8:16 and 16:32 patterns) on warp slices: the
-// M / 4 consecutive lanes of a slice hold one group, four elements each.  Same
-// method as the one-thread-per-group kernels (Sec. 4.2.2 Eq. 10-12, Algorithm 1;
-// Eq. 5; backward through the relaxation), with the per-group sums, maxima and
-// "sum of the other members" formed across the slice by a shuffle butterfly
-// that never subtracts.  Hard ranks compare every key of the group through
-// shuffles.  Groups whose exclusive sums underflow go to ExactGroup, run by the
+// SL = M / 4 consecutive lanes of a slice hold one group, four members each.  Same method as the
+// one-thread-per-group kernels (Sec. 4.2.2 Eq. 10-12, Algorithm 1; Eq. 5;
+// backward through the relaxation), with the per-group sums, maxima and "sum of
+// the other members" formed across the slice by a shuffle butterfly that never
+// subtracts.  A thread holds the slots t and t + 256 of a tile; where registers
+// allow, the two groups of those slots are relaxed in lockstep on packed FP32
+// (V = F2, one group per half), otherwise one after the other (V = float).
+// Groups whose keys leave the fast path's range go to ExactGroup, run by the
 // slice's first lane.
 #include "roi_launch.h"
 #include "roi_tiles.cuh"
@@ -13,34 +15,51 @@ namespace roi {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kTile = 2048;  // 512 four-element slots: two per thread
+constexpr int kTile = 2048;  // 512 four-member slots: slots t and t + 256 per thread
 constexpr int kStagesFwd = 4;
 constexpr int kStagesBwd = 3;
 
-template <int SL>
+// Pairing doubles the per-thread state: the forward pairs M = 16; the backward,
+// which keeps the N steps of the relaxation in registers, runs one group at a time.
+template <int M>
+constexpr bool kPairedFwd = M <= 16;
+constexpr int kMinBlocksFwd = 2;
+template <int M>
+constexpr int kMinBlocksBwd = M == 32 ? 1 : 2;
+
+__device__ __forceinline__ float shfl_xor(float v, int o) { return __shfl_xor_sync(0xffffffffu, v, o); }
+__device__ __forceinline__ F2 shfl_xor(F2 v, int o) {
+  return f2(__shfl_xor_sync(0xffffffffu, lo(v), o), __shfl_xor_sync(0xffffffffu, hi(v), o));
+}
+__device__ __forceinline__ float shfl_idx(float v, int src) { return __shfl_sync(0xffffffffu, v, src); }
+__device__ __forceinline__ F2 shfl_idx(F2 v, int src) {
+  return f2(__shfl_sync(0xffffffffu, lo(v), src), __shfl_sync(0xffffffffu, hi(v), src));
+}
+
+template <int SL, class V>
 struct Slice {
   static_assert(SL == 4 || SL == 8, "slices of 4 or 8 lanes");
   // Sum over the slice's other lanes (never total minus own) and the total,
   // identical on every lane of the slice.
-  __device__ __forceinline__ static float others(float p, float& tot) {
-    float oth = 0.f, acc = p;
+  __device__ __forceinline__ static V others(V p, V& tot) {
+    V oth = shfl_xor(p, 1), acc = vadd(p, oth);
 #pragma unroll
-    for (int o = 1; o < SL; o <<= 1) {
-      const float sib = __shfl_xor_sync(0xffffffffu, acc, o);
-      oth = __fadd_rn(oth, sib);
-      acc = __fadd_rn(acc, sib);
+    for (int o = 2; o < SL; o <<= 1) {
+      const V sib = shfl_xor(acc, o);
+      oth = vadd(oth, sib);
+      acc = vadd(acc, sib);
     }
     tot = acc;
     return oth;
   }
-  __device__ __forceinline__ static float total(float p) {
-    float t;
+  __device__ __forceinline__ static V total(V p) {
+    V t;
     others(p, t);
     return t;
   }
-  __device__ __forceinline__ static float max(float v) {
+  __device__ __forceinline__ static V max(V v) {
 #pragma unroll
-    for (int o = 1; o < SL; o <<= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    for (int o = 1; o < SL; o <<= 1) v = vmax(v, shfl_xor(v, o));
     return v;
   }
   __device__ __forceinline__ static uint32_t any(uint32_t f) {
@@ -50,18 +69,34 @@ struct Slice {
   }
 };
 
-__device__ __forceinline__ float sum4(const float (&x)[4]) {
-  return __fadd_rn(__fadd_rn(x[0], x[1]), __fadd_rn(x[2], x[3]));
+template <class V>
+__device__ __forceinline__ V sum4(const V (&x)[4]) {
+  return vadd(vadd(x[0], x[1]), vadd(x[2], x[3]));
 }
-__device__ __forceinline__ void excl4(const float (&x)[4], float oth, float (&ex)[4]) {
-  const float p01 = __fadd_rn(x[0], x[1]), p23 = __fadd_rn(x[2], x[3]);
-  ex[0] = __fadd_rn(__fadd_rn(x[1], p23), oth);
-  ex[1] = __fadd_rn(__fadd_rn(x[0], p23), oth);
-  ex[2] = __fadd_rn(__fadd_rn(p01, x[3]), oth);
-  ex[3] = __fadd_rn(__fadd_rn(p01, x[2]), oth);
+template <class V>
+__device__ __forceinline__ void excl4(const V (&x)[4], V oth, V (&ex)[4]) {
+  const V p01 = vadd(x[0], x[1]), p23 = vadd(x[2], x[3]);
+  ex[0] = vadd(vadd(x[1], p23), oth);
+  ex[1] = vadd(vadd(x[0], p23), oth);
+  ex[2] = vadd(vadd(p01, x[3]), oth);
+  ex[3] = vadd(vadd(p01, x[2]), oth);
 }
-__device__ __forceinline__ float max4(const float (&x)[4]) { return fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3])); }
-__device__ __forceinline__ float min4(const float (&x)[4]) { return fminf(fminf(x[0], x[1]), fminf(x[2], x[3])); }
+template <class V>
+__device__ __forceinline__ V max4(const V (&x)[4]) {
+  return vmax(vmax(x[0], x[1]), vmax(x[2], x[3]));
+}
+template <class V>
+__device__ __forceinline__ V min4(const V (&x)[4]) {
+  return vmin(vmin(x[0], x[1]), vmin(x[2], x[3]));
+}
+template <class V>
+__device__ __forceinline__ float lane_of(V v, int h) {
+  if constexpr (vlanes<V>() == 1) {
+    return v;
+  } else {
+    return h == 0 ? lo(v) : hi(v);
+  }
+}
 
 struct SliceArgs {
   const float* phi;
@@ -79,140 +114,165 @@ struct SliceArgs {
   unsigned int* status;
 };
 
-// Keys of one four-element slot starting at call-flat index e0, in log2 units
-// (t = kappa log2 e).
-__device__ __forceinline__ void slot_keys(const float* phi4, int64_t e0, const NoiseParams& np, float (&kap)[4]) {
-  const float4 p = *reinterpret_cast<const float4*>(phi4);
-  const uint4 x = noise_block_q(np, (np.e_base + uint64_t(e0)) >> 2);
-  kap[0] = key_log2(p.x, uniform_from_word(x.x), np.l2e_inv_lam);
-  kap[1] = key_log2(p.y, uniform_from_word(x.y), np.l2e_inv_lam);
-  kap[2] = key_log2(p.z, uniform_from_word(x.z), np.l2e_inv_lam);
-  kap[3] = key_log2(p.w, uniform_from_word(x.w), np.l2e_inv_lam);
+// Keys (log2 units, t = kappa log2 e) of L four-member slots (one per lane of V)
+// whose first elements have call-flat indices e0[h].
+template <class V>
+__device__ __forceinline__ void slot_keys(const float* const* p4, const int64_t* e0, const NoiseParams& np,
+                                          V (&kap)[4]) {
+  constexpr int L = vlanes<V>();
+  float ph[L][4];
+  uint32_t x[L][4];
+#pragma unroll
+  for (int h = 0; h < L; ++h) {
+    const float4 p = *reinterpret_cast<const float4*>(p4[h]);
+    ph[h][0] = p.x, ph[h][1] = p.y, ph[h][2] = p.z, ph[h][3] = p.w;
+    const uint4 q = noise_block_q(np, (np.e_base + uint64_t(e0[h])) >> 2);
+    x[h][0] = q.x, x[h][1] = q.y, x[h][2] = q.z, x[h][3] = q.w;
+  }
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    V one_plus, phv;
+    if constexpr (L == 1) {
+      one_plus = one_plus_from_word(x[0][j]);
+      phv = ph[0][j];
+    } else {
+      one_plus = f2(one_plus_from_word(x[0][j]), one_plus_from_word(x[1][j]));
+      phv = f2(ph[0][j], ph[1][j]);
+    }
+    const V u = vsub(one_plus, vconst<V>(__uint_as_float(0x3f7fffffu)));
+    kap[j] = key_log2(phv, u, np.l2e_inv_lam);
+  }
 }
 
-// Forward relaxation of the group held by this slice; mu of every step kept if
-// KEEP.  Returns the slice-uniform fallback flag.
-template <int N, int M, bool TAU1, bool KEEP>
+// Forward relaxation of the group(s) held by this slice; mu of every step kept
+// if KEEP.  forward() returns the fallback flags (bit h: lane h of V), uniform
+// over the slice.
+template <int N, int M, bool TAU1, bool KEEP, class V>
 struct SliceRelax {
   static constexpr int SL = M / 4;
-  float mu[KEEP ? N : 1][4];
-  float S[4];
-  float rt_last;
+  V mu[KEEP ? N : 1][4];
+  V S[4];
+  V rt_last;
 
-  __device__ __forceinline__ uint32_t forward(const float (&kap)[4], float inv_tau, int base_lane) {
+  __device__ __forceinline__ uint32_t forward(const V (&kap)[4], float inv_tau, int base_lane) {
     uint32_t flag = 0;
-    float cur[4];
+    V cur[4];
     if constexpr (TAU1) {
-      const float kref = __shfl_sync(0xffffffffu, kap[0], base_lane);
-      float e[4];
+      // weights relative to the slice's first key; a member more than 100 log2
+      // units from it (or a non-finite key) sends the group to the exact routine
+      const V kref = shfl_idx(kap[0], base_lane);
+      V e[4];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) e[j] = ex2_approx(__fsub_rn(kap[j], kref));
-      float tot;
-      Slice<SL>::others(sum4(e), tot);
-      flag = (!(min4(e) >= kTinyExcl) || !(tot <= 1.0f / kTinyExcl)) ? 1u : 0u;
-      const float r = rcp_approx(tot);
+      for (int j = 0; j < 4; ++j) e[j] = vmap(vsub(kap[j], kref), ex2_approx);
+      V tot;
+      Slice<SL, V>::others(sum4(e), tot);
+      flag = vbelow(min4(e), kTinyExcl) | vbelow(vsub(vconst<V>(1.0f / kTinyExcl), tot), 0.0f);
+      const V r = vmap(tot, rcp_approx);
 #pragma unroll
-      for (int j = 0; j < 4; ++j) cur[j] = __fmul_rn(e[j], r);
+      for (int j = 0; j < 4; ++j) cur[j] = vmul(e[j], r);
 #pragma unroll
       for (int k = 0; k < N; ++k) {
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           if constexpr (KEEP) mu[k][j] = cur[j];
-          S[j] = k == 0 ? cur[j] : __fadd_rn(S[j], cur[j]);
+          S[j] = k == 0 ? cur[j] : vadd(S[j], cur[j]);
         }
         if (k + 1 < N) {
-          float totc, o[4], v[4];
-          const float oth = Slice<SL>::others(sum4(cur), totc);
+          V totc, o[4], v[4];
+          const V oth = Slice<SL, V>::others(sum4(cur), totc);
           excl4(cur, oth, o);
 #pragma unroll
-          for (int j = 0; j < 4; ++j) v[j] = __fmul_rn(cur[j], o[j]);
-          const float rt = rcp_approx(Slice<SL>::total(sum4(v)));
+          for (int j = 0; j < 4; ++j) v[j] = vmul(cur[j], o[j]);
+          const V rt = vmap(Slice<SL, V>::total(sum4(v)), rcp_approx);
           if (k == N - 2) rt_last = rt;
 #pragma unroll
-          for (int j = 0; j < 4; ++j) cur[j] = __fmul_rn(v[j], rt);
+          for (int j = 0; j < 4; ++j) cur[j] = vmul(v[j], rt);
         }
       }
     } else {
-      const float kmax = Slice<SL>::max(max4(kap));
-      const float sc = inv_tau;
-      float d[4];
+      const V kmax = Slice<SL, V>::max(max4(kap));
+      const V sc = vconst<V>(inv_tau);
+      V d[4];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) d[j] = __fmul_rn(__fsub_rn(kap[j], kmax), sc);
-      if (!(kmax - kmax == 0.0f)) flag = 1u;
+      for (int j = 0; j < 4; ++j) d[j] = vmul(vsub(kap[j], kmax), sc);
+      flag = vbelow(vsub(kmax, kmax), 0.0f);  // non-finite maximum
 #pragma unroll
       for (int k = 0; k < N; ++k) {
-        float e[4];
+        V e[4];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) e[j] = ex2_approx(d[j]);
-        float tot;
-        const float oth = Slice<SL>::others(sum4(e), tot);
-        const float r = rcp_approx(tot);
+        for (int j = 0; j < 4; ++j) e[j] = vmap(d[j], ex2_approx);
+        V tot;
+        const V oth = Slice<SL, V>::others(sum4(e), tot);
+        const V r = vmap(tot, rcp_approx);
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          cur[j] = __fmul_rn(e[j], r);
+          cur[j] = vmul(e[j], r);
           if constexpr (KEEP) mu[k][j] = cur[j];
-          S[j] = k == 0 ? cur[j] : __fadd_rn(S[j], cur[j]);
+          S[j] = k == 0 ? cur[j] : vadd(S[j], cur[j]);
         }
         if (k + 1 < N) {
-          float ex[4];
+          V ex[4];
           excl4(e, oth, ex);
-          if (!(min4(ex) >= kTinyExcl)) flag = 1u;
+          flag |= vbelow(min4(ex), kTinyExcl);
 #pragma unroll
-          for (int j = 0; j < 4; ++j) d[j] = __fmaf_rn(lg2_approx(__fmul_rn(ex[j], r)), inv_tau, d[j]);
-          const float dm = Slice<SL>::max(max4(d));
+          for (int j = 0; j < 4; ++j) d[j] = vfma(vmap(vmul(ex[j], r), lg2_approx), sc, d[j]);
+          const V dm = Slice<SL, V>::max(max4(d));
 #pragma unroll
-          for (int j = 0; j < 4; ++j) d[j] = __fsub_rn(d[j], dm);
+          for (int j = 0; j < 4; ++j) d[j] = vsub(d[j], dm);
         }
       }
     }
-    return Slice<SL>::any(flag);
+    return Slice<SL, V>::any(flag);
   }
 
-  // dk = dL/dkappa of this slot's elements for c = dL/dS (same sweep as FastGroup).
-  __device__ __forceinline__ void backward(const float (&c)[4], float inv_tau, float (&dk)[4]) const {
+  // dk = dL/dkappa of this slot's members for c = dL/dS (the sweep of FastGroup).
+  __device__ __forceinline__ void backward(const V (&c)[4], float inv_tau, V (&dk)[4]) const {
     static_assert(KEEP, "needs the steps");
-    float b[4], hl[4];
+    const V itau = vconst<V>(inv_tau);
+    V b[4], hl[4];
     {
-      float cm[4];
+      V cm[4];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) cm[j] = __fmul_rn(c[j], mu[N - 1][j]);
-      const float cmu = Slice<SL>::total(sum4(cm));
+      for (int j = 0; j < 4; ++j) cm[j] = vmul(c[j], mu[N - 1][j]);
+      const V cmu = Slice<SL, V>::total(sum4(cm));
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
-        const float t = __fmul_rn(inv_tau, __fsub_rn(c[j], cmu));
-        b[j] = __fmul_rn(mu[N - 1][j], t);
-        if constexpr (TAU1) hl[j] = __fmul_rn(__fmul_rn(mu[N - 2][j], rt_last), t);
+        V t = vsub(c[j], cmu);
+        if constexpr (!TAU1) t = vmul(itau, t);
+        b[j] = vmul(mu[N - 1][j], t);
+        if constexpr (TAU1) hl[j] = vmul(vmul(mu[N - 2][j], rt_last), t);
       }
     }
 #pragma unroll
     for (int k = N - 2; k >= 0; --k) {
-      float cm[4], h[4], H[4];
+      V cm[4], h[4], H[4];
       if (TAU1 && k == N - 2) {
 #pragma unroll
         for (int j = 0; j < 4; ++j) h[j] = hl[j];
       } else {
-        float om[4], tmp;
-        excl4(mu[k], Slice<SL>::others(sum4(mu[k]), tmp), om);
+        V om[4], tmp;
+        excl4(mu[k], Slice<SL, V>::others(sum4(mu[k]), tmp), om);
 #pragma unroll
-        for (int j = 0; j < 4; ++j) h[j] = __fmul_rn(b[j], rcp_approx(om[j]));
+        for (int j = 0; j < 4; ++j) h[j] = vmul(b[j], vmap(om[j], rcp_approx));
       }
 #pragma unroll
-      for (int j = 0; j < 4; ++j) cm[j] = __fmul_rn(c[j], mu[k][j]);
-      const float cmu = Slice<SL>::total(sum4(cm));
-      const float B = Slice<SL>::total(sum4(b));
-      float tmp;
-      excl4(h, Slice<SL>::others(sum4(h), tmp), H);
+      for (int j = 0; j < 4; ++j) cm[j] = vmul(c[j], mu[k][j]);
+      // c_l - <c, mu> + H_l - B as (c_l + H_l) - (<c, mu> + B)
+      const V K = vadd(Slice<SL, V>::total(sum4(cm)), Slice<SL, V>::total(sum4(b)));
+      V tmp;
+      excl4(h, Slice<SL, V>::others(sum4(h), tmp), H);
 #pragma unroll
-      for (int j = 0; j < 4; ++j)
-        b[j] = __fmaf_rn(__fmul_rn(mu[k][j], inv_tau),
-                         __fsub_rn(__fadd_rn(__fsub_rn(c[j], cmu), H[j]), B), b[j]);
+      for (int j = 0; j < 4; ++j) {
+        const V mu_j = TAU1 ? mu[k][j] : vmul(mu[k][j], itau);
+        b[j] = vfma(mu_j, vsub(vadd(c[j], H[j]), K), b[j]);
+      }
     }
 #pragma unroll
     for (int j = 0; j < 4; ++j) dk[j] = b[j];
   }
 };
 
-// Hard bits of this slot: rank of each own key among the group's M keys.
+// Hard bits of a slot: rank of each own key among the group's M keys.
 template <int M>
 __device__ __forceinline__ uint32_t slice_topn_bits(const float (&kap)[4], int N, int base_lane, int q) {
   constexpr int SL = M / 4;
@@ -239,14 +299,28 @@ __device__ __forceinline__ uint32_t slice_topn_bits(const float (&kap)[4], int N
   return bits;
 }
 
-// Exact fallback for the whole group, run by one lane: natural-log keys of all
+// Hard bits of L slots (one per lane of V): comparison ranking per slot.
+template <int N, int M, class V>
+__device__ __forceinline__ void slot_topn(const V (&kap)[4], int base_lane, int q, uint32_t (&bits)[vlanes<V>()]) {
+#pragma unroll
+  for (int h = 0; h < vlanes<V>(); ++h) {
+    float k[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) k[j] = lane_of(kap[j], h);
+    bits[h] = slice_topn_bits<M>(k, N, base_lane, q);
+  }
+}
+
+// Exact fallback for one whole group, run by one lane: natural-log keys of all
 // M elements from logits at phi_g (call-flat index g0).
 template <int N, int M>
 __device__ __forceinline__ void group_keys_all(const float* phi_g, int64_t g0, const NoiseParams& np, float (&k)[M]) {
 #pragma unroll 1
   for (int s = 0; s < M / 4; ++s) {
+    const float* p[1] = {phi_g + 4 * s};
+    const int64_t e[1] = {g0 + 4 * s};
     float k4[4];
-    slot_keys(phi_g + 4 * s, g0 + 4 * s, np, k4);
+    slot_keys<float>(p, e, np, k4);
 #pragma unroll
     for (int j = 0; j < 4; ++j) k[4 * s + j] = k4[j] * kLn2;
   }
@@ -265,113 +339,171 @@ __device__ __forceinline__ void unpack_bf16x4(uint2 q, float (&out)[4]) {
   out[3] = bf16_bits_to_float(q.y >> 16);
 }
 
-// One slot of the forward.  si: slot index within the launch's element range
-// starting at `base` (call-flat); p/w: the slot's logits and weights (shared or
-// global memory).  All 32 lanes of the warp must call this together.
-template <int N, int M, bool TAU1>
-__device__ __forceinline__ void fwd_slot(const float* p, const uint16_t* w, int64_t e0, bool active, const SliceArgs& a) {
+// Forward of L slots (one per lane of V; p/w: each slot's logits and weights in
+// shared or global memory, e0: call-flat index of its first element).  All 32
+// lanes of the warp call this together; inactive slots (ragged tail, V = float
+// only) take part in the shuffles with zero keys.  Returns each slot's hard bits.
+template <int N, int M, bool TAU1, class V>
+__device__ __forceinline__ void fwd_slots(const float* const* p, const uint16_t* const* w, const int64_t* e0,
+                                          bool active, const SliceArgs& a, uint32_t (&bits)[vlanes<V>()]) {
   constexpr int SL = M / 4;
+  constexpr int L = vlanes<V>();
   const int lane = threadIdx.x & 31;
   const int q = lane % SL;
   const int base_lane = lane - q;
-  float kap[4] = {0.f, 0.f, 0.f, 0.f};
-  if (active) slot_keys(p, e0, a.np, kap);
-  const uint32_t bits = slice_topn_bits<M>(kap, N, base_lane, q);
-  SliceRelax<N, M, TAU1, false> rx;
-  const uint32_t flag = rx.forward(kap, a.inv_tau, base_lane);
+  V kap[4];
   if (active) {
-    if (!flag) {
-      float wv[4];
-      unpack_bf16x4(*reinterpret_cast<const uint2*>(w), wv);
-      *reinterpret_cast<uint2*>(a.Wm + e0) = pack4(wv, rx.S);
-      if (a.soft != nullptr) *reinterpret_cast<float4*>(a.soft + e0) = make_float4(rx.S[0], rx.S[1], rx.S[2], rx.S[3]);
+    slot_keys<V>(p, e0, a.np, kap);
+  } else {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) kap[j] = vconst<V>(0.0f);
+  }
+  slot_topn<N, M, V>(kap, base_lane, q, bits);
+  SliceRelax<N, M, TAU1, false, V> rx;
+  const uint32_t flag = rx.forward(kap, a.inv_tau, base_lane);
+  if (!active) return;
+#pragma unroll
+  for (int h = 0; h < L; ++h) {
+    if (!((flag >> h) & 1u)) {
+      float wv[4], sv[4];
+      unpack_bf16x4(*reinterpret_cast<const uint2*>(w[h]), wv);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) sv[j] = lane_of(rx.S[j], h);
+      *reinterpret_cast<uint2*>(a.Wm + e0[h]) = pack4(wv, sv);
+      if (a.soft != nullptr) *reinterpret_cast<float4*>(a.soft + e0[h]) = make_float4(sv[0], sv[1], sv[2], sv[3]);
     } else if (q == 0) {
       float k[M], S[M];
-      group_keys_all<N, M>(p, e0, a.np, k);
+      group_keys_all<N, M>(p[h], e0[h], a.np, k);
       ExactGroup<N, M> ex;
       ex.forward(k, N, M, a.tau, S);
 #pragma unroll 1
       for (int s = 0; s < SL; ++s) {
         float wv[4], sv[4];
-        unpack_bf16x4(*reinterpret_cast<const uint2*>(w + 4 * s), wv);
+        unpack_bf16x4(*reinterpret_cast<const uint2*>(w[h] + 4 * s), wv);
 #pragma unroll
         for (int j = 0; j < 4; ++j) sv[j] = S[4 * s + j];
-        *reinterpret_cast<uint2*>(a.Wm + e0 + 4 * s) = pack4(wv, sv);
-        if (a.soft != nullptr) *reinterpret_cast<float4*>(a.soft + e0 + 4 * s) = make_float4(sv[0], sv[1], sv[2], sv[3]);
+        *reinterpret_cast<uint2*>(a.Wm + e0[h] + 4 * s) = pack4(wv, sv);
+        if (a.soft != nullptr)
+          *reinterpret_cast<float4*>(a.soft + e0[h] + 4 * s) = make_float4(sv[0], sv[1], sv[2], sv[3]);
       }
     }
   }
-  if (a.hard != nullptr) {
-    // 8 lanes hold the 32 elements of a word
-    uint32_t v = active ? bits << ((lane & 7) * 4) : 0u;
-    v |= __shfl_xor_sync(0xffffffffu, v, 1);
-    v |= __shfl_xor_sync(0xffffffffu, v, 2);
-    v |= __shfl_xor_sync(0xffffffffu, v, 4);
-    if (active && (lane & 7) == 0) a.hard[e0 >> 5] = v;
-  }
 }
 
-template <int N, int M, bool TAU1>
-__device__ __forceinline__ void bwd_slot(const float* p, const uint16_t* w, const uint16_t* dw, int64_t e0, bool active,
-                                         const SliceArgs& a) {
+// Backward of L slots (as fwd_slots).
+template <int N, int M, bool TAU1, class V>
+__device__ __forceinline__ void bwd_slots(const float* const* p, const uint16_t* const* w, const uint16_t* const* dw,
+                                          const int64_t* e0, bool active, const SliceArgs& a) {
   constexpr int SL = M / 4;
+  constexpr int L = vlanes<V>();
   const int lane = threadIdx.x & 31;
   const int q = lane % SL;
   const int base_lane = lane - q;
-  float kap[4] = {0.f, 0.f, 0.f, 0.f}, c[4] = {0.f, 0.f, 0.f, 0.f};
+  V kap[4], c[4];
   if (active) {
-    slot_keys(p, e0, a.np, kap);
-    float wv[4], dv[4];
-    unpack_bf16x4(*reinterpret_cast<const uint2*>(w), wv);
-    unpack_bf16x4(*reinterpret_cast<const uint2*>(dw), dv);
+    slot_keys<V>(p, e0, a.np, kap);
+    float wv[L][4], dv[L][4];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) c[j] = __fmul_rn(dv[j], wv[j]);
+    for (int h = 0; h < L; ++h) {
+      unpack_bf16x4(*reinterpret_cast<const uint2*>(w[h]), wv[h]);
+      unpack_bf16x4(*reinterpret_cast<const uint2*>(dw[h]), dv[h]);
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      if constexpr (L == 1) {
+        c[j] = vmul(dv[0][j], wv[0][j]);
+      } else {
+        c[j] = vmul(f2(dv[0][j], dv[1][j]), f2(wv[0][j], wv[1][j]));
+      }
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) kap[j] = c[j] = vconst<V>(0.0f);
   }
-  SliceRelax<N, M, TAU1, true> rx;
+  SliceRelax<N, M, TAU1, true, V> rx;
   const uint32_t flag = rx.forward(kap, a.inv_tau, base_lane);
-  if (active && !flag && a.dW != nullptr) {
-    float dv[4];
-    unpack_bf16x4(*reinterpret_cast<const uint2*>(dw), dv);
-    *reinterpret_cast<uint2*>(a.dW + e0) = pack4(dv, rx.S);
+  if (active && a.dW != nullptr) {
+#pragma unroll
+    for (int h = 0; h < L; ++h) {
+      if (!((flag >> h) & 1u)) {
+        float dv[4], sv[4];
+        unpack_bf16x4(*reinterpret_cast<const uint2*>(dw[h]), dv);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) sv[j] = lane_of(rx.S[j], h);
+        *reinterpret_cast<uint2*>(a.dW + e0[h]) = pack4(dv, sv);
+      }
+    }
   }
-  float dk[4];
+  V dk[4];
   rx.backward(c, a.inv_tau, dk);
   if (!active) return;
-  if (!flag) {
-    *reinterpret_cast<float4*>(a.dphi + e0) =
-        make_float4(dk[0] * a.np.inv_lam, dk[1] * a.np.inv_lam, dk[2] * a.np.inv_lam, dk[3] * a.np.inv_lam);
-  } else if (q == 0) {
-    float k[M], cc[M], S[M], dkk[M];
-    group_keys_all<N, M>(p, e0, a.np, k);
-#pragma unroll 1
-    for (int s = 0; s < SL; ++s) {
-      float wv[4], dv[4];
-      unpack_bf16x4(*reinterpret_cast<const uint2*>(w + 4 * s), wv);
-      unpack_bf16x4(*reinterpret_cast<const uint2*>(dw + 4 * s), dv);
 #pragma unroll
-      for (int j = 0; j < 4; ++j) cc[4 * s + j] = __fmul_rn(dv[j], wv[j]);
-    }
-    ExactGroup<N, M> ex;
-    ex.forward(k, N, M, a.tau, S);
-    ex.backward(cc, N, M, a.tau, dkk);
-#pragma unroll 1
-    for (int s = 0; s < SL; ++s) {
-      *reinterpret_cast<float4*>(a.dphi + e0 + 4 * s) =
-          make_float4(dkk[4 * s] * a.np.inv_lam, dkk[4 * s + 1] * a.np.inv_lam, dkk[4 * s + 2] * a.np.inv_lam,
-                      dkk[4 * s + 3] * a.np.inv_lam);
-      if (a.dW != nullptr) {
-        float dv[4], sv[4];
-        unpack_bf16x4(*reinterpret_cast<const uint2*>(dw + 4 * s), dv);
+  for (int j = 0; j < 4; ++j) dk[j] = vmul(dk[j], vconst<V>(a.np.inv_lam));
 #pragma unroll
-        for (int j = 0; j < 4; ++j) sv[j] = S[4 * s + j];
-        *reinterpret_cast<uint2*>(a.dW + e0 + 4 * s) = pack4(dv, sv);
+  for (int h = 0; h < L; ++h) {
+    if (!((flag >> h) & 1u)) {
+      *reinterpret_cast<float4*>(a.dphi + e0[h]) =
+          make_float4(lane_of(dk[0], h), lane_of(dk[1], h), lane_of(dk[2], h), lane_of(dk[3], h));
+    } else if (q == 0) {
+      float k[M], cc[M], S[M], dkk[M];
+      group_keys_all<N, M>(p[h], e0[h], a.np, k);
+#pragma unroll 1
+      for (int s = 0; s < SL; ++s) {
+        float wv[4], dv[4];
+        unpack_bf16x4(*reinterpret_cast<const uint2*>(w[h] + 4 * s), wv);
+        unpack_bf16x4(*reinterpret_cast<const uint2*>(dw[h] + 4 * s), dv);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) cc[4 * s + j] = __fmul_rn(dv[j], wv[j]);
+      }
+      ExactGroup<N, M> ex;
+      ex.forward(k, N, M, a.tau, S);
+      ex.backward(cc, N, M, a.tau, dkk);
+#pragma unroll 1
+      for (int s = 0; s < SL; ++s) {
+        *reinterpret_cast<float4*>(a.dphi + e0[h] + 4 * s) =
+            make_float4(__fmul_rn(dkk[4 * s], a.np.inv_lam), __fmul_rn(dkk[4 * s + 1], a.np.inv_lam),
+                        __fmul_rn(dkk[4 * s + 2], a.np.inv_lam), __fmul_rn(dkk[4 * s + 3], a.np.inv_lam));
+        if (a.dW != nullptr) {
+          float dv[4], sv[4];
+          unpack_bf16x4(*reinterpret_cast<const uint2*>(dw[h] + 4 * s), dv);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) sv[j] = S[4 * s + j];
+          *reinterpret_cast<uint2*>(a.dW + e0[h] + 4 * s) = pack4(dv, sv);
+        }
       }
     }
   }
 }
 
+// Hard words of one slot per lane (8 lanes fill a word).
+__device__ __forceinline__ void store_hard_slot(uint32_t* hard, int64_t e0, uint32_t bits, bool active) {
+  const int lane = threadIdx.x & 31;
+  uint32_t v = active ? bits << ((lane & 7) * 4) : 0u;
+  v |= __shfl_xor_sync(0xffffffffu, v, 1);
+  v |= __shfl_xor_sync(0xffffffffu, v, 2);
+  v |= __shfl_xor_sync(0xffffffffu, v, 4);
+  if (active && (lane & 7) == 0) hard[e0 >> 5] = v;
+}
+// The same for the two slots of a thread (first elements e0a, e0b; all lanes
+// active): both masks travel in one register, the first slot's in the low
+// half-word; after the shuffles within each 4-lane half, one exchange between
+// the halves completes the first slot's word on lane 0 of the 8 and the second
+// slot's word on lane 4.
+__device__ __forceinline__ void store_hard_slot_pair(uint32_t* hard, int64_t e0a, int64_t e0b, uint32_t bits_a,
+                                                     uint32_t bits_b) {
+  const int lane = threadIdx.x & 31;
+  const int sh = (lane & 3) * 4;
+  uint32_t v = (bits_a << sh) | (bits_b << (16 + sh));
+  v |= __shfl_xor_sync(0xffffffffu, v, 1);
+  v |= __shfl_xor_sync(0xffffffffu, v, 2);
+  const uint32_t o = __shfl_xor_sync(0xffffffffu, v, 4);
+  const bool upper = (lane & 4) != 0;
+  const uint32_t word = __byte_perm(v, o, upper ? 0x3276u : 0x5410u);
+  if ((lane & 3) == 0) hard[(upper ? e0b : e0a) >> 5] = word;
+}
+
 template <int N, int M, bool TAU1>
-__global__ void __launch_bounds__(kThreads, 2) roi_slice_fwd_kernel(SliceArgs a) {
+__global__ void __launch_bounds__(kThreads, kMinBlocksFwd) roi_slice_fwd_kernel(SliceArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   TileSrc<2> src;
   src.ptr[0] = reinterpret_cast<const uint8_t*>(a.phi);
@@ -383,11 +515,22 @@ __global__ void __launch_bounds__(kThreads, 2) roi_slice_fwd_kernel(SliceArgs a)
         const float* sphi = reinterpret_cast<const float*>(stage[0]);
         const uint16_t* sW = reinterpret_cast<const uint16_t*>(stage[1]);
         const int64_t base = tile * kTile;
+        const int s0 = threadIdx.x, s1 = threadIdx.x + kThreads;
+        const float* pp[2] = {sphi + 4 * s0, sphi + 4 * s1};
+        const uint16_t* pw[2] = {sW + 4 * s0, sW + 4 * s1};
+        const int64_t e0[2] = {base + 4 * s0, base + 4 * s1};
+        uint32_t bits[2];
+        if constexpr (kPairedFwd<M>) {
+          fwd_slots<N, M, TAU1, F2>(pp, pw, e0, true, a, bits);
+        } else {
 #pragma unroll 1
-        for (int j = 0; j < 2; ++j) {
-          const int si = threadIdx.x + j * kThreads;
-          fwd_slot<N, M, TAU1>(sphi + 4 * si, sW + 4 * si, base + 4 * si, true, a);
+          for (int j = 0; j < 2; ++j) {
+            uint32_t b1[1];
+            fwd_slots<N, M, TAU1, float>(pp + j, pw + j, e0 + j, true, a, b1);
+            bits[j] = b1[0];
+          }
         }
+        if (a.hard != nullptr) store_hard_slot_pair(a.hard, e0[0], e0[1], bits[0], bits[1]);
       });
   if (!ok) return;
   if (blockIdx.x == gridDim.x - 1) {
@@ -397,13 +540,18 @@ __global__ void __launch_bounds__(kThreads, 2) roi_slice_fwd_kernel(SliceArgs a)
       const int64_t si = threadIdx.x + r * kThreads;
       const bool active = si < slots;
       const int64_t off = t0 + 4 * (active ? si : 0);
-      fwd_slot<N, M, TAU1>(a.phi + off, a.W + off, t0 + 4 * si, active, a);
+      const float* pp[1] = {a.phi + off};
+      const uint16_t* pw[1] = {a.W + off};
+      const int64_t e0[1] = {t0 + 4 * si};
+      uint32_t bits[1];
+      fwd_slots<N, M, TAU1, float>(pp, pw, e0, active, a, bits);
+      if (a.hard != nullptr) store_hard_slot(a.hard, e0[0], bits[0], active);
     }
   }
 }
 
 template <int N, int M, bool TAU1>
-__global__ void __launch_bounds__(kThreads, M == 32 ? 1 : 2) roi_slice_bwd_kernel(SliceArgs a) {
+__global__ void __launch_bounds__(kThreads, kMinBlocksBwd<M>) roi_slice_bwd_kernel(SliceArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   TileSrc<3> src;
   src.ptr[0] = reinterpret_cast<const uint8_t*>(a.phi);
@@ -418,11 +566,13 @@ __global__ void __launch_bounds__(kThreads, M == 32 ? 1 : 2) roi_slice_bwd_kerne
         const uint16_t* sW = reinterpret_cast<const uint16_t*>(stage[1]);
         const uint16_t* sdW = reinterpret_cast<const uint16_t*>(stage[2]);
         const int64_t base = tile * kTile;
+        const int s0 = threadIdx.x, s1 = threadIdx.x + kThreads;
+        const float* pp[2] = {sphi + 4 * s0, sphi + 4 * s1};
+        const uint16_t* pw[2] = {sW + 4 * s0, sW + 4 * s1};
+        const uint16_t* pd[2] = {sdW + 4 * s0, sdW + 4 * s1};
+        const int64_t e0[2] = {base + 4 * s0, base + 4 * s1};
 #pragma unroll 1
-        for (int j = 0; j < 2; ++j) {
-          const int si = threadIdx.x + j * kThreads;
-          bwd_slot<N, M, TAU1>(sphi + 4 * si, sW + 4 * si, sdW + 4 * si, base + 4 * si, true, a);
-        }
+        for (int j = 0; j < 2; ++j) bwd_slots<N, M, TAU1, float>(pp + j, pw + j, pd + j, e0 + j, true, a);
       });
   if (!ok) return;
   if (blockIdx.x == gridDim.x - 1) {
@@ -432,7 +582,11 @@ __global__ void __launch_bounds__(kThreads, M == 32 ? 1 : 2) roi_slice_bwd_kerne
       const int64_t si = threadIdx.x + r * kThreads;
       const bool active = si < slots;
       const int64_t off = t0 + 4 * (active ? si : 0);
-      bwd_slot<N, M, TAU1>(a.phi + off, a.W + off, a.dWm + off, t0 + 4 * si, active, a);
+      const float* pp[1] = {a.phi + off};
+      const uint16_t* pw[1] = {a.W + off};
+      const uint16_t* pd[1] = {a.dWm + off};
+      const int64_t e0[1] = {t0 + 4 * si};
+      bwd_slots<N, M, TAU1, float>(pp, pw, pd, e0, active, a);
     }
   }
 }
@@ -469,6 +623,15 @@ int slice_bwd(const SliceArgs& a, cudaStream_t stream) {
   return launch_persistent(roi_slice_bwd_kernel<N, M, TAU1>, cache, tile_smem_bytes<kTile, kStagesBwd>(8), a, stream);
 }
 
+template <int N, int M>
+int slice_fwd_nm(const SliceArgs& a, cudaStream_t stream) {
+  return a.tau == 1.0f ? slice_fwd<N, M, true>(a, stream) : slice_fwd<N, M, false>(a, stream);
+}
+template <int N, int M>
+int slice_bwd_nm(const SliceArgs& a, cudaStream_t stream) {
+  return a.tau == 1.0f ? slice_bwd<N, M, true>(a, stream) : slice_bwd<N, M, false>(a, stream);
+}
+
 }  // namespace
 
 bool slice_supported(int N, int M) { return (N == 8 && M == 16) || (N == 16 && M == 32); }
@@ -486,9 +649,8 @@ int launch_slice_fwd(const FwdCall& c) {
   a.inv_tau = 1.0f / c.tau;
   a.np = c.np;
   a.status = c.status;
-  const bool t1 = c.tau == 1.0f;
-  if (c.N == 8 && c.M == 16) return t1 ? slice_fwd<8, 16, true>(a, c.stream) : slice_fwd<8, 16, false>(a, c.stream);
-  if (c.N == 16 && c.M == 32) return t1 ? slice_fwd<16, 32, true>(a, c.stream) : slice_fwd<16, 32, false>(a, c.stream);
+  if (c.N == 8 && c.M == 16) return slice_fwd_nm<8, 16>(a, c.stream);
+  if (c.N == 16 && c.M == 32) return slice_fwd_nm<16, 32>(a, c.stream);
   return -1;
 }
 
@@ -505,9 +667,8 @@ int launch_slice_bwd(const BwdCall& c) {
   a.inv_tau = 1.0f / c.tau;
   a.np = c.np;
   a.status = c.status;
-  const bool t1 = c.tau == 1.0f;
-  if (c.N == 8 && c.M == 16) return t1 ? slice_bwd<8, 16, true>(a, c.stream) : slice_bwd<8, 16, false>(a, c.stream);
-  if (c.N == 16 && c.M == 32) return t1 ? slice_bwd<16, 32, true>(a, c.stream) : slice_bwd<16, 32, false>(a, c.stream);
+  if (c.N == 8 && c.M == 16) return slice_bwd_nm<8, 16>(a, c.stream);
+  if (c.N == 16 && c.M == 32) return slice_bwd_nm<16, 32>(a, c.stream);
   return -1;
 }
 
