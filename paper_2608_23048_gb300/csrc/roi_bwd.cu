@@ -15,10 +15,11 @@ namespace {
 // shared-memory stages, and the CTAs per SM the register budget is sized for.
 template <int M>
 struct Cfg {
-  // M = 8: the paired sweep needs ~170 registers; 128 threads x 3 CTAs per SM
-  static constexpr int kThreads = M == 4 ? 256 : 128;
-  static constexpr int kPairs = 1;
-  static constexpr int kStages = M == 4 ? 3 : 2;
+  // M = 8: the paired sweep needs ~170 registers (3 CTAs per SM); M = 4: three
+  // pairs per thread with up to 128 registers (4 CTAs per SM)
+  static constexpr int kThreads = 128;
+  static constexpr int kPairs = M == 4 ? 3 : 1;
+  static constexpr int kStages = 2;  // 48 KB per CTA (M = 4), 32 KB + step history (M = 8)
   static constexpr int kMinBlocks = M == 4 ? 4 : 3;
   static constexpr int kTile = 2 * kPairs * kThreads * M;  // elements
 };

@@ -618,8 +618,7 @@ struct FastGroup {
         if constexpr (TAU1 && N >= 2) hl[l] = vmul(vmul(st.get(N - 2, l), rt_last), t);
       }
     }
-#pragma unroll
-    for (int k = N - 2; k >= 0; --k) {
+    auto sweep = [&](int k) {
       V mk[M], cm[M], h[M], H[M];
 #pragma unroll
       for (int l = 0; l < M; ++l) mk[l] = st.get(k, l);
@@ -642,7 +641,9 @@ struct FastGroup {
         const V mu_l = TAU1 ? mk[l] : vmul(mk[l], itau);
         b[l] = vfma(mu_l, vsub(vadd(c[l], H[l]), K), b[l]);
       }
-    }
+    };
+#pragma unroll
+    for (int k = N - 2; k >= 0; --k) sweep(k);
 #pragma unroll
     for (int l = 0; l < M; ++l) dk[l] = b[l];
   }

@@ -13,9 +13,9 @@ namespace {
 // shared-memory stages, and the CTAs per SM the register budget is sized for.
 template <int M>
 struct Cfg {
-  static constexpr int kThreads = 256;
-  static constexpr int kPairs = M == 4 ? 2 : 1;
-  static constexpr int kStages = 2;  // 48 KB per CTA (M = 4) or 48 KB (M = 8)
+  static constexpr int kThreads = M == 4 ? 128 : 256;
+  static constexpr int kPairs = M == 4 ? 3 : 1;
+  static constexpr int kStages = 2;  // 36 KB per CTA (M = 4) or 48 KB (M = 8)
   static constexpr int kMinBlocks = M == 4 ? 4 : 2;
   static constexpr int kTile = 2 * kPairs * kThreads * M;  // elements
 };
