@@ -114,23 +114,23 @@ __device__ __forceinline__ float uniform_from_word(uint32_t x) {
 
 // E = -ln(u) for u in [2^-24, 1) with a small relative error everywhere,
 // including u -> 1 where E -> 0 (the hardware log2 has an absolute error floor
-// there).  Method: u = 2^e m with e = rint(log2 u) and m = u 2^-e in
-// [sqrt(1/2), sqrt(2)], so ln u = e ln2 + ln m; ln m = 2 atanh(s),
-// s = (m - 1) / (m + 1), |s| < 0.172,
+// there).  Method: u = 2^e m with m in [sqrt(1/2), sqrt(2)), split exactly from
+// the float's bits (subtracting the bits of sqrt(1/2) makes the exponent field
+// round log2 u to the nearest integer at the sqrt(2) boundaries), so
+// ln u = e ln2 + ln m; ln m = 2 atanh(s), s = (m - 1) / (m + 1), |s| < 0.172,
 // 2 atanh(s) = 2s + (2/3)s^3 + (2/5)s^5 + (2/7)s^7 + (2/9)s^9 + O(s^11)
-// (truncation below 2^-28 relative).  e comes from the hardware log2 rounded to
-// the nearest integer (its error only moves m across the boundary of the
-// interval when log2 u is within 2^-22 of a half-integer, which the series
-// tolerates); 2^-e from the hardware exp2, exact on integers (verified on the
-// GPU for all integers in [-100, 127]); m - 1 is exact (Sterbenz).  The Horner
+// (truncation below 2^-28 relative).  m - 1 is exact (Sterbenz).  The Horner
 // chain runs on negated coefficients so the result needs no final negation.
+__device__ __forceinline__ int rounded_exponent(float x) {
+  return int(__float_as_uint(x) - 0x3f3504f3u) >> 23;  // 0x3f3504f3: sqrt(1/2)
+}
 template <class V>
 __device__ __forceinline__ V neg_log_unit(V u) {
-  const V y = vmap(u, lg2_approx);
-  const V tt = vadd(y, vconst<V>(12582912.0f));               // 1.5 * 2^23: rounds y to an integer
-  const V ef = vsub(tt, vconst<V>(12582912.0f));              // e = rint(log2 u)
-  const V p2 = vmap(vsub(vconst<V>(12582912.0f), tt), ex2_approx);  // 2^-e, exact
-  const V m = vmul(u, p2);                                     // exact power-of-two scaling
+  // m = u 2^-e (the exponent field moved by e) and e as a float (the integer
+  // added into the mantissa of 1.5 * 2^23)
+  const V m = vmap(u, [](float x) { return __uint_as_float(__float_as_uint(x) - (uint32_t(rounded_exponent(x)) << 23)); });
+  const V ef = vsub(vmap(u, [](float x) { return __int_as_float(rounded_exponent(x) + 0x4B400000); }),
+                    vconst<V>(12582912.0f));
   const V one = vconst<V>(1.0f);
   const V f = vsub(m, one);
   const V s = vmul(f, vmap(vadd(m, one), rcp_approx));
@@ -527,9 +527,11 @@ struct FastGroup {
       // normalised next).  A group with a key more than 100 (log2 units, ~69
       // natural) from the first one, or with a non-finite key, goes to the exact
       // routine: the squared offsets are summed on the FMA pipe and compared once.
+      // (a non-finite first key makes every offset non-finite, so it is caught too)
       V e[M], x[M];
+      e[0] = vconst<V>(1.0f);
 #pragma unroll
-      for (int l = 0; l < M; ++l) {
+      for (int l = 1; l < M; ++l) {
         x[l] = vsub(kap[l], kap[0]);
         e[l] = vmap(x[l], ex2_approx);
       }
@@ -543,10 +545,13 @@ struct FastGroup {
       for (int l = 0; l < M; ++l) cur[l] = vmul(e[l], r);
 #pragma unroll
       for (int k = 0; k < N; ++k) {
+        // without KEEP the last step is added into S as it is formed (one fma)
+        if (KEEP || k == 0 || k + 1 < N) {
 #pragma unroll
-        for (int l = 0; l < M; ++l) {
-          if constexpr (KEEP) st.put(k, l, cur[l]);
-          if constexpr (kSumS) S[l] = k == 0 ? cur[l] : vadd(S[l], cur[l]);
+          for (int l = 0; l < M; ++l) {
+            if constexpr (KEEP) st.put(k, l, cur[l]);
+            if constexpr (kSumS) S[l] = k == 0 ? cur[l] : vadd(S[l], cur[l]);
+          }
         }
         if (k + 1 < N) {
           V o[M], v[M];
@@ -557,8 +562,13 @@ struct FastGroup {
           if constexpr (KEEP) {
             if (k == N - 2) rt_last = rt;
           }
+          if (!KEEP && k + 2 == N) {
 #pragma unroll
-          for (int l = 0; l < M; ++l) cur[l] = vmul(v[l], rt);
+            for (int l = 0; l < M; ++l) S[l] = vfma(v[l], rt, S[l]);
+          } else {
+#pragma unroll
+            for (int l = 0; l < M; ++l) cur[l] = vmul(v[l], rt);
+          }
         }
       }
     } else {
@@ -576,11 +586,17 @@ struct FastGroup {
 #pragma unroll
         for (int l = 0; l < M; ++l) e[l] = vmap(d[l], ex2_approx);
         const V r = vmap(sum_of(e), rcp_approx);
+        if (!KEEP && k > 0 && k + 1 == N) {
+          // last step without KEEP: added into S as it is formed (one fma)
 #pragma unroll
-        for (int l = 0; l < M; ++l) {
-          cur[l] = vmul(e[l], r);
-          if constexpr (KEEP) st.put(k, l, cur[l]);
-          if constexpr (kSumS) S[l] = k == 0 ? cur[l] : vadd(S[l], cur[l]);
+          for (int l = 0; l < M; ++l) S[l] = vfma(e[l], r, S[l]);
+        } else {
+#pragma unroll
+          for (int l = 0; l < M; ++l) {
+            cur[l] = vmul(e[l], r);
+            if constexpr (KEEP) st.put(k, l, cur[l]);
+            if constexpr (kSumS) S[l] = k == 0 ? cur[l] : vadd(S[l], cur[l]);
+          }
         }
         if (k + 1 < N) {
           V ex[M];
