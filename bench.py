@@ -422,7 +422,9 @@ def run_ours(args):
 def run_e2e(args, roi, tensors, lset, N, M, tau, dev, world):
     """Same step through the C ABI with host buffers: per tensor, copy logits, W and
     dWm from pinned host memory, run fwd + bwd, copy Wm, the hard bits and the logit
-    gradients back; two streams alternate so copies overlap compute."""
+    gradients back.  Three streams form a pipeline (host->device copies, kernels,
+    device->host copies) ordered by per-tensor events, so both copy directions and
+    the kernels overlap."""
     import torch
     host = {}
     for t in tensors:
@@ -434,24 +436,37 @@ def run_e2e(args, roi, tensors, lset, N, M, tau, dev, world):
             "Wm": torch.empty_like(t["Wm"], device="cpu").pin_memory(),
             "hard": torch.empty_like(t["hard"], device="cpu").pin_memory(),
             "dphi": torch.empty_like(t["dphi"], device="cpu").pin_memory()}
-    streams = [torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)]
+    s_in, s_run, s_out = (torch.cuda.Stream(device=dev) for _ in range(3))
+    ev_in = [torch.cuda.Event() for _ in tensors]
+    ev_run = [torch.cuda.Event() for _ in tensors]
+    ev_out = [torch.cuda.Event() for _ in tensors]
     h2d = sum(t["rows"] * t["cols"] * 8 for t in tensors)
     d2h = sum(t["rows"] * t["cols"] * 6 + t["hard"].numel() * 4 for t in tensors)
+    started = [False]
 
     def one(s):
         for i, t in enumerate(tensors):
             hs = host[t["id"] % len(WL.PROJS)]
-            stm = streams[i % 2]
             st = roi.NoiseState(0, s, t["id"], 1.0, 0)
-            with torch.cuda.stream(stm):
+            with torch.cuda.stream(s_in):
+                if started[0]:
+                    s_in.wait_event(ev_out[i])  # the previous step is done with this tensor's buffers
                 t["phi"].copy_(hs["phi"], non_blocking=True)
                 t["W"].copy_(hs["W"], non_blocking=True)
                 t["dWm"].copy_(hs["dWm"], non_blocking=True)
-                roi.roi_mask_fwd_ex(t["phi"], t["W"], N, M, tau, st, t["Wm"], None, t["hard"], stream=stm)
-                roi.roi_mask_bwd(t["phi"], t["W"], st, N, M, t["dWm"], tau, t["dphi"], None, stream=stm)
+                ev_in[i].record(s_in)
+            with torch.cuda.stream(s_run):
+                s_run.wait_event(ev_in[i])
+                roi.roi_mask_fwd_ex(t["phi"], t["W"], N, M, tau, st, t["Wm"], None, t["hard"], stream=s_run)
+                roi.roi_mask_bwd(t["phi"], t["W"], st, N, M, t["dWm"], tau, t["dphi"], None, stream=s_run)
+                ev_run[i].record(s_run)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(ev_run[i])
                 hs["Wm"].copy_(t["Wm"], non_blocking=True)
                 hs["hard"].copy_(t["hard"], non_blocking=True)
                 hs["dphi"].copy_(t["dphi"], non_blocking=True)
+                ev_out[i].record(s_out)
+        started[0] = True
 
     one(10_000)
     torch.cuda.synchronize()
