@@ -13,14 +13,14 @@ namespace {
 // Launch shape per group size M: threads per CTA, pairs of groups per thread per
 // tile (the two groups of a pair are relaxed in lockstep on packed FP32),
 // shared-memory stages, and the CTAs per SM the register budget is sized for.
+// One CTA per SM (see roi_fwd.cu): M = 4 with two pairs per thread and up to 128
+// registers; M = 8, whose paired sweep needs ~170 registers, with 384 threads.
 template <int M>
 struct Cfg {
-  // M = 8: the paired sweep needs ~170 registers (3 CTAs per SM); M = 4: three
-  // pairs per thread with up to 128 registers (4 CTAs per SM)
-  static constexpr int kThreads = 128;
-  static constexpr int kPairs = M == 4 ? 3 : 1;
-  static constexpr int kStages = 2;  // 48 KB per CTA (M = 4), 32 KB + step history (M = 8)
-  static constexpr int kMinBlocks = M == 4 ? 4 : 3;
+  static constexpr int kThreads = M == 4 ? 512 : 384;
+  static constexpr int kPairs = M == 4 ? 2 : 1;
+  static constexpr int kStages = M == 4 ? 3 : 2;  // 192 KB (M = 4), 96 KB + 72 KB step history (M = 8)
+  static constexpr int kMinBlocks = 1;
   static constexpr int kTile = 2 * kPairs * kThreads * M;  // elements
 };
 // Byte offset of the shared-memory step history (M = 8) behind the tile ring,

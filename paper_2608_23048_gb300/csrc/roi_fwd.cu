@@ -11,12 +11,15 @@ namespace {
 // Launch shape per group size M: threads per CTA, pairs of groups per thread per
 // tile (the two groups of a pair are relaxed in lockstep on packed FP32, F2),
 // shared-memory stages, and the CTAs per SM the register budget is sized for.
+// One CTA per SM: CTAs sharing an SM progress at very different rates (the
+// scheduler favours the older one) and the last ones then finish alone, so all of
+// an SM's warps work through one tile ring instead.
 template <int M>
 struct Cfg {
-  static constexpr int kThreads = M == 4 ? 128 : 256;
+  static constexpr int kThreads = 512;
   static constexpr int kPairs = M == 4 ? 3 : 1;
-  static constexpr int kStages = 2;  // 36 KB per CTA (M = 4) or 48 KB (M = 8)
-  static constexpr int kMinBlocks = M == 4 ? 4 : 2;
+  static constexpr int kStages = 2;  // 144 KB (M = 4) or 96 KB (M = 8)
+  static constexpr int kMinBlocks = 1;
   static constexpr int kTile = 2 * kPairs * kThreads * M;  // elements
 };
 
