@@ -426,16 +426,18 @@ __device__ __forceinline__ void exclusive_sums(const V (&x)[M], V (&ex)[M]) {
     ex[2] = vadd(p01, x[3]);
     ex[3] = vadd(p01, x[2]);
   } else {
+    // pair sums, then each pair's exclusive sum (the other three pairs), then the partner
     const V p01 = vadd(x[0], x[1]), p23 = vadd(x[2], x[3]), p45 = vadd(x[4], x[5]), p67 = vadd(x[6], x[7]);
     const V q0 = vadd(p01, p23), q1 = vadd(p45, p67);
-    ex[0] = vadd(vadd(x[1], p23), q1);
-    ex[1] = vadd(vadd(x[0], p23), q1);
-    ex[2] = vadd(vadd(p01, x[3]), q1);
-    ex[3] = vadd(vadd(p01, x[2]), q1);
-    ex[4] = vadd(vadd(x[5], p67), q0);
-    ex[5] = vadd(vadd(x[4], p67), q0);
-    ex[6] = vadd(vadd(p45, x[7]), q0);
-    ex[7] = vadd(vadd(p45, x[6]), q0);
+    const V e01 = vadd(p23, q1), e23 = vadd(p01, q1), e45 = vadd(q0, p67), e67 = vadd(q0, p45);
+    ex[0] = vadd(x[1], e01);
+    ex[1] = vadd(x[0], e01);
+    ex[2] = vadd(x[3], e23);
+    ex[3] = vadd(x[2], e23);
+    ex[4] = vadd(x[5], e45);
+    ex[5] = vadd(x[4], e45);
+    ex[6] = vadd(x[7], e67);
+    ex[7] = vadd(x[6], e67);
   }
 }
 
@@ -647,10 +649,10 @@ struct FastGroup {
 #pragma unroll
         for (int l = 0; l < M; ++l) h[l] = hl[l];
       }
+      // c_l - <c, mu> + H_l - B as (c_l + H_l) - K, K = <c, mu> + B = sum of (c mu + b)
 #pragma unroll
-      for (int l = 0; l < M; ++l) cm[l] = vmul(c[l], mk[l]);
-      // c_l - <c, mu> + H_l - B as (c_l + H_l) - (<c, mu> + B)
-      const V K = vadd(sum_of(cm), sum_of(b));
+      for (int l = 0; l < M; ++l) cm[l] = vfma(c[l], mk[l], b[l]);
+      const V K = sum_of(cm);
       exclusive_sums(h, H);
 #pragma unroll
       for (int l = 0; l < M; ++l) {

@@ -255,10 +255,10 @@ struct SliceRelax {
 #pragma unroll
         for (int j = 0; j < 4; ++j) h[j] = vmul(b[j], vmap(om[j], rcp_approx));
       }
+      // c_l - <c, mu> + H_l - B as (c_l + H_l) - K, K = <c, mu> + B = sum of (c mu + b)
 #pragma unroll
-      for (int j = 0; j < 4; ++j) cm[j] = vmul(c[j], mu[k][j]);
-      // c_l - <c, mu> + H_l - B as (c_l + H_l) - (<c, mu> + B)
-      const V K = vadd(Slice<SL, V>::total(sum4(cm)), Slice<SL, V>::total(sum4(b)));
+      for (int j = 0; j < 4; ++j) cm[j] = vfma(c[j], mu[k][j], b[j]);
+      const V K = Slice<SL, V>::total(sum4(cm));
       V tmp;
       excl4(h, Slice<SL, V>::others(sum4(h), tmp), H);
 #pragma unroll
