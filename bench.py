@@ -402,6 +402,28 @@ def run_ours(args):
                 "bwd_ms_per_step": round(1e3 * bwd_t / args.steps, 3),
                 "step_gbs": round(step_gbs / world, 1), "step_frac": round(step_gbs / world / peak, 4)}
 
+    # per-step device time: first forward launch to last backward launch of each step
+    T = len(tensors)
+    step_ms = sorted(ev[0][s * T].elapsed_time(ev[3][s * T + T - 1]) for s in range(args.steps))
+    pct = lambda q: round(step_ms[min(len(step_ms) - 1, int(q * (len(step_ms) - 1) + 0.5))], 3)
+    step_stats = {"p10": pct(0.1), "median": pct(0.5), "p90": pct(0.9)}
+
+    # the hard masks change with the step and each step reproduces (outside the timed region)
+    t0 = tensors[0]
+    last = args.warmup + args.steps - 1
+    h_last = t0["hard"].clone()
+    scratch_Wm = torch.empty_like(t0["Wm"])
+    h_again = torch.empty_like(t0["hard"])
+    h_prev = torch.empty_like(t0["hard"])
+    other = last - 1 if last > 0 else last + 1
+    for s_, out_h in ((last, h_again), (other, h_prev)):
+        st = roi.NoiseState(0, s_, t0["id"], 1.0, 0)
+        roi.roi_mask_fwd_ex(t0["phi"], t0["W"], N, M, tau, st, scratch_Wm, None, out_h, stream=stream)
+    torch.cuda.synchronize()
+    checks = {"step_reproducible": bool(torch.equal(h_again, h_last)),
+              "masks_differ_across_steps": bool(not torch.equal(h_prev, h_last)),
+              "checked_on": f"tensor {t0['id']} ({t0['rows']}x{t0['cols']}), steps {other} and {last}"}
+
     e2e = None
     if not args.no_e2e:
         e2e = run_e2e(args, roi, tensors, lset, N, M, tau, dev, world)
@@ -412,7 +434,7 @@ def run_ours(args):
                "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": cfg,
                "hbm_gbs": round(step_gbs, 1), "hbm_frac": round(step_gbs / world / peak, 4),
                "roofline": roofline, "cpu_baseline": base, "e2e": e2e,
-               "gpu_launches": int(launches), "clocks": clocks.summary(),
+               "gpu_launches": int(launches), "step_ms": step_stats, "checks": checks, "clocks": clocks.summary(),
                "clocks_note": "sampled with nvidia-smi every 100 ms during the timed region"}
         print(json.dumps(out), flush=True)
     if world > 1:
