@@ -321,3 +321,75 @@ def hard_mask_export(logits, N, M, W_bits=None):
         wb = np.asarray(W_bits, dtype=np.uint16).ravel()
         out["W_pruned"] = np.where(hard, wb, np.uint16(0)).reshape(rows, cols)
     return out
+
+
+def mask_fwd_st(logits, W_bits, N, M, tau, seed, step, tensor_id=0, lam=1.0,
+                row_offset=0, dtype=np.float64):
+    """Forward of the straight-through Gumbel-top-N variant (Appendix, "Comparison
+    with Straight-Through Gumbel-Top-K"): the forward applies the discrete mask,
+    argtop_N of the Gumbel-perturbed keys, so Wm = W where the hard mask is set and
+    +0 elsewhere (the bf16 bits of W copied); S is still formed (the backward runs
+    through it) and is returned like the soft forward's."""
+    out = mask_fwd(logits, W_bits, N, M, tau, seed, step, tensor_id, lam, row_offset, dtype)
+    wb = np.asarray(W_bits, dtype=np.uint16).reshape(out["hard"].shape)
+    out["Wm"] = np.where(out["hard"], wb, np.uint16(0))
+    return out
+
+
+def mask_bwd_st(logits, W_bits, dWm_bits, hard_bits, N, M, tau, seed, step, tensor_id=0,
+                lam=1.0, row_offset=0, dtype=np.float64):
+    """Backward of the straight-through variant (same appendix): the logit gradient
+    passes through the continuous relaxation exactly as in the soft method
+    (dL/dS = dWm * W), while the weight gradient follows the forward's actual
+    product W * hard: dW = dWm where the forward's hard mask is set, +0 elsewhere.
+    `hard_bits` are the forward's packed hard-mask words."""
+    out = mask_bwd(logits, W_bits, dWm_bits, N, M, tau, seed, step, tensor_id, lam, row_offset, dtype)
+    rows, cols = np.asarray(logits).shape
+    hard = unpack_bits(np.asarray(hard_bits, dtype=np.uint32), rows * cols).reshape(rows, cols)
+    db = np.asarray(dWm_bits, dtype=np.uint16).reshape(rows, cols)
+    out["dW"] = np.where(hard, db, np.uint16(0))
+    return out
+
+
+def export_compressed_2of4(logits, W_bits):
+    """2:4 deployment export in compressed form (the semi-structured layout that
+    sparse tensor cores consume, Sec. 1 and the Throughput appendix): per group of
+    four, the deployment mask argtop_2(phi) (ties: lower index) selects two
+    members, and
+      * values[g] = the two kept weights, in index order  -> bf16 [rows, cols/2]
+      * meta: the two in-group indices i0 < i1 as a 4-bit code i0 | i1 << 2, eight
+        groups per uint32 word, group g in bits 4*(g % 8) .. 4*(g % 8) + 3 of word
+        g // 8 (groups in row-major order)              -> uint32 [rows*cols/32]
+    """
+    logits = np.asarray(logits, dtype=np.float32)
+    rows, cols = logits.shape
+    _check(rows, cols, 2, 4)
+    if (rows * cols) % 32:
+        raise ValueError("rows * cols must be a multiple of 32 (eight groups per metadata word)")
+    hard = hard_topn(_grouped(logits.ravel(), 4), 2)                 # [G, 4] bool
+    G = hard.shape[0]
+    wb = np.asarray(W_bits, dtype=np.uint16).reshape(G, 4)
+    values = np.empty((G, 2), dtype=np.uint16)
+    codes = np.empty(G, dtype=np.uint32)
+    for g in range(G):                                               # plain loop: obviously correct
+        idx = [j for j in range(4) if hard[g, j]]
+        values[g] = wb[g, idx]
+        codes[g] = idx[0] | (idx[1] << 2)
+    meta = np.zeros(G // 8, dtype=np.uint32)
+    for g in range(G):
+        meta[g // 8] |= codes[g] << np.uint32(4 * (g % 8))
+    return {"values": values.reshape(rows, cols // 2), "meta": meta, "hard": hard.reshape(rows, cols)}
+
+
+def decompress_2of4(values, meta, rows, cols):
+    """Inverse of export_compressed_2of4's layout: dense bf16 bits with the kept
+    values at their indices and +0 elsewhere."""
+    G = rows * cols // 4
+    v = np.asarray(values, dtype=np.uint16).reshape(G, 2)
+    m = np.asarray(meta, dtype=np.uint32)
+    dense = np.zeros((G, 4), dtype=np.uint16)
+    for g in range(G):
+        code = (int(m[g // 8]) >> (4 * (g % 8))) & 0xF
+        dense[g, code & 3] = v[g, 0]
+        dense[g, code >> 2] = v[g, 1]
+    return dense.reshape(rows, cols)
