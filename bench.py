@@ -52,6 +52,9 @@ def parse_args():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--layers", type=int, default=None, help="only the first L layers (profiling cases)")
     p.add_argument("--proj", default=None, help="comma-separated projections to keep, e.g. gate")
+    p.add_argument("--op", choices=("mask", "st", "export2of4"), default="mask",
+                   help="mask: the fwd+bwd step (default); st: the straight-through pair with dW; "
+                        "export2of4: the compressed 2:4 export (one GPU)")
     return p.parse_args()
 
 
@@ -509,10 +512,115 @@ def run_e2e(args, roi, tensors, lset, N, M, tau, dev, world):
             "note": "host buffers: one layer's tensors in pinned memory, reused for all layers"}
 
 
+ST_FWD_BYTES = FWD_BYTES
+ST_BWD_BYTES = BWD_BYTES + 2 + 1 / 8   # + dW out, + the forward's hard bits in
+EXPORT_2OF4_BYTES = 4 + 2 + 1 + 1 / 8  # logits, W in; kept values, index codes out
+
+
+def run_variant(args):
+    """The straight-through pair (roi_mask_fwd_st + roi_mask_bwd_st with dW) or the
+    compressed 2:4 export over the layer set: device-resident inputs, per-launch CUDA
+    events, algorithmic bytes against the measured copy bandwidth.  One GPU."""
+    import torch
+    if int(os.environ.get("RANK", "0")) != 0:
+        return
+    cfg = config_for(args)
+    N, M, tau = cfg["N"], cfg["M"], cfg["tau"]
+    if args.op == "export2of4" and (N, M) != (2, 4):
+        raise SystemExit("--op export2of4 needs --nm 2:4")
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    from paper_2608_23048_gb300 import _build
+    _build.build()
+    import paper_2608_23048_gb300 as roi
+    kind = WL.CONFIGS[args.set].logits
+    tensors = []
+    for layer, p, rows, cols in selected_tensors(args):
+        W, phi, dWm = WL.make_inputs(rows, cols, kind, WL.tensor_seed(layer, p), device=dev)
+        t = {"id": layer * len(WL.PROJS) + p, "rows": rows, "cols": cols, "phi": phi, "W": W, "dWm": dWm}
+        if args.op == "st":
+            t.update(Wm=torch.empty_like(W), dphi=torch.empty_like(phi), dW=torch.empty_like(W),
+                     hard=torch.empty(roi.hard_words(rows, cols), dtype=torch.int32, device=dev))
+        else:
+            t.update(values=torch.empty(rows, cols // 2, dtype=torch.bfloat16, device=dev),
+                     meta=torch.empty(rows * cols // 32, dtype=torch.int32, device=dev))
+        tensors.append(t)
+    stream = torch.cuda.Stream(device=dev)
+
+    def launches(s, ev):
+        def rec(lst):
+            if ev is not None:
+                lst.append(torch.cuda.Event(enable_timing=True))
+                lst[-1].record(stream)
+        for t in tensors:
+            st = roi.NoiseState(0, s, t["id"], 1.0, 0)
+            rec(ev[0] if ev else None)
+            if args.op == "st":
+                roi.roi_mask_fwd_st(t["phi"], t["W"], N, M, tau, st, t["Wm"], None, t["hard"], stream=stream)
+            else:
+                roi.roi_export_compressed_2of4(t["phi"], t["W"], t["values"], t["meta"], stream=stream)
+            rec(ev[1] if ev else None)
+        if args.op == "st":
+            for t in reversed(tensors):
+                st = roi.NoiseState(0, s, t["id"], 1.0, 0)
+                rec(ev[2] if ev else None)
+                roi.roi_mask_bwd_st(t["phi"], t["W"], st, N, M, t["dWm"], t["hard"], tau, t["dphi"], t["dW"],
+                                    stream=stream)
+                rec(ev[3] if ev else None)
+
+    for w in range(args.warmup):
+        launches(w, None)
+    torch.cuda.synchronize()
+    roi.roi_device_status(stream)
+    ev = ([], [], [], [])
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(0) as clocks:
+        start.record(stream)
+        for s in range(args.steps):
+            launches(args.warmup + s, ev)
+        end.record(stream)
+        torch.cuda.synchronize()
+    roi.roi_device_status(stream)
+    elapsed = start.elapsed_time(end) / 1e3
+    a_t = sum(x.elapsed_time(y) for x, y in zip(ev[0], ev[1])) / 1e3
+    b_t = sum(x.elapsed_time(y) for x, y in zip(ev[2], ev[3])) / 1e3
+    E = cfg["elements"]
+    peak, peak_kind = hbm_peak()
+    if args.op == "st":
+        a_gbs = E * ST_FWD_BYTES * args.steps / a_t / 1e9
+        b_gbs = E * ST_BWD_BYTES * args.steps / b_t / 1e9
+        dom = "bwd" if b_t >= a_t else "fwd"
+        achieved, per = (b_gbs, ST_BWD_BYTES) if dom == "bwd" else (a_gbs, ST_FWD_BYTES)
+        step_bytes = ST_FWD_BYTES + ST_BWD_BYTES
+        extra = {"fwd_gbs": round(a_gbs, 1), "bwd_gbs": round(b_gbs, 1),
+                 "fwd_ms_per_step": round(1e3 * a_t / args.steps, 3), "bwd_ms_per_step": round(1e3 * b_t / args.steps, 3)}
+        kernel = f"roi_{dom}_kernel<{N},{M},{'tau1' if tau == 1.0 else 'tau'}> (straight-through)"
+        metric = "straight-through RoI mask fwd+bwd (dW on) groups/s and HBM GB/s, 1 GPU"
+    else:
+        achieved = E * EXPORT_2OF4_BYTES * args.steps / a_t / 1e9
+        per, step_bytes = EXPORT_2OF4_BYTES, EXPORT_2OF4_BYTES
+        extra = {"ms_per_step": round(1e3 * a_t / args.steps, 3)}
+        kernel = "roi_export_2of4_kernel"
+        metric = "compressed 2:4 export groups/s and HBM GB/s, 1 GPU"
+    step_gbs = E * step_bytes * args.steps / elapsed / 1e9
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "traffic": None, "kernel": kernel, "peak_kind": peak_kind,
+                "algorithmic_bytes_per_element": per, "step_gbs": round(step_gbs, 1),
+                "step_frac": round(step_gbs / peak, 4), **extra}
+    cfg = dict(cfg, op=args.op)
+    print(json.dumps({"metric": metric, "value": (E // M) * args.steps / elapsed, "unit": "groups/s",
+                      "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+                      "ms_per_step": 1e3 * elapsed / args.steps, "higher_is_better": True, "scaling": "weak",
+                      "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": cfg,
+                      "roofline": roofline, "clocks": clocks.summary()}), flush=True)
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         run_reference(args)
+    elif args.op != "mask":
+        run_variant(args)
     else:
         run_ours(args)
 

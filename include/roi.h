@@ -104,6 +104,38 @@ roi_status roi_mask_bwd(const float* logits, const roi_bf16* W, const roi_noise_
                         int N, int M, const roi_bf16* dWm, float tau, int64_t rows, int64_t cols,
                         float* out_dlogits, roi_bf16* out_dW, void* stream);
 
+/* Straight-through Gumbel-top-N variant (Appendix, "Comparison with
+ * Straight-Through Gumbel-Top-K": the forward applies the discrete mask, the
+ * backward propagates through the continuous relaxation).
+ *  roi_mask_fwd_st: as roi_mask_fwd_ex, except out_Wm copies the bf16 bits of W
+ *    where the hard mask (Gumbel-top-N of the keys, as out_hard) is set and
+ *    writes +0 elsewhere.  out_soft, when given, is the relaxation's S.
+ *  roi_mask_bwd_st: as roi_mask_bwd (out_dlogits identical: dL/dS = dWm * W
+ *    through the relaxation), except out_dW = dWm where the forward's hard mask
+ *    is set, +0 elsewhere, the gradient of the forward's product W * hard.
+ *    hard: the forward's out_hard words ([ceil(rows*cols/32)] uint32, same
+ *    noise state); required when out_dW is given, read only then. */
+roi_status roi_mask_fwd_st(const float* logits, const roi_bf16* W, int N, int M, float tau,
+                           const roi_noise_state* st, int64_t rows, int64_t cols,
+                           roi_bf16* out_Wm, float* out_soft, uint32_t* out_hard, void* stream);
+roi_status roi_mask_bwd_st(const float* logits, const roi_bf16* W, const roi_noise_state* st,
+                           int N, int M, const roi_bf16* dWm, const uint32_t* hard, float tau,
+                           int64_t rows, int64_t cols, float* out_dlogits, roi_bf16* out_dW,
+                           void* stream);
+
+/* Compressed 2:4 export for semi-structured sparse inference (the deployment the
+ * paper targets, Sec. 1 and the Throughput appendix; it gives no format, so this
+ * is the library's): the deployment mask argtop_2(phi) of every group of four
+ * (as roi_hard_mask_export with N = 2, M = 4) and
+ *  out_values [rows, cols/2] bf16   the two kept weights of each group, in index order
+ *  out_meta   [rows*cols/32] uint32 per group the in-group indices i0 < i1 as the
+ *             4-bit code i0 | i1 << 2; group g (row-major) in bits 4*(g%8) ..
+ *             4*(g%8)+3 of word g/8.  This is the content of the sparse tensor
+ *             cores' 2-bit index metadata without their hardware interleave.
+ * cols % 4 == 0 and rows*cols % 32 == 0 (else ROI_ERR_SHAPE). */
+roi_status roi_export_compressed_2of4(const float* logits, const roi_bf16* W, int64_t rows, int64_t cols,
+                                      roi_bf16* out_values, uint32_t* out_meta, void* stream);
+
 /* Deployment mask (Sec. 4.2.3 anneals lambda towards 0; the limit of
  * Gumbel-top-N is the deterministic top-N of phi, which is also the most
  * probable subset of Eq. 8): argtop_N(phi) per group, NaN ranked as -inf,

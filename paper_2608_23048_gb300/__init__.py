@@ -16,6 +16,7 @@ __all__ = [
     "RoiError", "NoiseState", "lib", "roi_mask_fwd", "roi_mask_fwd_ex", "roi_mask_bwd",
     "roi_hard_mask_export", "roi_device_status", "roi_status_string", "roi_launch_count",
     "library_path", "hard_words", "roi_noise_words", "roi_gumbel_noise",
+    "roi_mask_fwd_st", "roi_mask_bwd_st", "roi_export_compressed_2of4",
 ]
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
@@ -55,6 +56,9 @@ def lib() -> ctypes.CDLL:
     L.roi_mask_fwd.argtypes = [_P, _P, i32, i32, f32, u64, u32, i64, i64, _P, _P, _P, _P]
     L.roi_mask_fwd_ex.argtypes = [_P, _P, i32, i32, f32, ctypes.POINTER(NoiseState), i64, i64, _P, _P, _P, _P]
     L.roi_mask_bwd.argtypes = [_P, _P, ctypes.POINTER(NoiseState), i32, i32, _P, f32, i64, i64, _P, _P, _P]
+    L.roi_mask_fwd_st.argtypes = [_P, _P, i32, i32, f32, ctypes.POINTER(NoiseState), i64, i64, _P, _P, _P, _P]
+    L.roi_mask_bwd_st.argtypes = [_P, _P, ctypes.POINTER(NoiseState), i32, i32, _P, _P, f32, i64, i64, _P, _P, _P]
+    L.roi_export_compressed_2of4.argtypes = [_P, _P, i64, i64, _P, _P, _P]
     L.roi_hard_mask_export.argtypes = [_P, i32, i32, i64, i64, _P, _P, _P, _P]
     L.roi_device_status.argtypes = [_P]
     L.roi_noise_words.argtypes = [ctypes.POINTER(NoiseState), i64, i64, _P, _P]
@@ -64,7 +68,8 @@ def lib() -> ctypes.CDLL:
     L.roi_launch_count.argtypes = []
     L.roi_launch_count.restype = ctypes.c_uint64
     for name in ("roi_mask_fwd", "roi_mask_fwd_ex", "roi_mask_bwd", "roi_hard_mask_export", "roi_device_status",
-                 "roi_noise_words", "roi_gumbel_noise"):
+                 "roi_noise_words", "roi_gumbel_noise", "roi_mask_fwd_st", "roi_mask_bwd_st",
+                 "roi_export_compressed_2of4"):
         getattr(L, name).restype = i32
     _LIB = L
     return L
@@ -159,6 +164,51 @@ def roi_mask_bwd(logits, W, state: NoiseState, N, M, dWm, tau, out_dlogits, out_
     s = lib().roi_mask_bwd(_ptr(logits), _ptr(W), ctypes.byref(st), int(N), int(M), _ptr(dWm), float(tau),
                            rows, cols, _ptr(out_dlogits), _ptr(out_dW), _stream(stream))
     _raise(s, "roi_mask_bwd")
+
+
+def roi_mask_fwd_st(logits, W, N, M, tau, state: NoiseState, out_Wm, out_soft=None, out_hard=None, stream=None):
+    """Straight-through forward: Wm = W where the Gumbel-top-N hard mask is set, +0 elsewhere."""
+    import torch
+    rows, cols = logits.shape
+    _check_tensor(logits, "logits", torch.float32)
+    _check_tensor(W, "W", torch.bfloat16, (rows, cols))
+    _check_tensor(out_Wm, "out_Wm", torch.bfloat16, (rows, cols))
+    _check_tensor(out_soft, "out_soft", torch.float32, (rows, cols))
+    _check_tensor(out_hard, "out_hard", torch.int32, (hard_words(rows, cols),))
+    st = state if isinstance(state, NoiseState) else NoiseState(*state)
+    s = lib().roi_mask_fwd_st(_ptr(logits), _ptr(W), int(N), int(M), float(tau), ctypes.byref(st), rows, cols,
+                              _ptr(out_Wm), _ptr(out_soft), _ptr(out_hard), _stream(stream))
+    _raise(s, "roi_mask_fwd_st")
+
+
+def roi_mask_bwd_st(logits, W, state: NoiseState, N, M, dWm, hard, tau, out_dlogits, out_dW=None, stream=None):
+    """Straight-through backward: logit gradients through the relaxation; dW = dWm where
+    the forward's hard mask (`hard`, its out_hard words) is set."""
+    import torch
+    rows, cols = logits.shape
+    _check_tensor(logits, "logits", torch.float32)
+    _check_tensor(W, "W", torch.bfloat16, (rows, cols))
+    _check_tensor(dWm, "dWm", torch.bfloat16, (rows, cols))
+    _check_tensor(hard, "hard", torch.int32, (hard_words(rows, cols),))
+    _check_tensor(out_dlogits, "out_dlogits", torch.float32, (rows, cols))
+    _check_tensor(out_dW, "out_dW", torch.bfloat16, (rows, cols))
+    st = state if isinstance(state, NoiseState) else NoiseState(*state)
+    s = lib().roi_mask_bwd_st(_ptr(logits), _ptr(W), ctypes.byref(st), int(N), int(M), _ptr(dWm), _ptr(hard),
+                              float(tau), rows, cols, _ptr(out_dlogits), _ptr(out_dW), _stream(stream))
+    _raise(s, "roi_mask_bwd_st")
+
+
+def roi_export_compressed_2of4(logits, W, out_values, out_meta, stream=None):
+    """Compressed 2:4 export: kept weights [rows, cols/2] and 4-bit index codes, 8 groups per word."""
+    import torch
+    rows, cols = logits.shape
+    _check_tensor(logits, "logits", torch.float32)
+    _check_tensor(W, "W", torch.bfloat16, (rows, cols))
+    _check_tensor(out_values, "out_values", torch.bfloat16, (rows, cols // 2))
+    _check_tensor(out_meta, "out_meta", torch.int32, ((rows * cols) // 32,))
+    s = lib().roi_export_compressed_2of4(_ptr(logits), _ptr(W), rows, cols, _ptr(out_values), _ptr(out_meta),
+                                         _stream(stream))
+    _raise(s, "roi_export_compressed_2of4")
 
 
 def roi_hard_mask_export(logits, N, M, out_bits, W=None, out_Wpruned=None, stream=None):

@@ -95,9 +95,9 @@ using namespace roi;
 
 extern "C" {
 
-roi_status roi_mask_fwd_ex(const float* logits, const roi_bf16* W, int N, int M, float tau,
-                           const roi_noise_state* st, int64_t rows, int64_t cols, roi_bf16* out_Wm,
-                           float* out_soft, uint32_t* out_hard, void* stream) {
+static roi_status mask_fwd(const float* logits, const roi_bf16* W, int N, int M, float tau, const roi_noise_state* st,
+                           int64_t rows, int64_t cols, roi_bf16* out_Wm, float* out_soft, uint32_t* out_hard,
+                           bool straight_through, void* stream) {
   if (st == nullptr) return ROI_ERR_NULL;
   roi_status s = check_common(N, M, tau, rows, cols);
   if (s != ROI_OK) return s;
@@ -118,6 +118,7 @@ roi_status roi_mask_fwd_ex(const float* logits, const roi_bf16* W, int N, int M,
   c.Wm = out_Wm;
   c.soft = out_soft;
   c.hard = out_hard;
+  c.st = straight_through;
   c.E = E;
   c.N = N;
   c.M = M;
@@ -127,6 +128,18 @@ roi_status roi_mask_fwd_ex(const float* logits, const roi_bf16* W, int N, int M,
   if (c.status == nullptr) return ROI_ERR_CUDA;
   c.stream = static_cast<cudaStream_t>(stream);
   return finish(launch_fwd(c));
+}
+
+roi_status roi_mask_fwd_ex(const float* logits, const roi_bf16* W, int N, int M, float tau,
+                           const roi_noise_state* st, int64_t rows, int64_t cols, roi_bf16* out_Wm,
+                           float* out_soft, uint32_t* out_hard, void* stream) {
+  return mask_fwd(logits, W, N, M, tau, st, rows, cols, out_Wm, out_soft, out_hard, false, stream);
+}
+
+roi_status roi_mask_fwd_st(const float* logits, const roi_bf16* W, int N, int M, float tau,
+                           const roi_noise_state* st, int64_t rows, int64_t cols, roi_bf16* out_Wm,
+                           float* out_soft, uint32_t* out_hard, void* stream) {
+  return mask_fwd(logits, W, N, M, tau, st, rows, cols, out_Wm, out_soft, out_hard, true, stream);
 }
 
 roi_status roi_mask_fwd(const float* logits, const roi_bf16* W, int N, int M, float tau, uint64_t seed,
@@ -141,9 +154,9 @@ roi_status roi_mask_fwd(const float* logits, const roi_bf16* W, int N, int M, fl
   return roi_mask_fwd_ex(logits, W, N, M, tau, &st, rows, cols, out_Wm, out_soft, out_hard, stream);
 }
 
-roi_status roi_mask_bwd(const float* logits, const roi_bf16* W, const roi_noise_state* st, int N, int M,
-                        const roi_bf16* dWm, float tau, int64_t rows, int64_t cols, float* out_dlogits,
-                        roi_bf16* out_dW, void* stream) {
+static roi_status mask_bwd(const float* logits, const roi_bf16* W, const roi_noise_state* st, int N, int M,
+                           const roi_bf16* dWm, const uint32_t* hard, float tau, int64_t rows, int64_t cols,
+                           float* out_dlogits, roi_bf16* out_dW, void* stream) {
   if (st == nullptr) return ROI_ERR_NULL;
   roi_status s = check_common(N, M, tau, rows, cols);
   if (s != ROI_OK) return s;
@@ -154,7 +167,8 @@ roi_status roi_mask_bwd(const float* logits, const roi_bf16* W, const roi_noise_
   if (!aligned16(logits) || !aligned16(W) || !aligned16(dWm) || !aligned16(out_dlogits) || !aligned16(out_dW))
     return ROI_ERR_ALIGN;
   const int64_t E = rows * cols;
-  const Range in[3] = {{logits, uint64_t(E) * 4}, {W, uint64_t(E) * 2}, {dWm, uint64_t(E) * 2}};
+  const Range in[4] = {{logits, uint64_t(E) * 4}, {W, uint64_t(E) * 2}, {dWm, uint64_t(E) * 2},
+                       {hard, uint64_t((E + 31) / 32) * 4}};
   const Range out[2] = {{out_dlogits, uint64_t(E) * 4}, {out_dW, uint64_t(E) * 2}};
   if (any_alias(in, out)) return ROI_ERR_ALIAS;
   if (E == 0) return ROI_OK;
@@ -164,6 +178,7 @@ roi_status roi_mask_bwd(const float* logits, const roi_bf16* W, const roi_noise_
   c.dWm = dWm;
   c.dphi = out_dlogits;
   c.dW = out_dW;
+  c.hard_in = hard;
   c.E = E;
   c.N = N;
   c.M = M;
@@ -173,6 +188,43 @@ roi_status roi_mask_bwd(const float* logits, const roi_bf16* W, const roi_noise_
   if (c.status == nullptr) return ROI_ERR_CUDA;
   c.stream = static_cast<cudaStream_t>(stream);
   return finish(launch_bwd(c));
+}
+
+roi_status roi_mask_bwd(const float* logits, const roi_bf16* W, const roi_noise_state* st, int N, int M,
+                        const roi_bf16* dWm, float tau, int64_t rows, int64_t cols, float* out_dlogits,
+                        roi_bf16* out_dW, void* stream) {
+  return mask_bwd(logits, W, st, N, M, dWm, nullptr, tau, rows, cols, out_dlogits, out_dW, stream);
+}
+
+roi_status roi_mask_bwd_st(const float* logits, const roi_bf16* W, const roi_noise_state* st, int N, int M,
+                           const roi_bf16* dWm, const uint32_t* hard, float tau, int64_t rows, int64_t cols,
+                           float* out_dlogits, roi_bf16* out_dW, void* stream) {
+  if (out_dW != nullptr && hard == nullptr && rows > 0) return ROI_ERR_NULL;
+  if (!aligned16(hard)) return ROI_ERR_ALIGN;
+  return mask_bwd(logits, W, st, N, M, dWm, out_dW != nullptr ? hard : nullptr, tau, rows, cols, out_dlogits,
+                  out_dW, stream);
+}
+
+roi_status roi_export_compressed_2of4(const float* logits, const roi_bf16* W, int64_t rows, int64_t cols,
+                                      roi_bf16* out_values, uint32_t* out_meta, void* stream) {
+  roi_status s = check_common(2, 4, 1.0f, rows, cols);
+  if (s != ROI_OK) return s;
+  if ((rows * cols) % 32 != 0) return ROI_ERR_SHAPE;
+  if (rows == 0) return ROI_OK;
+  if (logits == nullptr || W == nullptr || out_values == nullptr || out_meta == nullptr) return ROI_ERR_NULL;
+  if (!aligned16(logits) || !aligned16(W) || !aligned16(out_values) || !aligned16(out_meta)) return ROI_ERR_ALIGN;
+  const int64_t E = rows * cols;
+  const Range in[2] = {{logits, uint64_t(E) * 4}, {W, uint64_t(E) * 2}};
+  const Range out[2] = {{out_values, uint64_t(E)}, {out_meta, uint64_t(E / 32) * 4}};
+  if (any_alias(in, out)) return ROI_ERR_ALIAS;
+  CompressCall c;
+  c.phi = logits;
+  c.W = W;
+  c.values = out_values;
+  c.meta = out_meta;
+  c.E = E;
+  c.stream = static_cast<cudaStream_t>(stream);
+  return finish(launch_export_compressed_2of4(c));
 }
 
 roi_status roi_hard_mask_export(const float* logits, int N, int M, int64_t rows, int64_t cols, uint32_t* out_bits,

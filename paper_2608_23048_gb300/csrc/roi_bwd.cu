@@ -36,6 +36,7 @@ struct BwdArgs {
   const uint16_t* dWm;
   float* dphi;
   uint16_t* dW;
+  const uint32_t* hard_in;  // straight-through: dW = dWm where the forward's hard bit is set
   int64_t E;
   int64_t full_tiles;
   float tau, inv_tau;
@@ -157,11 +158,20 @@ __device__ __forceinline__ void bwd_inputs(const float* const* phi_g, const uint
 // whole history stays in registers.  With HIST (M = 8) registers are tight:
 // the keys die after the forward relaxation (a flagged group re-forms them) and
 // the upstream gradients are formed only for the sweep.
-template <int N, int M, bool TAU1, class V, bool HIST = false>
+template <int N, int M, bool TAU1, class V, bool HIST = false, bool ST = false>
 __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint16_t* const* W_g,
                                            const uint16_t* const* dWm_g, const int64_t* e0, const BwdArgs& a,
                                            V* hist = nullptr) {
   constexpr int L = vlanes<V>();
+  // straight-through: the forward's hard bits of these groups, loaded now so the
+  // load's latency hides behind the relaxation
+  uint32_t keep[ST ? L : 1][ST ? M / 4 : 1];
+  if constexpr (ST) {
+#pragma unroll
+    for (int h = 0; h < L; ++h)
+#pragma unroll
+      for (int s = 0; s < M / 4; ++s) keep[h][s] = hard4(a.hard_in, e0[h] + 4 * s);
+  }
   using Steps = typename std::conditional<HIST, SmemSteps<N, M, V, Cfg<M>::kThreads>, RegSteps<N, M, V>>::type;
   FastGroup<N, M, TAU1, true, V, Steps> fg;
   if constexpr (HIST) fg.st.at = hist;
@@ -175,10 +185,16 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
     fg.forward(kap, a.inv_tau);
   }
   if (a.dW != nullptr) {
-    // dW = bf16(dWm * S) now, while the relaxation is live anyway (dWm is re-read)
+    // dW = bf16(dWm * S) now, while the relaxation is live anyway (dWm is re-read);
+    // straight-through: dWm where the forward's hard mask is set, +0 elsewhere
 #pragma unroll
     for (int s = 0; s < M / 4; ++s) {
-      if constexpr (L == 2) {
+      if constexpr (ST) {
+#pragma unroll
+        for (int h = 0; h < L; ++h)
+          reinterpret_cast<uint2*>(a.dW + e0[h])[s] =
+              keep4(reinterpret_cast<const uint2*>(dWm_g[h])[s], keep[h][s]);
+      } else if constexpr (L == 2) {
         // both groups' products of member l in one packed multiply
         const uint2 qa = reinterpret_cast<const uint2*>(dWm_g[0])[s];
         const uint2 qb = reinterpret_cast<const uint2*>(dWm_g[1])[s];
@@ -233,7 +249,7 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
       ex.backward(cc, N, M, a.tau, dk);
 #pragma unroll
       for (int l = 0; l < M; ++l) dk[l] = __fmul_rn(dk[l], a.np.inv_lam);
-      if (a.dW != nullptr) {
+      if (!ST && a.dW != nullptr) {
 #pragma unroll
         for (int s = 0; s < M / 4; ++s) {
           float d[4];
@@ -251,7 +267,9 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
   }
 }
 
-template <int N, int M, bool TAU1>
+// ST: straight-through dW from the forward's hard bits (a separate instantiation,
+// so the soft kernel's code is not touched by it)
+template <int N, int M, bool TAU1, bool ST>
 __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_kernel(BwdArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   using C = Cfg<M>;
@@ -278,12 +296,12 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_
           const uint16_t* pd[2] = {sdW + g0 * M, sdW + g1 * M};
           const int64_t e0[2] = {base + g0 * M, base + g1 * M};
           if constexpr (M == 4) {
-            bwd_groups<N, M, TAU1, F2>(pp, pw, pd, e0, a);
+            bwd_groups<N, M, TAU1, F2, false, ST>(pp, pw, pd, e0, a);
           } else {
             // M = 8: the paired step history does not fit the register file; steps
             // 0 .. N-2 go to shared memory behind the tile ring
             F2* hist = reinterpret_cast<F2*>(smem + kHistOffset<M>) + threadIdx.x;
-            bwd_groups<N, M, TAU1, F2, true>(pp, pw, pd, e0, a, hist);
+            bwd_groups<N, M, TAU1, F2, true, ST>(pp, pw, pd, e0, a, hist);
           }
         }
       });
@@ -297,7 +315,7 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_
       const uint16_t* pw[1] = {a.W + t0 + gi * M};
       const uint16_t* pd[1] = {a.dWm + t0 + gi * M};
       const int64_t e0[1] = {t0 + gi * M};
-      bwd_groups<N, M, TAU1, float>(pp, pw, pd, e0, a);
+      bwd_groups<N, M, TAU1, float, false, ST>(pp, pw, pd, e0, a);
     }
   }
 }
@@ -317,9 +335,15 @@ __global__ void __launch_bounds__(128) roi_bwd_generic_kernel(BwdArgs a, int N, 
     ex.forward(kap, N, M, a.tau, S);
     ex.backward(c, N, M, a.tau, dk);
     for (int l = 0; l < M; ++l) {
-      a.dphi[e0 + l] = dk[l] * a.np.inv_lam;
-      if (a.dW != nullptr)
-        a.dW[e0 + l] = __bfloat16_as_ushort(__float2bfloat16_rn(bf16_bits_to_float(a.dWm[e0 + l]) * S[l]));
+      const int64_t e = e0 + l;
+      a.dphi[e] = dk[l] * a.np.inv_lam;
+      if (a.dW != nullptr) {
+        if (a.hard_in != nullptr) {
+          a.dW[e] = ((a.hard_in[e >> 5] >> (e & 31)) & 1u) ? a.dWm[e] : uint16_t(0);
+        } else {
+          a.dW[e] = __bfloat16_as_ushort(__float2bfloat16_rn(bf16_bits_to_float(a.dWm[e]) * S[l]));
+        }
+      }
     }
   }
 }
@@ -328,10 +352,10 @@ struct LaunchCache {
   int per_sm[64] = {0};
 };
 
-template <int N, int M, bool TAU1>
+template <int N, int M, bool TAU1, bool ST>
 int launch_tiles(const BwdArgs& a, cudaStream_t stream) {
   using C = Cfg<M>;
-  auto kern = roi_bwd_kernel<N, M, TAU1>;
+  auto kern = roi_bwd_kernel<N, M, TAU1, ST>;
   const size_t smem = kHistBytes<N, M> > 0 ? kHistOffset<M> + kHistBytes<N, M> : tile_smem_bytes<C::kTile, C::kStages>(8);
   static LaunchCache cache;
   int dev = 0;
@@ -351,7 +375,9 @@ int launch_tiles(const BwdArgs& a, cudaStream_t stream) {
 
 template <int N, int M>
 int launch_nm(const BwdArgs& a, cudaStream_t stream) {
-  return a.tau == 1.0f ? launch_tiles<N, M, true>(a, stream) : launch_tiles<N, M, false>(a, stream);
+  if (a.hard_in != nullptr && a.dW != nullptr)
+    return a.tau == 1.0f ? launch_tiles<N, M, true, true>(a, stream) : launch_tiles<N, M, false, true>(a, stream);
+  return a.tau == 1.0f ? launch_tiles<N, M, true, false>(a, stream) : launch_tiles<N, M, false, false>(a, stream);
 }
 
 }  // namespace
@@ -363,6 +389,7 @@ int launch_bwd(const BwdCall& c) {
   a.dWm = c.dWm;
   a.dphi = c.dphi;
   a.dW = c.dW;
+  a.hard_in = c.hard_in;
   a.E = c.E;
   a.full_tiles = c.E / (c.M == 8 ? Cfg<8>::kTile : Cfg<4>::kTile);
   a.tau = c.tau;

@@ -49,6 +49,17 @@ __device__ __forceinline__ float rcp_approx(float x) {
 __device__ __forceinline__ float bf16_bits_to_float(uint32_t bits16) {
   return __uint_as_float(bits16 << 16);
 }
+// Straight-through variant: the four bf16 weights of q where the low four bits of
+// `keep` are set (bit j: element j), +0 elsewhere.
+__device__ __forceinline__ uint2 keep4(uint2 q, uint32_t keep) {
+  const uint32_t m0 = ((keep & 1u) ? 0x0000ffffu : 0u) | ((keep & 2u) ? 0xffff0000u : 0u);
+  const uint32_t m1 = ((keep & 4u) ? 0x0000ffffu : 0u) | ((keep & 8u) ? 0xffff0000u : 0u);
+  return make_uint2(q.x & m0, q.y & m1);
+}
+// The hard-mask bits of elements e .. e + 3 (e % 4 == 0) from the flat word array.
+__device__ __forceinline__ uint32_t hard4(const uint32_t* hard, int64_t e) {
+  return (hard[e >> 5] >> (uint32_t(e) & 31u)) & 0xfu;
+}
 // Two floats -> two bf16 (round to nearest even), packed low|high.
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);

@@ -110,6 +110,60 @@ __global__ void __launch_bounds__(256) roi_export_vec_kernel(const float* __rest
   }
 }
 
+// Compressed 2:4 export.  A warp takes 1024 elements (256 groups) at a time; lane l
+// holds groups l + 32 j (j < 8), so every load and store instruction of the warp is
+// contiguous.  Per group: the two kept weights in index order (one 32-bit word) and
+// the 4-bit code i0 | i1 << 2; the codes of the eight groups of a metadata word sit
+// in eight consecutive lanes and are OR-combined with shuffles.
+__global__ void __launch_bounds__(256) roi_export_2of4_kernel(const float* __restrict__ phi,
+                                                              const uint16_t* __restrict__ W, int64_t E,
+                                                              uint32_t* __restrict__ values,
+                                                              uint32_t* __restrict__ meta) {
+  const int lane = threadIdx.x & 31;
+  const int64_t groups = E / 4;
+  const int64_t chunks = (groups + 255) / 256;
+  const int64_t warp = (blockIdx.x * int64_t(blockDim.x) + threadIdx.x) >> 5;
+  const int64_t warps = (int64_t(gridDim.x) * blockDim.x) >> 5;
+  const float4* p4 = reinterpret_cast<const float4*>(phi);
+  const uint2* w2 = reinterpret_cast<const uint2*>(W);
+  for (int64_t ch = warp; ch < chunks; ch += warps) {
+    const int64_t g0 = ch * 256 + lane;
+    float4 k[8];
+    uint2 q[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int64_t g = g0 + 32 * j;
+      if (g < groups) {
+        k[j] = p4[g];
+        q[j] = w2[g];
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int64_t g = g0 + 32 * j;
+      uint32_t code = 0;
+      if (g < groups) {
+        const float kk[4] = {k[j].x, k[j].y, k[j].z, k[j].w};
+        const uint32_t bits = topn_bits4(kk, 2);
+        // the two set bits of a 2-of-4 mask: lowest i0, then i1
+        const uint32_t i0 = __ffs(bits) - 1u;
+        const uint32_t i1 = __ffs(bits & (bits - 1u)) - 1u;
+        code = i0 | (i1 << 2);
+        auto at = [&q, j](uint32_t i) {
+          const uint32_t half = i < 2 ? q[j].x : q[j].y;
+          return (i & 1u) ? half >> 16 : half & 0xffffu;
+        };
+        values[g] = at(i0) | (at(i1) << 16);
+      }
+      uint32_t v = code << (4 * (lane & 7));
+      v |= __shfl_xor_sync(0xffffffffu, v, 1);
+      v |= __shfl_xor_sync(0xffffffffu, v, 2);
+      v |= __shfl_xor_sync(0xffffffffu, v, 4);
+      if ((lane & 7) == 0 && g < groups) meta[g >> 3] = v;
+    }
+  }
+}
+
 int grid_for(int64_t items, int threads) {
   int64_t blocks = (items + threads - 1) / threads;
   const int64_t cap = int64_t(sm_count()) * 8;
@@ -118,6 +172,13 @@ int grid_for(int64_t items, int threads) {
 }
 
 }  // namespace
+
+int launch_export_compressed_2of4(const CompressCall& c) {
+  const int64_t warps = (c.E / 4 + 255) / 256;
+  roi_export_2of4_kernel<<<grid_for(warps * 32, 256), 256, 0, c.stream>>>(
+      c.phi, c.W, c.E, reinterpret_cast<uint32_t*>(c.values), c.meta);
+  return cudaGetLastError() == cudaSuccess ? 1 : -1;
+}
 
 int launch_export(const ExportCall& c) {
   int launched = 0;

@@ -29,6 +29,7 @@ struct FwdArgs {
   uint16_t* Wm;
   float* soft;
   uint32_t* hard;
+  bool st;  // straight-through: Wm = W where the hard mask is set, +0 elsewhere
   int64_t E;
   int64_t full_tiles;
   float tau, inv_tau;
@@ -95,7 +96,7 @@ __device__ __forceinline__ float lane_of(V v, int h) {
 
 // L groups (one per lane of V) processed in lockstep by one thread; writes their
 // outputs and returns each group's hard bits in bits[h].
-template <int N, int M, bool TAU1, class V>
+template <int N, int M, bool TAU1, class V, bool ST = false>
 __device__ __forceinline__ void fwd_groups(const float* const* phi_g, const uint16_t* const* W_g, const int64_t* e0,
                                            const FwdArgs& a, uint32_t* bits) {
   constexpr int L = vlanes<V>();
@@ -181,7 +182,12 @@ __device__ __forceinline__ void fwd_groups(const float* const* phi_g, const uint
 #pragma unroll
   for (int s = 0; s < M / 4; ++s) {
     const float* sa = S[0] + 4 * s;
-    if constexpr (L == 2) {
+    if constexpr (ST) {
+      // straight-through: the weights the hard mask keeps, +0 elsewhere
+#pragma unroll
+      for (int h = 0; h < L; ++h)
+        reinterpret_cast<uint2*>(a.Wm + e0[h])[s] = keep4(reinterpret_cast<const uint2*>(W_g[h])[s], bits[h] >> (4 * s));
+    } else if constexpr (L == 2) {
       // both groups' products of member l in one packed multiply
       const float* sb = S[1] + 4 * s;
       const uint2 qa = reinterpret_cast<const uint2*>(W_g[0])[s];
@@ -247,7 +253,8 @@ __device__ __forceinline__ void store_hard_pair(uint32_t* hard, int64_t e0a, int
   if (lane % kHalf == 0) hard[(upper ? e0b : e0a) >> 5] = word;
 }
 
-template <int N, int M, bool TAU1>
+// ST: straight-through Wm (a separate instantiation)
+template <int N, int M, bool TAU1, bool ST>
 __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_fwd_kernel(FwdArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   using C = Cfg<M>;
@@ -271,7 +278,7 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_fwd_
           const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
           const int64_t e0[2] = {base + g0 * M, base + g1 * M};
           uint32_t bits[2];
-          fwd_groups<N, M, TAU1, F2>(pp, pw, e0, a, bits);
+          fwd_groups<N, M, TAU1, F2, ST>(pp, pw, e0, a, bits);
           if (a.hard != nullptr) store_hard_pair<M>(a.hard, e0[0], e0[1], bits[0], bits[1]);
         }
       });
@@ -290,7 +297,7 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_fwd_
         const float* pp[1] = {a.phi + t0 + gi * M};
         const uint16_t* pw[1] = {a.W + t0 + gi * M};
         const int64_t e0[1] = {t0 + gi * M};
-        fwd_groups<N, M, TAU1, float>(pp, pw, e0, a, &bits);
+        fwd_groups<N, M, TAU1, float, ST>(pp, pw, e0, a, &bits);
       }
       if (a.hard != nullptr) store_hard<M>(a.hard, t0 + gi * M, bits, active);
     }
@@ -311,13 +318,14 @@ __global__ void __launch_bounds__(128) roi_fwd_generic_kernel(FwdArgs a, int N, 
     }
     ExactGroup<31, 32> ex;
     ex.forward(kap, N, M, a.tau, S);
+    const uint32_t bits = (a.hard != nullptr || a.st) ? topn_bits_dyn(kap, N, M) : 0u;
     for (int l = 0; l < M; ++l) {
       const float w = bf16_bits_to_float(a.W[e0 + l]);
-      a.Wm[e0 + l] = __bfloat16_as_ushort(__float2bfloat16_rn(w * S[l]));
+      a.Wm[e0 + l] = a.st ? (((bits >> l) & 1u) ? a.W[e0 + l] : uint16_t(0))
+                          : __bfloat16_as_ushort(__float2bfloat16_rn(w * S[l]));
       if (a.soft != nullptr) a.soft[e0 + l] = S[l];
     }
     if (a.hard != nullptr) {
-      const uint32_t bits = topn_bits_dyn(kap, N, M);
       for (int l = 0; l < M; ++l)
         if ((bits >> l) & 1u) {
           const int64_t e = e0 + l;
@@ -331,10 +339,10 @@ struct LaunchCache {
   int per_sm[64] = {0};
 };
 
-template <int N, int M, bool TAU1>
+template <int N, int M, bool TAU1, bool ST>
 int launch_tiles(const FwdArgs& a, cudaStream_t stream) {
   using C = Cfg<M>;
-  auto kern = roi_fwd_kernel<N, M, TAU1>;
+  auto kern = roi_fwd_kernel<N, M, TAU1, ST>;
   const size_t smem = tile_smem_bytes<C::kTile, C::kStages>(6);
   static LaunchCache cache;  // per instantiation and device; racing writers store the same value
   int dev = 0;
@@ -354,7 +362,8 @@ int launch_tiles(const FwdArgs& a, cudaStream_t stream) {
 
 template <int N, int M>
 int launch_nm(const FwdArgs& a, cudaStream_t stream) {
-  return a.tau == 1.0f ? launch_tiles<N, M, true>(a, stream) : launch_tiles<N, M, false>(a, stream);
+  if (a.st) return a.tau == 1.0f ? launch_tiles<N, M, true, true>(a, stream) : launch_tiles<N, M, false, true>(a, stream);
+  return a.tau == 1.0f ? launch_tiles<N, M, true, false>(a, stream) : launch_tiles<N, M, false, false>(a, stream);
 }
 
 }  // namespace
@@ -366,6 +375,7 @@ int launch_fwd(const FwdCall& c) {
   a.Wm = c.Wm;
   a.soft = c.soft;
   a.hard = c.hard;
+  a.st = c.st;
   a.E = c.E;
   a.full_tiles = c.E / (c.M == 8 ? Cfg<8>::kTile : Cfg<4>::kTile);
   a.tau = c.tau;

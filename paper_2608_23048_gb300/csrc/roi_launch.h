@@ -14,6 +14,7 @@ struct FwdCall {
   uint16_t* Wm;
   float* soft;      // nullable
   uint32_t* hard;   // nullable
+  bool st;          // straight-through: Wm = W where the hard mask is set, +0 elsewhere
   int64_t E;        // rows * cols
   int N, M;
   float tau;
@@ -28,6 +29,7 @@ struct BwdCall {
   const uint16_t* dWm;
   float* dphi;
   uint16_t* dW;     // nullable
+  const uint32_t* hard_in;  // nullable; straight-through: dW = dWm where set, +0 elsewhere
   int64_t E;
   int N, M;
   float tau;
@@ -46,10 +48,20 @@ struct ExportCall {
   cudaStream_t stream;
 };
 
+struct CompressCall {
+  const float* phi;
+  const uint16_t* W;
+  uint16_t* values;  // [E / 2]
+  uint32_t* meta;    // [E / 32]
+  int64_t E;         // multiple of 32
+  cudaStream_t stream;
+};
+
 // Each returns the number of kernels launched (>= 0) or -1 after a CUDA error.
 int launch_fwd(const FwdCall& c);
 int launch_bwd(const BwdCall& c);
 int launch_export(const ExportCall& c);
+int launch_export_compressed_2of4(const CompressCall& c);
 // Warp-slice kernels for M = 16, 32 (roi_slice.cu).
 bool slice_supported(int N, int M);
 int launch_slice_fwd(const FwdCall& c);

@@ -107,6 +107,8 @@ struct SliceArgs {
   uint32_t* hard;
   float* dphi;
   uint16_t* dW;
+  bool st;                  // straight-through forward: Wm = W where the hard mask is set
+  const uint32_t* hard_in;  // straight-through backward: dW = dWm where the forward's bit is set
   int64_t E;
   int64_t full_tiles;
   float tau, inv_tau;
@@ -364,14 +366,16 @@ __device__ __forceinline__ void fwd_slots(const float* const* p, const uint16_t*
   if (!active) return;
 #pragma unroll
   for (int h = 0; h < L; ++h) {
+    // straight-through: every slot keeps the weights its hard bits select
+    if (a.st) *reinterpret_cast<uint2*>(a.Wm + e0[h]) = keep4(*reinterpret_cast<const uint2*>(w[h]), bits[h]);
     if (!((flag >> h) & 1u)) {
       float wv[4], sv[4];
       unpack_bf16x4(*reinterpret_cast<const uint2*>(w[h]), wv);
 #pragma unroll
       for (int j = 0; j < 4; ++j) sv[j] = lane_of(rx.S[j], h);
-      *reinterpret_cast<uint2*>(a.Wm + e0[h]) = pack4(wv, sv);
+      if (!a.st) *reinterpret_cast<uint2*>(a.Wm + e0[h]) = pack4(wv, sv);
       if (a.soft != nullptr) *reinterpret_cast<float4*>(a.soft + e0[h]) = make_float4(sv[0], sv[1], sv[2], sv[3]);
-    } else if (q == 0) {
+    } else if (q == 0 && (a.soft != nullptr || !a.st)) {
       float k[M], S[M];
       group_keys_all<N, M>(p[h], e0[h], a.np, k);
       ExactGroup<N, M> ex;
@@ -382,7 +386,7 @@ __device__ __forceinline__ void fwd_slots(const float* const* p, const uint16_t*
         unpack_bf16x4(*reinterpret_cast<const uint2*>(w[h] + 4 * s), wv);
 #pragma unroll
         for (int j = 0; j < 4; ++j) sv[j] = S[4 * s + j];
-        *reinterpret_cast<uint2*>(a.Wm + e0[h] + 4 * s) = pack4(wv, sv);
+        if (!a.st) *reinterpret_cast<uint2*>(a.Wm + e0[h] + 4 * s) = pack4(wv, sv);
         if (a.soft != nullptr)
           *reinterpret_cast<float4*>(a.soft + e0[h] + 4 * s) = make_float4(sv[0], sv[1], sv[2], sv[3]);
       }
@@ -425,7 +429,10 @@ __device__ __forceinline__ void bwd_slots(const float* const* p, const uint16_t*
   if (active && a.dW != nullptr) {
 #pragma unroll
     for (int h = 0; h < L; ++h) {
-      if (!((flag >> h) & 1u)) {
+      if (a.hard_in != nullptr) {
+        // straight-through: dWm where the forward's hard mask is set
+        *reinterpret_cast<uint2*>(a.dW + e0[h]) = keep4(*reinterpret_cast<const uint2*>(dw[h]), hard4(a.hard_in, e0[h]));
+      } else if (!((flag >> h) & 1u)) {
         float dv[4], sv[4];
         unpack_bf16x4(*reinterpret_cast<const uint2*>(dw[h]), dv);
 #pragma unroll
@@ -463,7 +470,7 @@ __device__ __forceinline__ void bwd_slots(const float* const* p, const uint16_t*
         *reinterpret_cast<float4*>(a.dphi + e0[h] + 4 * s) =
             make_float4(__fmul_rn(dkk[4 * s], a.np.inv_lam), __fmul_rn(dkk[4 * s + 1], a.np.inv_lam),
                         __fmul_rn(dkk[4 * s + 2], a.np.inv_lam), __fmul_rn(dkk[4 * s + 3], a.np.inv_lam));
-        if (a.dW != nullptr) {
+        if (a.dW != nullptr && a.hard_in == nullptr) {
           float dv[4], sv[4];
           unpack_bf16x4(*reinterpret_cast<const uint2*>(dw[h] + 4 * s), dv);
 #pragma unroll
@@ -643,6 +650,7 @@ int launch_slice_fwd(const FwdCall& c) {
   a.Wm = c.Wm;
   a.soft = c.soft;
   a.hard = c.hard;
+  a.st = c.st;
   a.E = c.E;
   a.full_tiles = c.E / kTile;
   a.tau = c.tau;
@@ -661,6 +669,7 @@ int launch_slice_bwd(const BwdCall& c) {
   a.dWm = c.dWm;
   a.dphi = c.dphi;
   a.dW = c.dW;
+  a.hard_in = c.hard_in;
   a.E = c.E;
   a.full_tiles = c.E / kTile;
   a.tau = c.tau;

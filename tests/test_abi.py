@@ -78,6 +78,23 @@ def test_validation_codes(L):
     assert L.roi_hard_mask_export(_fake(A), 2, 4, 4, 8, _fake(C), _fake(B), None, None) == 1
     assert L.roi_hard_mask_export(_fake(A), 2, 4, 4, 8, _fake(C + 4), None, None, None) == 5
     assert L.roi_hard_mask_export(_fake(A), 2, 4, 0, 8, _fake(C), None, None, None) == 0
+    # straight-through: as the soft calls; the backward needs the forward's bits when dW is asked for
+    assert L.roi_mask_fwd_st(None, _fake(B), 2, 4, 1.0, ctypes.byref(st), 4, 8, _fake(C), None, None, None) == 1
+    assert L.roi_mask_fwd_st(_fake(A), _fake(B), 2, 4, 1.0, ctypes.byref(st), 4, 8, _fake(A + 16), None, None,
+                             None) == 6
+    assert L.roi_mask_bwd_st(_fake(A), _fake(B), ctypes.byref(st), 2, 4, _fake(D), None, 1.0, 4, 8, _fake(C),
+                             _fake(E), None) == 1
+    assert L.roi_mask_bwd_st(_fake(A), _fake(B), ctypes.byref(st), 2, 4, _fake(D), _fake(E + 4), 1.0, 4, 8,
+                             _fake(C), _fake(D + 0x1000), None) == 5
+    assert L.roi_mask_bwd_st(_fake(A), _fake(B), ctypes.byref(st), 2, 4, _fake(D), _fake(C), 1.0, 4, 8,
+                             _fake(C), _fake(E), None) == 6
+    # compressed export: 2:4 only, rows*cols a multiple of 32
+    assert L.roi_export_compressed_2of4(_fake(A), _fake(B), 1, 12, _fake(C), _fake(D), None) == 2
+    assert L.roi_export_compressed_2of4(_fake(A), _fake(B), 4, 6, _fake(C), _fake(D), None) == 2
+    assert L.roi_export_compressed_2of4(None, _fake(B), 4, 8, _fake(C), _fake(D), None) == 1
+    assert L.roi_export_compressed_2of4(_fake(A), _fake(B), 4, 8, _fake(C + 2), _fake(D), None) == 5
+    assert L.roi_export_compressed_2of4(_fake(A), _fake(B), 4, 8, _fake(A + 16), _fake(D), None) == 6
+    assert L.roi_export_compressed_2of4(None, None, 0, 8, None, None, None) == 0
     for s in range(9):
         assert L.roi_status_string(s)
 

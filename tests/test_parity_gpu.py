@@ -353,3 +353,82 @@ def test_gumbel_noise_error_bound(roi):
     want = O.gumbel_noise(99, 1, 0, rows, cols)
     err = np.abs(g - want)
     assert np.all(err <= 5e-7 + 2.0 ** -22 * np.abs(want)), float(np.max(err))
+
+
+ST_CASES = [
+    (37, 1000, 2, 4, 1.0, "logw"),     # tiles + ragged tail
+    (29, 1536, 4, 8, 1.0, "normal"),
+    (37, 1000, 2, 4, 0.5, "normal"),
+    (29, 1536, 4, 8, 0.5, "normal"),
+    (9, 1024, 8, 16, 0.5, "logw"),     # warp-slice kernels
+    (7, 1024, 16, 32, 1.0, "normal"),
+    (13, 960, 3, 4, 1.0, "normal"),    # generic kernels
+]
+
+
+@pytest.mark.parametrize("rows,cols,N,M,tau,kind", ST_CASES)
+def test_straight_through_variant(roi, rows, cols, N, M, tau, kind):
+    """Straight-through forward/backward: hard bits, soft output and logit gradients
+    are those of the soft calls (bit for bit); Wm and dW are W and dWm where the hard
+    mask is set, +0 elsewhere; the hard mask agrees with the oracle outside near ties."""
+    import torch
+    W, phi, dWm, ph, Wb, dWb = make(rows, cols, kind, data_seed=rows * 3 + M)
+    phi = phi.clone()
+    phi[0, :M] = float("nan")          # a flagged group
+    ph = phi.numpy()
+    dev = torch.device("cuda")
+    st = roi.NoiseState(77, 4, 5, 1.0, 0)
+    phi_d, W_d, dWm_d = phi.to(dev), W.to(dev), dWm.to(dev)
+    nw = roi.hard_words(rows, cols)
+    outs = {}
+    for mode in ("soft", "st"):
+        Wm = torch.empty(rows, cols, dtype=torch.bfloat16, device=dev)
+        soft = torch.empty(rows, cols, dtype=torch.float32, device=dev)
+        hard = torch.empty(nw, dtype=torch.int32, device=dev)
+        dphi = torch.empty(rows, cols, dtype=torch.float32, device=dev)
+        dW = torch.empty(rows, cols, dtype=torch.bfloat16, device=dev)
+        if mode == "soft":
+            roi.roi_mask_fwd_ex(phi_d, W_d, N, M, tau, st, Wm, soft, hard)
+            roi.roi_mask_bwd(phi_d, W_d, st, N, M, dWm_d, tau, dphi, dW)
+        else:
+            roi.roi_mask_fwd_st(phi_d, W_d, N, M, tau, st, Wm, soft, hard)
+            roi.roi_mask_bwd_st(phi_d, W_d, st, N, M, dWm_d, hard, tau, dphi, dW)
+        roi.roi_device_status()
+        outs[mode] = {"Wm": _u16(Wm), "soft": soft.cpu().numpy(), "hard": _bits(hard),
+                      "dphi": dphi.cpu().numpy(), "dW": _u16(dW)}
+    a, b = outs["soft"], outs["st"]
+    assert np.array_equal(a["hard"], b["hard"])
+    assert np.array_equal(a["soft"].view(np.uint32), b["soft"].view(np.uint32))
+    assert np.array_equal(a["dphi"].view(np.uint32), b["dphi"].view(np.uint32))
+    keep = O.unpack_bits(b["hard"], rows * cols).reshape(rows, cols)
+    assert np.array_equal(b["Wm"], np.where(keep, Wb, np.uint16(0)))
+    assert np.array_equal(b["dW"], np.where(keep, dWb, np.uint16(0)))
+    # the hard mask itself against the oracle (the straight-through oracle's Wm follows)
+    ref = O.mask_fwd_st(ph, Wb, N, M, tau, 77, 4, tensor_id=5)
+    mism = (keep != ref["hard"]).reshape(-1, M).any(-1)
+    with np.errstate(invalid="ignore"):
+        near = ~(O.topn_key_gap(ref["keys"].reshape(-1, M), N) >= 1e-6)
+    assert not np.any(mism & ~near)
+    ok = ~np.repeat(mism, M).reshape(rows, cols)
+    assert np.array_equal(b["Wm"][ok], ref["Wm"][ok])
+    refb = O.mask_bwd_st(ph, Wb, dWb, ref["hard_bits"], N, M, tau, 77, 4, tensor_id=5)
+    assert np.array_equal(b["dW"][ok], refb["dW"][ok])
+
+
+@pytest.mark.parametrize("rows,cols", [(37, 1024), (1, 32), (64, 256), (3, 96)])
+def test_compressed_2of4_export_bit_exact(roi, rows, cols):
+    import torch
+    W, phi, *_ = make(rows, cols, "normal", data_seed=rows + 2 * cols)
+    phi = phi.clone()
+    phi[0, :8] = 0.5                   # ties
+    if rows > 1:
+        phi[1, 4] = float("nan")
+        phi[1, 9] = float("inf")
+    dev = torch.device("cuda")
+    values = torch.empty(rows, cols // 2, dtype=torch.bfloat16, device=dev)
+    meta = torch.empty(rows * cols // 32, dtype=torch.int32, device=dev)
+    roi.roi_export_compressed_2of4(phi.to(dev), W.to(dev), values, meta)
+    roi.roi_device_status()
+    ref = O.export_compressed_2of4(phi.numpy(), WL.bf16_bits(W))
+    assert np.array_equal(_u16(values), ref["values"])
+    assert np.array_equal(_bits(meta), ref["meta"])
