@@ -393,3 +393,31 @@ def decompress_2of4(values, meta, rows, cols):
         dense[g, code & 3] = v[g, 0]
         dense[g, code >> 2] = v[g, 1]
     return dense.reshape(rows, cols)
+
+
+def anneal(init: float, end: float, t, T_anneal: float):
+    """Exponential annealing of tau and lambda (Sec. 4.2.3, Eq. 9):
+    x_t = max(x_end, x_init * (x_end / x_init) ** (t / T_anneal))."""
+    t = np.asarray(t, dtype=np.float64)
+    return np.maximum(end, init * (end / init) ** (t / T_anneal))
+
+
+def adamw_step(phi, g, m, v, lr, beta1, beta2, eps, weight_decay, t, dtype=np.float64):
+    """One AdamW step on the logits (decoupled weight decay; the optimizer and its
+    hyper-parameters of Sec. 5.1 and the hyper-parameter table: beta1 = 0.9,
+    beta2 = 0.95, weight decay 0.05), written out from its definition:
+        phi <- phi * (1 - lr * weight_decay)
+        m   <- beta1 m + (1 - beta1) g
+        v   <- beta2 v + (1 - beta2) g^2
+        phi <- phi - lr * (m / (1 - beta1^t)) / (sqrt(v / (1 - beta2^t)) + eps)
+    t is the 1-based step count.  Returns (phi, m, v)."""
+    ar = _Arith(dtype)
+    phi, g, m, v = (ar.cast(np.asarray(x, dtype=np.float64)) for x in (phi, g, m, v))
+    c = lambda x: ar.cast(np.float64(x))
+    phi = phi * (c(1.0) - c(lr) * c(weight_decay))
+    m = c(beta1) * m + (c(1.0) - c(beta1)) * g
+    v = c(beta2) * v + (c(1.0) - c(beta2)) * (g * g)
+    bc1 = c(1.0 - beta1 ** t)
+    bc2 = c(1.0 - beta2 ** t)
+    phi = phi - c(lr) * (m / bc1) / (ar.cast(np.sqrt(v / bc2)) + c(eps))
+    return phi, m, v
