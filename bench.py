@@ -52,8 +52,9 @@ def parse_args():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--layers", type=int, default=None, help="only the first L layers (profiling cases)")
     p.add_argument("--proj", default=None, help="comma-separated projections to keep, e.g. gate")
-    p.add_argument("--op", choices=("mask", "st", "export2of4"), default="mask",
+    p.add_argument("--op", choices=("mask", "st", "adamw", "export2of4"), default="mask",
                    help="mask: the fwd+bwd step (default); st: the straight-through pair with dW; "
+                        "adamw: fwd + the backward fused with the logits' AdamW step; "
                         "export2of4: the compressed 2:4 export (one GPU)")
     return p.parse_args()
 
@@ -515,6 +516,7 @@ def run_e2e(args, roi, tensors, lset, N, M, tau, dev, world):
 ST_FWD_BYTES = FWD_BYTES
 ST_BWD_BYTES = BWD_BYTES + 2 + 1 / 8   # + dW out, + the forward's hard bits in
 EXPORT_2OF4_BYTES = 4 + 2 + 1 + 1 / 8  # logits, W in; kept values, index codes out
+ADAMW_BWD_BYTES = 4 + 2 + 2 + 4 + 4 + 4 + 4 + 4  # logits, W, dWm, m, v in; logits, m, v out
 
 
 def run_variant(args):
@@ -538,9 +540,11 @@ def run_variant(args):
     for layer, p, rows, cols in selected_tensors(args):
         W, phi, dWm = WL.make_inputs(rows, cols, kind, WL.tensor_seed(layer, p), device=dev)
         t = {"id": layer * len(WL.PROJS) + p, "rows": rows, "cols": cols, "phi": phi, "W": W, "dWm": dWm}
-        if args.op == "st":
+        if args.op in ("st", "adamw"):
             t.update(Wm=torch.empty_like(W), dphi=torch.empty_like(phi), dW=torch.empty_like(W),
                      hard=torch.empty(roi.hard_words(rows, cols), dtype=torch.int32, device=dev))
+        if args.op == "adamw":
+            t.update(m=torch.zeros_like(phi), v=torch.zeros_like(phi))
         else:
             t.update(values=torch.empty(rows, cols // 2, dtype=torch.bfloat16, device=dev),
                      meta=torch.empty(rows * cols // 32, dtype=torch.int32, device=dev))
@@ -557,15 +561,22 @@ def run_variant(args):
             rec(ev[0] if ev else None)
             if args.op == "st":
                 roi.roi_mask_fwd_st(t["phi"], t["W"], N, M, tau, st, t["Wm"], None, t["hard"], stream=stream)
+            elif args.op == "adamw":
+                roi.roi_mask_fwd_ex(t["phi"], t["W"], N, M, tau, st, t["Wm"], None, t["hard"], stream=stream)
             else:
                 roi.roi_export_compressed_2of4(t["phi"], t["W"], t["values"], t["meta"], stream=stream)
             rec(ev[1] if ev else None)
-        if args.op == "st":
+        if args.op in ("st", "adamw"):
             for t in reversed(tensors):
                 st = roi.NoiseState(0, s, t["id"], 1.0, 0)
                 rec(ev[2] if ev else None)
-                roi.roi_mask_bwd_st(t["phi"], t["W"], st, N, M, t["dWm"], t["hard"], tau, t["dphi"], t["dW"],
-                                    stream=stream)
+                if args.op == "st":
+                    roi.roi_mask_bwd_st(t["phi"], t["W"], st, N, M, t["dWm"], t["hard"], tau, t["dphi"], t["dW"],
+                                        stream=stream)
+                else:
+                    opt = roi.AdamW(1e-3, 0.9, 0.95, 1e-8, 0.05, s + 1)
+                    roi.roi_mask_bwd_adamw(t["phi"], t["W"], st, N, M, t["dWm"], tau, t["m"], t["v"], opt,
+                                           stream=stream)
                 rec(ev[3] if ev else None)
 
     for w in range(args.warmup):
@@ -586,16 +597,19 @@ def run_variant(args):
     b_t = sum(x.elapsed_time(y) for x, y in zip(ev[2], ev[3])) / 1e3
     E = cfg["elements"]
     peak, peak_kind = hbm_peak()
-    if args.op == "st":
-        a_gbs = E * ST_FWD_BYTES * args.steps / a_t / 1e9
-        b_gbs = E * ST_BWD_BYTES * args.steps / b_t / 1e9
+    if args.op in ("st", "adamw"):
+        fb, bb = (ST_FWD_BYTES, ST_BWD_BYTES) if args.op == "st" else (FWD_BYTES, ADAMW_BWD_BYTES)
+        a_gbs = E * fb * args.steps / a_t / 1e9
+        b_gbs = E * bb * args.steps / b_t / 1e9
         dom = "bwd" if b_t >= a_t else "fwd"
-        achieved, per = (b_gbs, ST_BWD_BYTES) if dom == "bwd" else (a_gbs, ST_FWD_BYTES)
-        step_bytes = ST_FWD_BYTES + ST_BWD_BYTES
+        achieved, per = (b_gbs, bb) if dom == "bwd" else (a_gbs, fb)
+        step_bytes = fb + bb
         extra = {"fwd_gbs": round(a_gbs, 1), "bwd_gbs": round(b_gbs, 1),
                  "fwd_ms_per_step": round(1e3 * a_t / args.steps, 3), "bwd_ms_per_step": round(1e3 * b_t / args.steps, 3)}
-        kernel = f"roi_{dom}_kernel<{N},{M},{'tau1' if tau == 1.0 else 'tau'}> (straight-through)"
-        metric = "straight-through RoI mask fwd+bwd (dW on) groups/s and HBM GB/s, 1 GPU"
+        what = "straight-through" if args.op == "st" else "backward fused with AdamW"
+        kernel = f"roi_{dom}_kernel<{N},{M},{'tau1' if tau == 1.0 else 'tau'}> ({what})"
+        metric = ("straight-through RoI mask fwd+bwd (dW on) groups/s and HBM GB/s, 1 GPU" if args.op == "st" else
+                  "RoI mask fwd + bwd fused with the logits' AdamW step, groups/s and HBM GB/s, 1 GPU")
     else:
         achieved = E * EXPORT_2OF4_BYTES * args.steps / a_t / 1e9
         per, step_bytes = EXPORT_2OF4_BYTES, EXPORT_2OF4_BYTES

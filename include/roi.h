@@ -58,7 +58,8 @@ typedef enum {
     ROI_ERR_ALIGN = 5,     /* a tensor pointer is not 16-byte aligned                    */
     ROI_ERR_ALIAS = 6,     /* an output overlaps an input or another output              */
     ROI_ERR_CUDA = 7,      /* launch failed (cudaGetLastError after the launch)          */
-    ROI_ERR_TIMEOUT = 8    /* a kernel gave up waiting on its own copies (see below)     */
+    ROI_ERR_TIMEOUT = 8,   /* a kernel gave up waiting on its own copies (see below)     */
+    ROI_ERR_OPT = 9        /* bad optimizer settings (roi_mask_bwd_adamw)                */
 } roi_status;
 
 /* Noise state of one call (Sec. 4.2.3 sampling temperature included).
@@ -122,6 +123,45 @@ roi_status roi_mask_bwd_st(const float* logits, const roi_bf16* W, const roi_noi
                            int N, int M, const roi_bf16* dWm, const uint32_t* hard, float tau,
                            int64_t rows, int64_t cols, float* out_dlogits, roi_bf16* out_dW,
                            void* stream);
+
+/* Settings of one AdamW step on the logits (the paper's optimizer, hyper-parameter
+ * table: beta1 = 0.9, beta2 = 0.95, weight decay 0.05, lr 1e-3 decaying to 1e-4).
+ *  lr, weight_decay: finite, >= 0; beta1, beta2 in [0, 1); eps > 0 (1e-8);
+ *  t: 1-based count of steps taken, this one included (bias correction). */
+typedef struct {
+    float lr;
+    float beta1;
+    float beta2;
+    float eps;
+    float weight_decay;
+    uint32_t t;
+} roi_adamw;
+
+/* Backward fused with the logits' optimizer step: the logit gradient g of
+ * roi_mask_bwd is formed in registers and used at once for one AdamW step
+ * (decoupled weight decay):
+ *     phi <- phi (1 - lr wd);  m <- b1 m + (1 - b1) g;  v <- b2 v + (1 - b2) g^2;
+ *     phi <- phi - (step m) / (sqrt(v) r + eps),
+ *     step = lr / (1 - b1^t),  r = 1 / sqrt(1 - b2^t)   (scalars, on the host in double)
+ * in float32, every operation rounded (divide and square root correctly rounded).
+ * Unlike the other calls, logits is read AND written: it holds phi_t on entry
+ * and phi_{t+1} on return (elements not shared with any other tensor).
+ *  m, v         [rows, cols] float32, the optimizer moments, updated in place
+ *  out_dlogits  nullable: the gradient g as well
+ *  out_dW       nullable: bf16_rne(float(dWm) * S), as roi_mask_bwd
+ * The step needs the gradient of this mask op alone (one use of phi per step;
+ * a data-parallel run reduces gradients first and uses roi_mask_bwd instead).
+ * ROI_ERR_OPT for settings outside the ranges above. */
+roi_status roi_mask_bwd_adamw(float* logits, const roi_bf16* W, const roi_noise_state* st, int N, int M,
+                              const roi_bf16* dWm, float tau, int64_t rows, int64_t cols,
+                              float* m, float* v, const roi_adamw* opt,
+                              float* out_dlogits, roi_bf16* out_dW, void* stream);
+
+/* Exponential annealing of tau and lambda (Sec. 4.2.3, Eq. 9), on the host:
+ *     x_t = max(x_end, x_init (x_end / x_init)^(t / T_anneal))
+ * (the paper: tau 1.0 -> 0.05, lambda 1.0 -> 0.002, T_anneal = 1500).
+ * init, end > 0; T_anneal == 0 gives end. */
+float roi_anneal(float init, float end, uint32_t t, uint32_t T_anneal);
 
 /* Compressed 2:4 export for semi-structured sparse inference (the deployment the
  * paper targets, Sec. 1 and the Throughput appendix; it gives no format, so this

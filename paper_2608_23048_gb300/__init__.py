@@ -16,7 +16,8 @@ __all__ = [
     "RoiError", "NoiseState", "lib", "roi_mask_fwd", "roi_mask_fwd_ex", "roi_mask_bwd",
     "roi_hard_mask_export", "roi_device_status", "roi_status_string", "roi_launch_count",
     "library_path", "hard_words", "roi_noise_words", "roi_gumbel_noise",
-    "roi_mask_fwd_st", "roi_mask_bwd_st", "roi_export_compressed_2of4",
+    "roi_mask_fwd_st", "roi_mask_bwd_st", "roi_export_compressed_2of4", "AdamW", "roi_mask_bwd_adamw",
+    "roi_anneal",
 ]
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
@@ -24,7 +25,7 @@ library_path = os.path.join(_PKG, "libroi.so")
 
 ROI_OK = 0
 STATUS_NAMES = {0: "ROI_OK", 1: "ROI_ERR_NULL", 2: "ROI_ERR_SHAPE", 3: "ROI_ERR_NM", 4: "ROI_ERR_TAU",
-                5: "ROI_ERR_ALIGN", 6: "ROI_ERR_ALIAS", 7: "ROI_ERR_CUDA", 8: "ROI_ERR_TIMEOUT"}
+                5: "ROI_ERR_ALIGN", 6: "ROI_ERR_ALIAS", 7: "ROI_ERR_CUDA", 8: "ROI_ERR_TIMEOUT", 9: "ROI_ERR_OPT"}
 
 
 class RoiError(RuntimeError):
@@ -37,6 +38,12 @@ class NoiseState(ctypes.Structure):
     """roi_noise_state: seed, step, tensor_id, lambda (sampling temperature), row_offset."""
     _fields_ = [("seed", ctypes.c_uint64), ("step", ctypes.c_uint32), ("tensor_id", ctypes.c_uint32),
                 ("lam", ctypes.c_float), ("row_offset", ctypes.c_int64)]
+
+
+class AdamW(ctypes.Structure):
+    """roi_adamw: lr, beta1, beta2, eps, weight_decay, t (1-based step count)."""
+    _fields_ = [("lr", ctypes.c_float), ("beta1", ctypes.c_float), ("beta2", ctypes.c_float),
+                ("eps", ctypes.c_float), ("weight_decay", ctypes.c_float), ("t", ctypes.c_uint32)]
 
 
 _LIB = None
@@ -59,6 +66,10 @@ def lib() -> ctypes.CDLL:
     L.roi_mask_fwd_st.argtypes = [_P, _P, i32, i32, f32, ctypes.POINTER(NoiseState), i64, i64, _P, _P, _P, _P]
     L.roi_mask_bwd_st.argtypes = [_P, _P, ctypes.POINTER(NoiseState), i32, i32, _P, _P, f32, i64, i64, _P, _P, _P]
     L.roi_export_compressed_2of4.argtypes = [_P, _P, i64, i64, _P, _P, _P]
+    L.roi_mask_bwd_adamw.argtypes = [_P, _P, ctypes.POINTER(NoiseState), i32, i32, _P, f32, i64, i64, _P, _P,
+                                     ctypes.POINTER(AdamW), _P, _P, _P]
+    L.roi_anneal.argtypes = [f32, f32, u32, u32]
+    L.roi_anneal.restype = f32
     L.roi_hard_mask_export.argtypes = [_P, i32, i32, i64, i64, _P, _P, _P, _P]
     L.roi_device_status.argtypes = [_P]
     L.roi_noise_words.argtypes = [ctypes.POINTER(NoiseState), i64, i64, _P, _P]
@@ -69,7 +80,7 @@ def lib() -> ctypes.CDLL:
     L.roi_launch_count.restype = ctypes.c_uint64
     for name in ("roi_mask_fwd", "roi_mask_fwd_ex", "roi_mask_bwd", "roi_hard_mask_export", "roi_device_status",
                  "roi_noise_words", "roi_gumbel_noise", "roi_mask_fwd_st", "roi_mask_bwd_st",
-                 "roi_export_compressed_2of4"):
+                 "roi_export_compressed_2of4", "roi_mask_bwd_adamw"):
         getattr(L, name).restype = i32
     _LIB = L
     return L
@@ -196,6 +207,30 @@ def roi_mask_bwd_st(logits, W, state: NoiseState, N, M, dWm, hard, tau, out_dlog
     s = lib().roi_mask_bwd_st(_ptr(logits), _ptr(W), ctypes.byref(st), int(N), int(M), _ptr(dWm), _ptr(hard),
                               float(tau), rows, cols, _ptr(out_dlogits), _ptr(out_dW), _stream(stream))
     _raise(s, "roi_mask_bwd_st")
+
+
+def roi_mask_bwd_adamw(logits, W, state: NoiseState, N, M, dWm, tau, m, v, opt: AdamW, out_dlogits=None,
+                       out_dW=None, stream=None):
+    """Backward fused with one AdamW step: `logits`, `m`, `v` are updated in place."""
+    import torch
+    rows, cols = logits.shape
+    _check_tensor(logits, "logits", torch.float32)
+    _check_tensor(W, "W", torch.bfloat16, (rows, cols))
+    _check_tensor(dWm, "dWm", torch.bfloat16, (rows, cols))
+    _check_tensor(m, "m", torch.float32, (rows, cols))
+    _check_tensor(v, "v", torch.float32, (rows, cols))
+    _check_tensor(out_dlogits, "out_dlogits", torch.float32, (rows, cols))
+    _check_tensor(out_dW, "out_dW", torch.bfloat16, (rows, cols))
+    st = state if isinstance(state, NoiseState) else NoiseState(*state)
+    s = lib().roi_mask_bwd_adamw(_ptr(logits), _ptr(W), ctypes.byref(st), int(N), int(M), _ptr(dWm), float(tau),
+                                 rows, cols, _ptr(m), _ptr(v), ctypes.byref(opt), _ptr(out_dlogits), _ptr(out_dW),
+                                 _stream(stream))
+    _raise(s, "roi_mask_bwd_adamw")
+
+
+def roi_anneal(init, end, t, T_anneal):
+    """Eq. 9: max(end, init * (end / init) ** (t / T_anneal)), evaluated by the library."""
+    return float(lib().roi_anneal(float(init), float(end), int(t), int(T_anneal)))
 
 
 def roi_export_compressed_2of4(logits, W, out_values, out_meta, stream=None):

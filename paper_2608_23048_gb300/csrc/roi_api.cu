@@ -154,22 +154,37 @@ roi_status roi_mask_fwd(const float* logits, const roi_bf16* W, int N, int M, fl
   return roi_mask_fwd_ex(logits, W, N, M, tau, &st, rows, cols, out_Wm, out_soft, out_hard, stream);
 }
 
+// The fused optimizer of roi_mask_bwd_adamw: logits updated in place, moments m, v.
+struct FusedAdamW {
+  float* phi;
+  float* m;
+  float* v;
+  AdamW opt;
+};
+
 static roi_status mask_bwd(const float* logits, const roi_bf16* W, const roi_noise_state* st, int N, int M,
                            const roi_bf16* dWm, const uint32_t* hard, float tau, int64_t rows, int64_t cols,
-                           float* out_dlogits, roi_bf16* out_dW, void* stream) {
+                           float* out_dlogits, roi_bf16* out_dW, const FusedAdamW* fo, void* stream) {
   if (st == nullptr) return ROI_ERR_NULL;
   roi_status s = check_common(N, M, tau, rows, cols);
   if (s != ROI_OK) return s;
   if (st->row_offset < 0) return ROI_ERR_SHAPE;
   if (!finite_positive(st->lambda)) return ROI_ERR_TAU;
   if (rows == 0) return ROI_OK;
-  if (logits == nullptr || W == nullptr || dWm == nullptr || out_dlogits == nullptr) return ROI_ERR_NULL;
+  if (logits == nullptr || W == nullptr || dWm == nullptr || (out_dlogits == nullptr && fo == nullptr))
+    return ROI_ERR_NULL;
+  if (fo != nullptr && (fo->m == nullptr || fo->v == nullptr)) return ROI_ERR_NULL;
   if (!aligned16(logits) || !aligned16(W) || !aligned16(dWm) || !aligned16(out_dlogits) || !aligned16(out_dW))
     return ROI_ERR_ALIGN;
+  if (fo != nullptr && (!aligned16(fo->m) || !aligned16(fo->v))) return ROI_ERR_ALIGN;
   const int64_t E = rows * cols;
-  const Range in[4] = {{logits, uint64_t(E) * 4}, {W, uint64_t(E) * 2}, {dWm, uint64_t(E) * 2},
+  // with the fused optimizer the logits are updated in place: they count as an
+  // output for the overlap check against every other tensor (but not themselves)
+  const Range in[4] = {{fo ? nullptr : logits, uint64_t(E) * 4}, {W, uint64_t(E) * 2}, {dWm, uint64_t(E) * 2},
                        {hard, uint64_t((E + 31) / 32) * 4}};
-  const Range out[2] = {{out_dlogits, uint64_t(E) * 4}, {out_dW, uint64_t(E) * 2}};
+  const Range out[5] = {{out_dlogits, uint64_t(E) * 4}, {out_dW, uint64_t(E) * 2},
+                        {fo ? logits : nullptr, uint64_t(E) * 4}, {fo ? fo->m : nullptr, uint64_t(E) * 4},
+                        {fo ? fo->v : nullptr, uint64_t(E) * 4}};
   if (any_alias(in, out)) return ROI_ERR_ALIAS;
   if (E == 0) return ROI_OK;
   BwdCall c;
@@ -179,6 +194,10 @@ static roi_status mask_bwd(const float* logits, const roi_bf16* W, const roi_noi
   c.dphi = out_dlogits;
   c.dW = out_dW;
   c.hard_in = hard;
+  c.phi_out = fo ? fo->phi : nullptr;
+  c.m = fo ? fo->m : nullptr;
+  c.v = fo ? fo->v : nullptr;
+  c.opt = fo ? fo->opt : AdamW{};
   c.E = E;
   c.N = N;
   c.M = M;
@@ -193,7 +212,7 @@ static roi_status mask_bwd(const float* logits, const roi_bf16* W, const roi_noi
 roi_status roi_mask_bwd(const float* logits, const roi_bf16* W, const roi_noise_state* st, int N, int M,
                         const roi_bf16* dWm, float tau, int64_t rows, int64_t cols, float* out_dlogits,
                         roi_bf16* out_dW, void* stream) {
-  return mask_bwd(logits, W, st, N, M, dWm, nullptr, tau, rows, cols, out_dlogits, out_dW, stream);
+  return mask_bwd(logits, W, st, N, M, dWm, nullptr, tau, rows, cols, out_dlogits, out_dW, nullptr, stream);
 }
 
 roi_status roi_mask_bwd_st(const float* logits, const roi_bf16* W, const roi_noise_state* st, int N, int M,
@@ -202,7 +221,40 @@ roi_status roi_mask_bwd_st(const float* logits, const roi_bf16* W, const roi_noi
   if (out_dW != nullptr && hard == nullptr && rows > 0) return ROI_ERR_NULL;
   if (!aligned16(hard)) return ROI_ERR_ALIGN;
   return mask_bwd(logits, W, st, N, M, dWm, out_dW != nullptr ? hard : nullptr, tau, rows, cols, out_dlogits,
-                  out_dW, stream);
+                  out_dW, nullptr, stream);
+}
+
+roi_status roi_mask_bwd_adamw(float* logits, const roi_bf16* W, const roi_noise_state* st, int N, int M,
+                              const roi_bf16* dWm, float tau, int64_t rows, int64_t cols, float* m, float* v,
+                              const roi_adamw* opt, float* out_dlogits, roi_bf16* out_dW, void* stream) {
+  if (opt == nullptr) return ROI_ERR_NULL;
+  const bool ok = std::isfinite(opt->lr) && opt->lr >= 0.0f && opt->beta1 >= 0.0f && opt->beta1 < 1.0f &&
+                  opt->beta2 >= 0.0f && opt->beta2 < 1.0f && finite_positive(opt->eps) &&
+                  std::isfinite(opt->weight_decay) && opt->weight_decay >= 0.0f && opt->t >= 1;
+  if (!ok) return ROI_ERR_OPT;
+  FusedAdamW fo;
+  fo.phi = logits;
+  fo.m = m;
+  fo.v = v;
+  // constants rounded to float as the float32 statement of the step forms them
+  fo.opt.b1 = opt->beta1;
+  fo.opt.omb1 = 1.0f - opt->beta1;
+  fo.opt.b2 = opt->beta2;
+  fo.opt.omb2 = 1.0f - opt->beta2;
+  fo.opt.eps = opt->eps;
+  fo.opt.decay = 1.0f - opt->lr * opt->weight_decay;
+  const double t = static_cast<double>(opt->t);
+  fo.opt.step = static_cast<float>(static_cast<double>(opt->lr) / (1.0 - std::pow(static_cast<double>(opt->beta1), t)));
+  fo.opt.r = static_cast<float>(1.0 / std::sqrt(1.0 - std::pow(static_cast<double>(opt->beta2), t)));
+  return mask_bwd(logits, W, st, N, M, dWm, nullptr, tau, rows, cols, out_dlogits, out_dW, &fo, stream);
+}
+
+float roi_anneal(float init, float end, uint32_t t, uint32_t T_anneal) {
+  if (T_anneal == 0) return end;
+  const double x = static_cast<double>(init) *
+                   std::pow(static_cast<double>(end) / static_cast<double>(init),
+                            static_cast<double>(t) / static_cast<double>(T_anneal));
+  return static_cast<float>(x > static_cast<double>(end) ? x : static_cast<double>(end));
 }
 
 roi_status roi_export_compressed_2of4(const float* logits, const roi_bf16* W, int64_t rows, int64_t cols,
@@ -296,6 +348,7 @@ const char* roi_status_string(roi_status s) {
     case ROI_ERR_ALIAS: return "an output overlaps an input or another output";
     case ROI_ERR_CUDA: return "CUDA error while launching";
     case ROI_ERR_TIMEOUT: return "a kernel gave up waiting on its own copies";
+    case ROI_ERR_OPT: return "bad optimizer settings: need lr, weight_decay >= 0 finite, 0 <= beta < 1, eps > 0, t >= 1";
   }
   return "unknown status";
 }

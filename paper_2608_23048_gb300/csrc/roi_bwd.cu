@@ -29,6 +29,21 @@ template <int M>
 constexpr size_t kHistOffset = (tile_smem_bytes<Cfg<M>::kTile, Cfg<M>::kStages>(8) + 15) & ~size_t(15);
 template <int N, int M>
 constexpr size_t kHistBytes = M == 8 ? size_t(N - 1) * M * Cfg<M>::kThreads * sizeof(F2) : 0;
+// Fused optimizer with the step history in shared memory (M = 8): each thread's
+// AdamW moments (two groups, m and v) are staged behind the history by per-thread
+// async copies issued when the groups start, so their latency hides behind the
+// relaxation without holding registers.
+template <int N, int M>
+constexpr size_t kMomOffset = (kHistOffset<M> + kHistBytes<N, M> + 15) & ~size_t(15);
+template <int M>
+constexpr size_t kMomBytes = size_t(2) * M * 2 * sizeof(float) * Cfg<M>::kThreads;
+
+// This thread's moment slot (M = 8 fused optimizer) in the dynamic shared memory.
+extern __shared__ __align__(128) uint8_t roi_bwd_smem[];
+template <int N, int M>
+__device__ __forceinline__ float4* moment_slot() {
+  return reinterpret_cast<float4*>(roi_bwd_smem + kMomOffset<N, M>) + threadIdx.x;
+}
 
 struct BwdArgs {
   const float* phi;
@@ -42,6 +57,14 @@ struct BwdArgs {
   float tau, inv_tau;
   NoiseParams np;
   unsigned int* status;
+};
+
+// The fused optimizer's arguments (read only by the OPT instantiations).
+struct BwdOptArgs {
+  float* phi_out;  // logits updated in place
+  float* m;
+  float* v;
+  AdamW opt;
 };
 
 __device__ __forceinline__ void unpack4(uint2 q, float* out) {
@@ -158,10 +181,10 @@ __device__ __forceinline__ void bwd_inputs(const float* const* phi_g, const uint
 // whole history stays in registers.  With HIST (M = 8) registers are tight:
 // the keys die after the forward relaxation (a flagged group re-forms them) and
 // the upstream gradients are formed only for the sweep.
-template <int N, int M, bool TAU1, class V, bool HIST = false, bool ST = false>
+template <int N, int M, bool TAU1, class V, bool HIST = false, bool ST = false, bool OPT = false>
 __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint16_t* const* W_g,
                                            const uint16_t* const* dWm_g, const int64_t* e0, const BwdArgs& a,
-                                           V* hist = nullptr) {
+                                           const BwdOptArgs& o, V* hist = nullptr) {
   constexpr int L = vlanes<V>();
   // straight-through: the forward's hard bits of these groups, loaded now so the
   // load's latency hides behind the relaxation
@@ -171,6 +194,33 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
     for (int h = 0; h < L; ++h)
 #pragma unroll
       for (int s = 0; s < M / 4; ++s) keep[h][s] = hard4(a.hard_in, e0[h] + 4 * s);
+  }
+  // fused optimizer: the moments, fetched now for the epilogue, into registers
+  // (M = 4) or into this thread's shared-memory slot `mom` (with HIST)
+  constexpr bool kPrefetchMoments = OPT && !HIST;
+  constexpr bool kStageMoments = OPT && HIST;
+  constexpr int kT = Cfg<M>::kThreads;
+  if constexpr (kStageMoments) {
+    float4* mom = moment_slot<N, M>();
+#pragma unroll
+    for (int h = 0; h < L; ++h)
+#pragma unroll
+      for (int s = 0; s < M / 4; ++s) {
+        cp_async16(mom + (2 * (h * (M / 4) + s)) * kT, o.m + e0[h] + 4 * s);
+        cp_async16(mom + (2 * (h * (M / 4) + s) + 1) * kT, o.v + e0[h] + 4 * s);
+      }
+    cp_async_commit();
+  }
+  float4 mom_m[kPrefetchMoments ? L : 1][kPrefetchMoments ? M / 4 : 1];
+  float4 mom_v[kPrefetchMoments ? L : 1][kPrefetchMoments ? M / 4 : 1];
+  if constexpr (kPrefetchMoments) {
+#pragma unroll
+    for (int h = 0; h < L; ++h)
+#pragma unroll
+      for (int s = 0; s < M / 4; ++s) {
+        mom_m[h][s] = reinterpret_cast<const float4*>(o.m + e0[h])[s];
+        mom_v[h][s] = reinterpret_cast<const float4*>(o.v + e0[h])[s];
+      }
   }
   using Steps = typename std::conditional<HIST, SmemSteps<N, M, V, Cfg<M>::kThreads>, RegSteps<N, M, V>>::type;
   FastGroup<N, M, TAU1, true, V, Steps> fg;
@@ -221,6 +271,7 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
   // dL/dphi = dL/dkappa / lambda
 #pragma unroll
   for (int l = 0; l < M; ++l) dkv[l] = vmul(dkv[l], vconst<V>(a.np.inv_lam));
+  if constexpr (kStageMoments) cp_async_wait_all();
 #pragma unroll
   for (int h = 0; h < L; ++h) {
     float dk[M];
@@ -261,17 +312,36 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
         }
       }
     }
+    if constexpr (OPT) {
+      // fused AdamW step on these logits (their old values are still in phi_g)
 #pragma unroll
-    for (int s = 0; s < M / 4; ++s)
-      reinterpret_cast<float4*>(a.dphi + e0[h])[s] = make_float4(dk[4 * s], dk[4 * s + 1], dk[4 * s + 2], dk[4 * s + 3]);
+      for (int s = 0; s < M / 4; ++s) {
+        const float g4[4] = {dk[4 * s], dk[4 * s + 1], dk[4 * s + 2], dk[4 * s + 3]};
+        if constexpr (kPrefetchMoments) {
+          adamw4(o.phi_out, o.m, o.v, e0[h] + 4 * s, reinterpret_cast<const float4*>(phi_g[h])[s], g4, o.opt,
+                 mom_m[h][s], mom_v[h][s]);
+        } else if constexpr (kStageMoments) {
+          const float4* mom = moment_slot<N, M>();
+          adamw4(o.phi_out, o.m, o.v, e0[h] + 4 * s, reinterpret_cast<const float4*>(phi_g[h])[s], g4, o.opt,
+                 mom[(2 * (h * (M / 4) + s)) * kT], mom[(2 * (h * (M / 4) + s) + 1) * kT]);
+        } else {
+          adamw4(o.phi_out, o.m, o.v, e0[h] + 4 * s, reinterpret_cast<const float4*>(phi_g[h])[s], g4, o.opt);
+        }
+      }
+    }
+    if (!OPT || a.dphi != nullptr) {
+#pragma unroll
+      for (int s = 0; s < M / 4; ++s)
+        reinterpret_cast<float4*>(a.dphi + e0[h])[s] = make_float4(dk[4 * s], dk[4 * s + 1], dk[4 * s + 2], dk[4 * s + 3]);
+    }
   }
 }
 
-// ST: straight-through dW from the forward's hard bits (a separate instantiation,
-// so the soft kernel's code is not touched by it)
-template <int N, int M, bool TAU1, bool ST>
-__global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_kernel(BwdArgs a) {
-  extern __shared__ __align__(128) uint8_t smem[];
+// ST: straight-through dW from the forward's hard bits; OPT: fused AdamW step on
+// the logits (separate instantiations, so the plain kernel's code is not touched)
+template <int N, int M, bool TAU1, bool ST, bool OPT>
+__global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_kernel(BwdArgs a, BwdOptArgs o) {
+  uint8_t* smem = roi_bwd_smem;
   using C = Cfg<M>;
   constexpr int kT = C::kTile;
   TileSrc<3> src;
@@ -296,12 +366,12 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_
           const uint16_t* pd[2] = {sdW + g0 * M, sdW + g1 * M};
           const int64_t e0[2] = {base + g0 * M, base + g1 * M};
           if constexpr (M == 4) {
-            bwd_groups<N, M, TAU1, F2, false, ST>(pp, pw, pd, e0, a);
+            bwd_groups<N, M, TAU1, F2, false, ST, OPT>(pp, pw, pd, e0, a, o);
           } else {
             // M = 8: the paired step history does not fit the register file; steps
             // 0 .. N-2 go to shared memory behind the tile ring
             F2* hist = reinterpret_cast<F2*>(smem + kHistOffset<M>) + threadIdx.x;
-            bwd_groups<N, M, TAU1, F2, true, ST>(pp, pw, pd, e0, a, hist);
+            bwd_groups<N, M, TAU1, F2, true, ST, OPT>(pp, pw, pd, e0, a, o, hist);
           }
         }
       });
@@ -315,12 +385,12 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_
       const uint16_t* pw[1] = {a.W + t0 + gi * M};
       const uint16_t* pd[1] = {a.dWm + t0 + gi * M};
       const int64_t e0[1] = {t0 + gi * M};
-      bwd_groups<N, M, TAU1, float, false, ST>(pp, pw, pd, e0, a);
+      bwd_groups<N, M, TAU1, float, false, ST, OPT>(pp, pw, pd, e0, a, o);
     }
   }
 }
 
-__global__ void __launch_bounds__(128) roi_bwd_generic_kernel(BwdArgs a, int N, int M) {
+__global__ void __launch_bounds__(128) roi_bwd_generic_kernel(BwdArgs a, BwdOptArgs o, int N, int M) {
   const int64_t groups = a.E / M;
   for (int64_t g = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; g < groups;
        g += int64_t(gridDim.x) * blockDim.x) {
@@ -336,7 +406,15 @@ __global__ void __launch_bounds__(128) roi_bwd_generic_kernel(BwdArgs a, int N, 
     ex.backward(c, N, M, a.tau, dk);
     for (int l = 0; l < M; ++l) {
       const int64_t e = e0 + l;
-      a.dphi[e] = dk[l] * a.np.inv_lam;
+      const float g = dk[l] * a.np.inv_lam;
+      if (a.dphi != nullptr) a.dphi[e] = g;
+      if (o.phi_out != nullptr) {
+        float ph = a.phi[e], mm = o.m[e], vv = o.v[e];
+        adamw_elem(ph, g, mm, vv, o.opt);
+        o.phi_out[e] = ph;
+        o.m[e] = mm;
+        o.v[e] = vv;
+      }
       if (a.dW != nullptr) {
         if (a.hard_in != nullptr) {
           a.dW[e] = ((a.hard_in[e >> 5] >> (e & 31)) & 1u) ? a.dWm[e] : uint16_t(0);
@@ -352,11 +430,14 @@ struct LaunchCache {
   int per_sm[64] = {0};
 };
 
-template <int N, int M, bool TAU1, bool ST>
-int launch_tiles(const BwdArgs& a, cudaStream_t stream) {
+template <int N, int M, bool TAU1, bool ST, bool OPT>
+int launch_tiles(const BwdArgs& a, const BwdOptArgs& o, cudaStream_t stream) {
   using C = Cfg<M>;
-  auto kern = roi_bwd_kernel<N, M, TAU1, ST>;
-  const size_t smem = kHistBytes<N, M> > 0 ? kHistOffset<M> + kHistBytes<N, M> : tile_smem_bytes<C::kTile, C::kStages>(8);
+  auto kern = roi_bwd_kernel<N, M, TAU1, ST, OPT>;
+  const size_t smem = kHistBytes<N, M> == 0 ? tile_smem_bytes<C::kTile, C::kStages>(8)
+                      : OPT               ? kMomOffset<N, M> + kMomBytes<M>
+                                          : kHistOffset<M> + kHistBytes<N, M>;
+  static_assert(kMomOffset<N, M> + kMomBytes<M> <= 232448, "shared memory per CTA");
   static LaunchCache cache;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return -1;
@@ -369,15 +450,18 @@ int launch_tiles(const BwdArgs& a, cudaStream_t stream) {
   }
   const int64_t cap = int64_t(sm_count()) * cache.per_sm[dev];
   const int grid = int(a.full_tiles < 1 ? 1 : (a.full_tiles < cap ? a.full_tiles : cap));
-  kern<<<grid, C::kThreads, smem, stream>>>(a);
+  kern<<<grid, C::kThreads, smem, stream>>>(a, o);
   return cudaGetLastError() == cudaSuccess ? 1 : -1;
 }
 
 template <int N, int M>
-int launch_nm(const BwdArgs& a, cudaStream_t stream) {
+int launch_nm(const BwdArgs& a, const BwdOptArgs& o, cudaStream_t stream) {
+  const bool t1 = a.tau == 1.0f;
+  if (o.phi_out != nullptr)
+    return t1 ? launch_tiles<N, M, true, false, true>(a, o, stream) : launch_tiles<N, M, false, false, true>(a, o, stream);
   if (a.hard_in != nullptr && a.dW != nullptr)
-    return a.tau == 1.0f ? launch_tiles<N, M, true, true>(a, stream) : launch_tiles<N, M, false, true>(a, stream);
-  return a.tau == 1.0f ? launch_tiles<N, M, true, false>(a, stream) : launch_tiles<N, M, false, false>(a, stream);
+    return t1 ? launch_tiles<N, M, true, true, false>(a, o, stream) : launch_tiles<N, M, false, true, false>(a, o, stream);
+  return t1 ? launch_tiles<N, M, true, false, false>(a, o, stream) : launch_tiles<N, M, false, false, false>(a, o, stream);
 }
 
 }  // namespace
@@ -390,22 +474,27 @@ int launch_bwd(const BwdCall& c) {
   a.dphi = c.dphi;
   a.dW = c.dW;
   a.hard_in = c.hard_in;
+  BwdOptArgs o;
+  o.phi_out = c.phi_out;
+  o.m = c.m;
+  o.v = c.v;
+  o.opt = c.opt;
   a.E = c.E;
   a.full_tiles = c.E / (c.M == 8 ? Cfg<8>::kTile : Cfg<4>::kTile);
   a.tau = c.tau;
   a.inv_tau = 1.0f / c.tau;
   a.np = c.np;
   a.status = c.status;
-  if (c.N == 2 && c.M == 4) return launch_nm<2, 4>(a, c.stream);
-  if (c.N == 4 && c.M == 8) return launch_nm<4, 8>(a, c.stream);
-  if (c.N == 2 && c.M == 8) return launch_nm<2, 8>(a, c.stream);
+  if (c.N == 2 && c.M == 4) return launch_nm<2, 4>(a, o, c.stream);
+  if (c.N == 4 && c.M == 8) return launch_nm<4, 8>(a, o, c.stream);
+  if (c.N == 2 && c.M == 8) return launch_nm<2, 8>(a, o, c.stream);
   if (slice_supported(c.N, c.M)) return launch_slice_bwd(c);
   const int64_t groups = c.E / c.M;
   int64_t blocks = (groups + 127) / 128;
   const int64_t cap = int64_t(sm_count()) * 16;
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
-  roi_bwd_generic_kernel<<<int(blocks), 128, 0, c.stream>>>(a, c.N, c.M);
+  roi_bwd_generic_kernel<<<int(blocks), 128, 0, c.stream>>>(a, o, c.N, c.M);
   return cudaGetLastError() == cudaSuccess ? 1 : -1;
 }
 

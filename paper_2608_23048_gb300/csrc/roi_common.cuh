@@ -60,6 +60,40 @@ __device__ __forceinline__ uint2 keep4(uint2 q, uint32_t keep) {
 __device__ __forceinline__ uint32_t hard4(const uint32_t* hard, int64_t e) {
   return (hard[e >> 5] >> (uint32_t(e) & 31u)) & 0xfu;
 }
+// One AdamW step on a logit (decoupled weight decay, bias-corrected moments):
+//   phi <- phi (1 - lr wd); m <- b1 m + (1 - b1) g; v <- b2 v + (1 - b2) g^2;
+//   phi <- phi - (step m) / (sqrt(v) r + eps),  step = lr / (1 - b1^t), r = 1 / sqrt(1 - b2^t).
+// Explicitly rounded operations, correctly rounded divide and square root.
+struct AdamW {
+  float b1, omb1, b2, omb2, eps, decay, step, r;  // decay = 1 - lr wd, omb_i = 1 - b_i
+};
+__device__ __forceinline__ void adamw_elem(float& phi, float g, float& m, float& v, const AdamW& o) {
+  phi = __fmul_rn(phi, o.decay);
+  m = __fadd_rn(__fmul_rn(o.b1, m), __fmul_rn(o.omb1, g));
+  v = __fadd_rn(__fmul_rn(o.b2, v), __fmul_rn(o.omb2, __fmul_rn(g, g)));
+  const float den = __fadd_rn(__fmul_rn(__fsqrt_rn(v), o.r), o.eps);
+  phi = __fsub_rn(phi, __fdiv_rn(__fmul_rn(o.step, m), den));
+}
+// The step for four consecutive logits at `e` (16-byte aligned): old logits phi4
+// (from the tile stage or global memory), gradients g, moments mm, vv; the new
+// logits and moments are stored.
+__device__ __forceinline__ void adamw4(float* phi_out, float* m, float* v, int64_t e, float4 phi4,
+                                       const float (&g)[4], const AdamW& o, float4 mm, float4 vv) {
+  adamw_elem(phi4.x, g[0], mm.x, vv.x, o);
+  adamw_elem(phi4.y, g[1], mm.y, vv.y, o);
+  adamw_elem(phi4.z, g[2], mm.z, vv.z, o);
+  adamw_elem(phi4.w, g[3], mm.w, vv.w, o);
+  *reinterpret_cast<float4*>(phi_out + e) = phi4;
+  *reinterpret_cast<float4*>(m + e) = mm;
+  *reinterpret_cast<float4*>(v + e) = vv;
+}
+// ... loading the moments here.
+__device__ __forceinline__ void adamw4(float* phi_out, float* m, float* v, int64_t e, float4 phi4,
+                                       const float (&g)[4], const AdamW& o) {
+  adamw4(phi_out, m, v, e, phi4, g, o, *reinterpret_cast<const float4*>(m + e),
+         *reinterpret_cast<const float4*>(v + e));
+}
+
 // Two floats -> two bf16 (round to nearest even), packed low|high.
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
@@ -727,5 +761,13 @@ __device__ __forceinline__ void bulk_g2s(void* dst_smem, const void* src_gmem, u
       "l"(src_gmem), "r"(bytes), "r"(smem_addr(bar))
       : "memory");
 }
+
+// Per-thread 16-byte global -> shared copy (cp.async, L2 only); the issuing
+// thread waits for its own copies with cp_async_wait_all before reading them.
+__device__ __forceinline__ void cp_async16(void* dst_smem, const void* src_gmem) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst_smem)), "l"(src_gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
 }  // namespace roi

@@ -30,6 +30,10 @@ struct BwdCall {
   float* dphi;
   uint16_t* dW;     // nullable
   const uint32_t* hard_in;  // nullable; straight-through: dW = dWm where set, +0 elsewhere
+  float* phi_out;   // nullable; fused AdamW: the logits updated in place (== phi)
+  float* m;         // AdamW first and second moments (with phi_out)
+  float* v;
+  AdamW opt;
   int64_t E;
   int N, M;
   float tau;

@@ -109,6 +109,10 @@ struct SliceArgs {
   uint16_t* dW;
   bool st;                  // straight-through forward: Wm = W where the hard mask is set
   const uint32_t* hard_in;  // straight-through backward: dW = dWm where the forward's bit is set
+  float* phi_out;           // fused AdamW: logits updated in place
+  float* m;
+  float* v;
+  AdamW opt;
   int64_t E;
   int64_t full_tiles;
   float tau, inv_tau;
@@ -449,8 +453,9 @@ __device__ __forceinline__ void bwd_slots(const float* const* p, const uint16_t*
 #pragma unroll
   for (int h = 0; h < L; ++h) {
     if (!((flag >> h) & 1u)) {
-      *reinterpret_cast<float4*>(a.dphi + e0[h]) =
-          make_float4(lane_of(dk[0], h), lane_of(dk[1], h), lane_of(dk[2], h), lane_of(dk[3], h));
+      const float g4[4] = {lane_of(dk[0], h), lane_of(dk[1], h), lane_of(dk[2], h), lane_of(dk[3], h)};
+      if (a.dphi != nullptr) *reinterpret_cast<float4*>(a.dphi + e0[h]) = make_float4(g4[0], g4[1], g4[2], g4[3]);
+      if (a.phi_out != nullptr) adamw4(a.phi_out, a.m, a.v, e0[h], *reinterpret_cast<const float4*>(p[h]), g4, a.opt);
     } else if (q == 0) {
       float k[M], cc[M], S[M], dkk[M];
       group_keys_all<N, M>(p[h], e0[h], a.np, k);
@@ -467,9 +472,12 @@ __device__ __forceinline__ void bwd_slots(const float* const* p, const uint16_t*
       ex.backward(cc, N, M, a.tau, dkk);
 #pragma unroll 1
       for (int s = 0; s < SL; ++s) {
-        *reinterpret_cast<float4*>(a.dphi + e0[h] + 4 * s) =
-            make_float4(__fmul_rn(dkk[4 * s], a.np.inv_lam), __fmul_rn(dkk[4 * s + 1], a.np.inv_lam),
-                        __fmul_rn(dkk[4 * s + 2], a.np.inv_lam), __fmul_rn(dkk[4 * s + 3], a.np.inv_lam));
+        const float g4[4] = {__fmul_rn(dkk[4 * s], a.np.inv_lam), __fmul_rn(dkk[4 * s + 1], a.np.inv_lam),
+                             __fmul_rn(dkk[4 * s + 2], a.np.inv_lam), __fmul_rn(dkk[4 * s + 3], a.np.inv_lam)};
+        if (a.dphi != nullptr)
+          *reinterpret_cast<float4*>(a.dphi + e0[h] + 4 * s) = make_float4(g4[0], g4[1], g4[2], g4[3]);
+        if (a.phi_out != nullptr)
+          adamw4(a.phi_out, a.m, a.v, e0[h] + 4 * s, reinterpret_cast<const float4*>(p[h])[s], g4, a.opt);
         if (a.dW != nullptr && a.hard_in == nullptr) {
           float dv[4], sv[4];
           unpack_bf16x4(*reinterpret_cast<const uint2*>(dw[h] + 4 * s), dv);
@@ -670,6 +678,10 @@ int launch_slice_bwd(const BwdCall& c) {
   a.dphi = c.dphi;
   a.dW = c.dW;
   a.hard_in = c.hard_in;
+  a.phi_out = c.phi_out;
+  a.m = c.m;
+  a.v = c.v;
+  a.opt = c.opt;
   a.E = c.E;
   a.full_tiles = c.E / kTile;
   a.tau = c.tau;

@@ -95,8 +95,32 @@ def test_validation_codes(L):
     assert L.roi_export_compressed_2of4(_fake(A), _fake(B), 4, 8, _fake(C + 2), _fake(D), None) == 5
     assert L.roi_export_compressed_2of4(_fake(A), _fake(B), 4, 8, _fake(A + 16), _fake(D), None) == 6
     assert L.roi_export_compressed_2of4(None, None, 0, 8, None, None, None) == 0
-    for s in range(9):
+    # fused optimizer: settings checked; logits are in/out and must not overlap m, v or outputs
+    opt = roi.AdamW(1e-3, 0.9, 0.95, 1e-8, 0.05, 1)
+    bad = roi.AdamW(1e-3, 1.0, 0.95, 1e-8, 0.05, 1)
+    zero_t = roi.AdamW(1e-3, 0.9, 0.95, 1e-8, 0.05, 0)
+    def bwd_opt(o, m=C, v=D, logits=A, dl=None):
+        return L.roi_mask_bwd_adamw(_fake(logits), _fake(B), ctypes.byref(st), 2, 4, _fake(E), 1.0, 4, 8,
+                                    _fake(m) if m else None, _fake(v) if v else None,
+                                    ctypes.byref(o) if o is not None else None, _fake(dl) if dl else None, None, None)
+    assert bwd_opt(None) == 1
+    assert bwd_opt(bad) == 9 and bwd_opt(zero_t) == 9
+    assert bwd_opt(opt, m=None) == 1
+    assert bwd_opt(opt, m=A + 64) == 6               # m overlaps the logits
+    assert bwd_opt(opt, dl=D + 16) == 6              # gradient output overlaps v
+    assert bwd_opt(opt, v=D + 8) == 5
+    assert L.roi_mask_bwd_adamw(None, None, ctypes.byref(st), 2, 4, None, 1.0, 0, 8, None, None,
+                                ctypes.byref(opt), None, None, None) == 0
+    for s in range(10):
         assert L.roi_status_string(s)
+
+
+def test_anneal_schedule_on_the_host(L):
+    from oracle import roi_oracle as O
+    for t in (0, 1, 700, 1500, 1999):    # the float result of the float64 formula: within 2 float ulps
+        for end in (0.05, 0.002):
+            want = float(O.anneal(1.0, end, t, 1500))
+            assert abs(L.roi_anneal(1.0, end, t, 1500) - want) <= 2 * 2.0 ** -24 * want
 
 
 def test_short_form_validates_like_ex(L):

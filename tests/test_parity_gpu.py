@@ -432,3 +432,54 @@ def test_compressed_2of4_export_bit_exact(roi, rows, cols):
     ref = O.export_compressed_2of4(phi.numpy(), WL.bf16_bits(W))
     assert np.array_equal(_u16(values), ref["values"])
     assert np.array_equal(_bits(meta), ref["meta"])
+
+
+ADAMW_CASES = [
+    (37, 1000, 2, 4, 1.0, "logw"),
+    (29, 1536, 4, 8, 1.0, "normal"),
+    (29, 1536, 4, 8, 0.5, "normal"),
+    (9, 1024, 8, 16, 0.5, "logw"),    # warp-slice kernels
+    (13, 960, 3, 4, 1.0, "normal"),   # generic kernels
+]
+
+
+@pytest.mark.parametrize("rows,cols,N,M,tau,kind", ADAMW_CASES)
+def test_backward_fused_with_adamw(roi, rows, cols, N, M, tau, kind):
+    """roi_mask_bwd_adamw: its gradient is roi_mask_bwd's, and the logits / moments it
+    writes are the float32 AdamW step (oracle, same rounded operations) of that
+    gradient, bit for bit; with and without the gradient output."""
+    import torch
+    W, phi, dWm, ph, Wb, dWb = make(rows, cols, kind, data_seed=rows * 5 + M)
+    phi = phi.clone()
+    phi[1, :M] = 100.0 * torch.arange(M, dtype=torch.float32)   # a fallback group
+    ph = phi.numpy()
+    dev = torch.device("cuda")
+    gen = torch.Generator().manual_seed(rows + cols)
+    m0 = (torch.randn(rows, cols, generator=gen) * 1e-6).float()
+    v0 = (torch.rand(rows, cols, generator=gen) * 1e-10).float()
+    st = roi.NoiseState(42, 9, 3, 0.5, 0)
+    f32 = lambda x: float(np.float32(x))
+    lr, b1, b2, eps, wd, t = f32(1e-3), f32(0.9), f32(0.95), f32(1e-8), f32(0.05), 4
+    opt = roi.AdamW(lr, b1, b2, eps, wd, t)
+    phi_d, W_d, dWm_d = phi.to(dev), W.to(dev), dWm.to(dev)
+    g_ref = torch.empty(rows, cols, dtype=torch.float32, device=dev)
+    dW_ref = torch.empty(rows, cols, dtype=torch.bfloat16, device=dev)
+    roi.roi_mask_bwd(phi_d, W_d, st, N, M, dWm_d, tau, g_ref, dW_ref)
+    results = []
+    for with_grad in (True, False):
+        p_io, m, v = phi_d.clone(), m0.to(dev), v0.to(dev)
+        g = torch.empty(rows, cols, dtype=torch.float32, device=dev) if with_grad else None
+        dW = torch.empty(rows, cols, dtype=torch.bfloat16, device=dev) if with_grad else None
+        roi.roi_mask_bwd_adamw(p_io, W_d, st, N, M, dWm_d, tau, m, v, opt, g, dW)
+        roi.roi_device_status()
+        results.append((p_io.cpu().numpy(), m.cpu().numpy(), v.cpu().numpy()))
+        if with_grad:
+            gg, gr = g.cpu().numpy(), g_ref.cpu().numpy()
+            scale = np.abs(gr).reshape(-1, M).max(-1, keepdims=True).repeat(M, -1).reshape(rows, cols)
+            assert np.all(np.abs(gg - gr) <= 1e-6 * scale + 1e-30)
+            assert np.array_equal(_u16(dW), _u16(dW_ref))
+            want = O.adamw_step(ph, gg, m0.numpy(), v0.numpy(), lr, b1, b2, eps, wd, t, dtype=np.float32)
+            for got, exp in zip(results[-1], want):
+                assert np.array_equal(got.view(np.uint32), exp.astype(np.float32).view(np.uint32))
+    for a, b in zip(results[0], results[1]):
+        assert np.array_equal(a.view(np.uint32), b.view(np.uint32))
