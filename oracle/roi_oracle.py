@@ -424,3 +424,19 @@ def adamw_step(phi, g, m, v, lr, beta1, beta2, eps, weight_decay, t, dtype=np.fl
     den = ar.cast(np.sqrt(v)) * r + c(eps)
     phi = phi - (step * m) / den
     return phi, m, v
+
+
+def masked_linear_fwd(X_bits, logits, W_bits, N, M, tau, seed, step, tensor_id=0, lam=1.0,
+                      row_offset=0, dtype=np.float64):
+    """The layer's product with the masked weights (Eq. 5: the linear layer uses
+    W (.) S in place of W): Y[t, r] = sum_c X[t, c] * Wm[r, c], where Wm is
+    mask_fwd's bfloat16 Wm for the same arguments.  X is bfloat16 [T, cols]; the
+    sum of the decoded values is taken in float64 (a plain matrix product; the
+    products of two bfloat16 values are exact there).
+
+    Returns Y [T, rows] (float64), the Wm bits it used, and |X| |Wm|^T, the
+    scale of the rounding error of any other evaluation order."""
+    f = mask_fwd(logits, W_bits, N, M, tau, seed, step, tensor_id, lam, row_offset, dtype)
+    Wm = bf16_to_f32(f["Wm"]).astype(np.float64)
+    X = bf16_to_f32(np.asarray(X_bits)).astype(np.float64)
+    return {"Y": X @ Wm.T, "Wm": f["Wm"], "abs": np.abs(X) @ np.abs(Wm).T}

@@ -12,6 +12,8 @@ of M along in_features) and these value distributions:
   * logits "logw": log(max(|W|, 2^-126)) + N(0, 0.1^2)   (magnitude-initialised)
            "normal": N(0, 1)
   * dWm    ~ N(0, (1e-3)^2), bfloat16 (the upstream gradient of the masked weight)
+  * X      ~ N(0, 1), bfloat16 [T, in_features] (a layer's normalised input
+           activations, for the masked-linear product; seed 7000 + tensor seed)
 Seed of tensor (layer l, projection p in q,k,v,o,gate,up,down = 0..6):
 1000 + 16 * l + p.
 """
@@ -96,6 +98,13 @@ def make_inputs(rows: int, cols: int, logits: str, seed: int, device="cpu"):
         raise ValueError(logits)
     dWm = (torch.randn(rows, cols, generator=g, device=device) * 1e-3).to(torch.bfloat16)
     return W, phi.contiguous(), dWm
+
+
+def make_tokens(T: int, cols: int, seed: int, device="cpu"):
+    """X bf16 [T, cols] ~ N(0, 1): the input tokens of one linear layer."""
+    import torch
+    g = torch.Generator(device=device).manual_seed(7000 + int(seed))
+    return torch.randn(T, cols, generator=g, device=device).to(torch.bfloat16).contiguous()
 
 
 def bf16_bits(t):
