@@ -35,6 +35,7 @@ METRIC = "fused RoI mask fwd+bwd groups/s and HBM GB/s (% of GB300 peak), 1 GPU"
 FWD_BYTES = 4 + 2 + 2 + 1 / 8     # logits, W in; Wm, hard bits out
 BWD_BYTES = 4 + 2 + 2 + 4         # logits, W, dWm in; dlogits out
 FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
 
 
 def parse_args():
@@ -52,10 +53,12 @@ def parse_args():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--layers", type=int, default=None, help="only the first L layers (profiling cases)")
     p.add_argument("--proj", default=None, help="comma-separated projections to keep, e.g. gate")
-    p.add_argument("--op", choices=("mask", "st", "adamw", "export2of4"), default="mask",
+    p.add_argument("--op", choices=("mask", "st", "adamw", "export2of4", "linear"), default="mask",
                    help="mask: the fwd+bwd step (default); st: the straight-through pair with dW; "
                         "adamw: fwd + the backward fused with the logits' AdamW step; "
-                        "export2of4: the compressed 2:4 export (one GPU)")
+                        "export2of4: the compressed 2:4 export; linear: the masked linear forward "
+                        "(mask formed in a tensor-core GEMM's prologue) over --tokens tokens (one GPU)")
+    p.add_argument("--tokens", type=int, default=256, help="tokens per layer for --op linear (1..256)")
     return p.parse_args()
 
 
@@ -629,10 +632,140 @@ def run_variant(args):
                       "roofline": roofline, "clocks": clocks.summary()}), flush=True)
 
 
+def bf16_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_BF16_TFLOPS, "fallback"
+
+
+def run_linear(args):
+    """Masked linear forward over the layer set: every tensor's Y = X Wm^T for
+    --tokens tokens with the mask formed in the GEMM's prologue
+    (roi_masked_linear_fwd), device-resident inputs, per-launch CUDA events.  Beside
+    it, the unfused pair the fusion replaces: roi_mask_fwd_ex writing Wm, then a
+    cuBLAS bf16 GEMM (torch.mm) reading it.  One GPU."""
+    import torch
+    if int(os.environ.get("RANK", "0")) != 0:
+        return
+    cfg = config_for(args)
+    N, M, tau, T = cfg["N"], cfg["M"], cfg["tau"], args.tokens
+    if not 1 <= T <= 256:
+        raise SystemExit("--tokens must be in 1..256")
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    from paper_2608_23048_gb300 import _build
+    _build.build()
+    import paper_2608_23048_gb300 as roi
+    kind = WL.CONFIGS[args.set].logits
+    tensors, ws_bytes = [], 16
+    for layer, p, rows, cols in selected_tensors(args):
+        seed = WL.tensor_seed(layer, p)
+        W, phi, _ = WL.make_inputs(rows, cols, kind, seed, device=dev)
+        t = {"id": layer * len(WL.PROJS) + p, "rows": rows, "cols": cols, "phi": phi, "W": W,
+             "X": WL.make_tokens(T, cols, seed, device=dev),
+             "Y": torch.empty(T, rows, dtype=torch.float32, device=dev)}
+        ws_bytes = max(ws_bytes, roi.roi_masked_linear_workspace_size(T, rows, cols))
+        tensors.append(t)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    Wm = torch.empty(max(t["rows"] * t["cols"] for t in tensors), dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def fused(s, ev):
+        for t in tensors:
+            st = roi.NoiseState(0, s, t["id"], 1.0, 0)
+            if ev is not None:
+                ev[0].append(torch.cuda.Event(enable_timing=True))
+                ev[0][-1].record(stream)
+            roi.roi_masked_linear_fwd(t["X"], t["phi"], t["W"], N, M, tau, st, t["Y"], ws, stream=stream)
+            if ev is not None:
+                ev[1].append(torch.cuda.Event(enable_timing=True))
+                ev[1][-1].record(stream)
+
+    def unfused(s, ev=None):
+        with torch.cuda.stream(stream):
+            for t in tensors:
+                st = roi.NoiseState(0, s, t["id"], 1.0, 0)
+                wm = Wm[:t["rows"] * t["cols"]].view(t["rows"], t["cols"])
+                if ev is not None:
+                    ev[0].append(torch.cuda.Event(enable_timing=True))
+                    ev[0][-1].record(stream)
+                roi.roi_mask_fwd_ex(t["phi"], t["W"], N, M, tau, st, wm, stream=stream)
+                torch.mm(t["X"], wm.t())
+                if ev is not None:
+                    ev[1].append(torch.cuda.Event(enable_timing=True))
+                    ev[1][-1].record(stream)
+
+    for w in range(args.warmup):
+        fused(w, None)
+    torch.cuda.synchronize()
+    roi.roi_device_status(stream)
+    ev = ([], [])
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(0) as clocks:
+        start.record(stream)
+        for s in range(args.steps):
+            fused(args.warmup + s, ev)
+        end.record(stream)
+        torch.cuda.synchronize()
+    roi.roi_device_status(stream)
+    elapsed = start.elapsed_time(end) / 1e3
+    k_t = sum(x.elapsed_time(y) for x, y in zip(ev[0], ev[1])) / 1e3
+    # the unfused pair, same inputs and steps
+    for w in range(args.warmup):
+        unfused(w)
+    u0, u1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    uev = ([], [])
+    u0.record(stream)
+    for s in range(args.steps):
+        unfused(args.warmup + s, uev)
+    u1.record(stream)
+    torch.cuda.synchronize()
+    unfused_t = u0.elapsed_time(u1) / 1e3
+    # per projection (summed over layers), per step: fused kernel vs the unfused pair
+    per_proj = {}
+    for i, (x, y) in enumerate(zip(ev[0], ev[1])):
+        name = WL.PROJS[tensors[i % len(tensors)]["id"] % len(WL.PROJS)]
+        per_proj.setdefault(name, [0.0, 0.0])[0] += x.elapsed_time(y) / args.steps
+    for i, (x, y) in enumerate(zip(uev[0], uev[1])):
+        name = WL.PROJS[tensors[i % len(tensors)]["id"] % len(WL.PROJS)]
+        per_proj.setdefault(name, [0.0, 0.0])[1] += x.elapsed_time(y) / args.steps
+    E = cfg["elements"]
+    bytes_step = sum(6 * t["rows"] * t["cols"] + 2 * T * t["cols"] + 4 * T * t["rows"] for t in tensors)
+    flops_step = sum(2 * T * t["rows"] * t["cols"] for t in tensors)
+    peak, peak_kind = hbm_peak()
+    tpeak, tpeak_kind = bf16_peak()
+    gbs = bytes_step * args.steps / k_t / 1e9
+    tflops = flops_step * args.steps / k_t / 1e12
+    bound = "hbm" if bytes_step / (peak * 1e9) >= flops_step / (tpeak * 1e12) else "tensor"
+    roofline = {"bound": bound, "achieved": round(gbs, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(gbs / peak, 4), "traffic": None,
+                "kernel": f"roi_masked_linear_kernel<{N},{M},{'tau1' if tau == 1.0 else 'tau'}>",
+                "peak_kind": peak_kind, "algorithmic_bytes_per_element": 6,
+                "algorithmic_bytes_per_step": bytes_step, "tensor_tflops": round(tflops, 1),
+                "tensor_peak_tflops": tpeak, "tensor_frac": round(tflops / tpeak, 4),
+                "tensor_peak_kind": tpeak_kind, "kernel_ms_per_step": round(1e3 * k_t / args.steps, 3),
+                "unfused_ms_per_step": round(1e3 * unfused_t / args.steps, 3),
+                "unfused": "roi_mask_fwd_ex (Wm written) + cuBLAS bf16 GEMM reading Wm (torch.mm)",
+                "per_projection_ms_fused_unfused": {k: [round(a, 3), round(b, 3)] for k, (a, b) in per_proj.items()}}
+    cfg = dict(cfg, op="linear", tokens=T, y_dtype="f32")
+    print(json.dumps({"metric": "masked linear forward (RoI mask in the GEMM prologue) groups/s and HBM GB/s, 1 GPU",
+                      "value": (E // M) * args.steps / elapsed, "unit": "groups/s",
+                      "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+                      "ms_per_step": 1e3 * elapsed / args.steps, "higher_is_better": True, "scaling": "weak",
+                      "vs_baseline": None, "dtype": "bf16 (products) / f32 (mask, accumulation)",
+                      "data": "synthetic", "config": cfg, "roofline": roofline, "clocks": clocks.summary()}),
+          flush=True)
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         run_reference(args)
+    elif args.op == "linear":
+        run_linear(args)
     elif args.op != "mask":
         run_variant(args)
     else:

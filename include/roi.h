@@ -41,6 +41,7 @@
 #ifndef ROI_H_
 #define ROI_H_
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -175,6 +176,30 @@ float roi_anneal(float init, float end, uint32_t t, uint32_t T_anneal);
  * cols % 4 == 0 and rows*cols % 32 == 0 (else ROI_ERR_SHAPE). */
 roi_status roi_export_compressed_2of4(const float* logits, const roi_bf16* W, int64_t rows, int64_t cols,
                                       roi_bf16* out_values, uint32_t* out_meta, void* stream);
+
+/* Masked linear forward: the layer's product with the masked weights (Eq. 5),
+ *     Y[t, r] = sum_c X[t, c] Wm[r, c],   Wm = bf16_rne(float(W) * S),
+ * where S is the relaxed mask of roi_mask_fwd_ex for the same (logits, W, N, M,
+ * tau, st), bit for bit, formed in the prologue of a tensor-core GEMM: Wm is
+ * never written to memory and the logits and W are read once.  The sum runs in
+ * float32 on the tensor cores (products of bf16 exact, accumulation order the
+ * hardware's), Y is float32.
+ *  X             [T, cols] bf16, the layer's input tokens; 1 <= T <= 256
+ *  out_Y         [T, rows] float32
+ *  workspace     nullable caller-owned device memory for split-K partials
+ *                (roi_masked_linear_workspace_size bytes; with less, or NULL,
+ *                K is split less or not at all: same result, fewer CTAs).  The
+ *                partials are added in a fixed order, so Y does not depend on
+ *                the run.  Must not overlap the other tensors.
+ * Supported (N, M): (2, 4), (4, 8), (2, 8) (else ROI_ERR_NM); cols % 8 == 0
+ * and T <= 256 (else ROI_ERR_SHAPE).  With T == 0 or rows == 0 nothing is
+ * read or written. */
+roi_status roi_masked_linear_fwd(const roi_bf16* X, const float* logits, const roi_bf16* W, int N, int M,
+                                 float tau, const roi_noise_state* st, int64_t T, int64_t rows, int64_t cols,
+                                 float* out_Y, void* workspace, size_t workspace_bytes, void* stream);
+/* Workspace bytes that let roi_masked_linear_fwd split K as far as it wants on
+ * the current device (0: no split; also 0 for shapes the call rejects). */
+size_t roi_masked_linear_workspace_size(int64_t T, int64_t rows, int64_t cols);
 
 /* Deployment mask (Sec. 4.2.3 anneals lambda towards 0; the limit of
  * Gumbel-top-N is the deterministic top-N of phi, which is also the most

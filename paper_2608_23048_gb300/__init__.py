@@ -68,6 +68,10 @@ def lib() -> ctypes.CDLL:
     L.roi_export_compressed_2of4.argtypes = [_P, _P, i64, i64, _P, _P, _P]
     L.roi_mask_bwd_adamw.argtypes = [_P, _P, ctypes.POINTER(NoiseState), i32, i32, _P, f32, i64, i64, _P, _P,
                                      ctypes.POINTER(AdamW), _P, _P, _P]
+    L.roi_masked_linear_fwd.argtypes = [_P, _P, _P, i32, i32, f32, ctypes.POINTER(NoiseState), i64, i64, i64, _P,
+                                        _P, ctypes.c_size_t, _P]
+    L.roi_masked_linear_workspace_size.argtypes = [i64, i64, i64]
+    L.roi_masked_linear_workspace_size.restype = ctypes.c_size_t
     L.roi_anneal.argtypes = [f32, f32, u32, u32]
     L.roi_anneal.restype = f32
     L.roi_hard_mask_export.argtypes = [_P, i32, i32, i64, i64, _P, _P, _P, _P]
@@ -80,7 +84,7 @@ def lib() -> ctypes.CDLL:
     L.roi_launch_count.restype = ctypes.c_uint64
     for name in ("roi_mask_fwd", "roi_mask_fwd_ex", "roi_mask_bwd", "roi_hard_mask_export", "roi_device_status",
                  "roi_noise_words", "roi_gumbel_noise", "roi_mask_fwd_st", "roi_mask_bwd_st",
-                 "roi_export_compressed_2of4", "roi_mask_bwd_adamw"):
+                 "roi_export_compressed_2of4", "roi_mask_bwd_adamw", "roi_masked_linear_fwd"):
         getattr(L, name).restype = i32
     _LIB = L
     return L
@@ -244,6 +248,30 @@ def roi_export_compressed_2of4(logits, W, out_values, out_meta, stream=None):
     s = lib().roi_export_compressed_2of4(_ptr(logits), _ptr(W), rows, cols, _ptr(out_values), _ptr(out_meta),
                                          _stream(stream))
     _raise(s, "roi_export_compressed_2of4")
+
+
+def roi_masked_linear_workspace_size(T, rows, cols) -> int:
+    """Bytes of workspace that let roi_masked_linear_fwd split K fully on the current device."""
+    return int(lib().roi_masked_linear_workspace_size(int(T), int(rows), int(cols)))
+
+
+def roi_masked_linear_fwd(X, logits, W, N, M, tau, state: NoiseState, out_Y, workspace=None, stream=None):
+    """Y[T, rows] = X[T, cols] @ bf16(W * S)^T with the mask formed inside the GEMM (float32 Y)."""
+    import torch
+    rows, cols = logits.shape
+    T = X.shape[0]
+    _check_tensor(logits, "logits", torch.float32)
+    _check_tensor(X, "X", torch.bfloat16, (T, cols))
+    _check_tensor(W, "W", torch.bfloat16, (rows, cols))
+    _check_tensor(out_Y, "out_Y", torch.float32, (T, rows))
+    ws_bytes = 0
+    if workspace is not None:
+        _check_tensor(workspace, "workspace", workspace.dtype)
+        ws_bytes = workspace.numel() * workspace.element_size()
+    st = state if isinstance(state, NoiseState) else NoiseState(*state)
+    s = lib().roi_masked_linear_fwd(_ptr(X), _ptr(logits), _ptr(W), int(N), int(M), float(tau), ctypes.byref(st), T,
+                                    rows, cols, _ptr(out_Y), _ptr(workspace), ws_bytes, _stream(stream))
+    _raise(s, "roi_masked_linear_fwd")
 
 
 def roi_hard_mask_export(logits, N, M, out_bits, W=None, out_Wpruned=None, stream=None):

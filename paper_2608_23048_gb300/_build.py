@@ -16,7 +16,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libroi.so")
-SOURCES = ["roi_api.cu", "roi_fwd.cu", "roi_bwd.cu", "roi_export.cu", "roi_noise.cu", "roi_slice.cu"]
+SOURCES = ["roi_api.cu", "roi_fwd.cu", "roi_bwd.cu", "roi_export.cu", "roi_noise.cu", "roi_slice.cu", "roi_linear.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "--expt-relaxed-constexpr", "-I", INCLUDE, "-I", CSRC]

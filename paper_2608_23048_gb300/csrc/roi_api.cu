@@ -304,6 +304,48 @@ roi_status roi_hard_mask_export(const float* logits, int N, int M, int64_t rows,
   return finish(launch_export(c));
 }
 
+size_t roi_masked_linear_workspace_size(int64_t T, int64_t rows, int64_t cols) {
+  if (T <= 0 || T > 256 || rows <= 0 || cols <= 0 || cols > INT64_MAX / 64 / rows) return 0;
+  return linear_workspace_bytes(T, rows, cols);
+}
+
+roi_status roi_masked_linear_fwd(const roi_bf16* X, const float* logits, const roi_bf16* W, int N, int M, float tau,
+                                 const roi_noise_state* st, int64_t T, int64_t rows, int64_t cols, float* out_Y,
+                                 void* workspace, size_t workspace_bytes, void* stream) {
+  if (st == nullptr) return ROI_ERR_NULL;
+  roi_status s = check_common(N, M, tau, rows, cols);
+  if (s != ROI_OK) return s;
+  if (!linear_supported(N, M)) return ROI_ERR_NM;
+  if (st->row_offset < 0 || T < 0 || T > 256 || cols % 8 != 0) return ROI_ERR_SHAPE;
+  if (!finite_positive(st->lambda)) return ROI_ERR_TAU;
+  if (rows == 0 || T == 0) return ROI_OK;  // nothing is read or written; pointers may be NULL
+  if (X == nullptr || logits == nullptr || W == nullptr || out_Y == nullptr) return ROI_ERR_NULL;
+  if (!aligned16(X) || !aligned16(logits) || !aligned16(W) || !aligned16(out_Y) || !aligned16(workspace))
+    return ROI_ERR_ALIGN;
+  const int64_t E = rows * cols;
+  const Range in[3] = {{X, uint64_t(T * cols) * 2}, {logits, uint64_t(E) * 4}, {W, uint64_t(E) * 2}};
+  const Range out[2] = {{out_Y, uint64_t(T * rows) * 4}, {workspace, workspace == nullptr ? 0 : uint64_t(workspace_bytes)}};
+  if (any_alias(in, out)) return ROI_ERR_ALIAS;
+  LinearCall c;
+  c.X = X;
+  c.phi = logits;
+  c.W = W;
+  c.Y = out_Y;
+  c.workspace = workspace;
+  c.workspace_bytes = workspace == nullptr ? 0 : workspace_bytes;
+  c.T = T;
+  c.rows = rows;
+  c.cols = cols;
+  c.N = N;
+  c.M = M;
+  c.tau = tau;
+  c.np = make_noise(*st, cols);
+  c.status = status_word();
+  if (c.status == nullptr) return ROI_ERR_CUDA;
+  c.stream = static_cast<cudaStream_t>(stream);
+  return finish(launch_masked_linear(c));
+}
+
 static roi_status noise_call(const roi_noise_state* st, int64_t rows, int64_t cols, uint32_t* words, float* g,
                              void* stream) {
   if (st == nullptr) return ROI_ERR_NULL;

@@ -61,6 +61,21 @@ struct CompressCall {
   cudaStream_t stream;
 };
 
+struct LinearCall {
+  const uint16_t* X;    // [T, cols] bf16
+  const float* phi;     // [rows, cols]
+  const uint16_t* W;    // [rows, cols] bf16
+  float* Y;             // [T, rows]
+  void* workspace;      // nullable: split-K partials and tickets
+  size_t workspace_bytes;
+  int64_t T, rows, cols;
+  int N, M;
+  float tau;
+  NoiseParams np;
+  unsigned int* status;
+  cudaStream_t stream;
+};
+
 // Each returns the number of kernels launched (>= 0) or -1 after a CUDA error.
 int launch_fwd(const FwdCall& c);
 int launch_bwd(const BwdCall& c);
@@ -71,6 +86,12 @@ bool slice_supported(int N, int M);
 int launch_slice_fwd(const FwdCall& c);
 int launch_slice_bwd(const BwdCall& c);
 int launch_noise(const NoiseParams& np, int64_t E, uint32_t* words, float* g, cudaStream_t stream);
+
+// Masked linear forward on the tensor cores (roi_linear.cu).
+bool linear_supported(int N, int M);
+int linear_splits(int64_t T, int64_t rows, int64_t cols);
+size_t linear_workspace_bytes(int64_t T, int64_t rows, int64_t cols);
+int launch_masked_linear(const LinearCall& c);
 
 // Streaming multiprocessors of the current device (cached).
 int sm_count();

@@ -111,6 +111,20 @@ def test_validation_codes(L):
     assert bwd_opt(opt, v=D + 8) == 5
     assert L.roi_mask_bwd_adamw(None, None, ctypes.byref(st), 2, 4, None, 1.0, 0, 8, None, None,
                                 ctypes.byref(opt), None, None, None) == 0
+    # masked linear: (2,4), (4,8), (2,8); T <= 256; cols % 8 == 0; Y and workspace are outputs
+    def lin(N=2, M=4, T=4, rows=128, cols=64, X=D, logits=A, W=B, Y=C, ws=None, wsb=0, tau=1.0, state=st):
+        return L.roi_masked_linear_fwd(_fake(X) if X else None, _fake(logits) if logits else None,
+                                       _fake(W) if W else None, N, M, tau, ctypes.byref(state) if state else None,
+                                       T, rows, cols, _fake(Y) if Y else None, _fake(ws) if ws else None, wsb, None)
+    assert lin(state=None) == 1 and lin(X=0) == 1 and lin(Y=0) == 1
+    assert lin(N=1) == 3 and lin(N=3, M=8) == 3 and lin(N=8, M=16, cols=64) == 3
+    assert lin(T=257) == 2 and lin(T=-1) == 2 and lin(cols=12) == 2
+    assert lin(tau=0.0) == 4
+    assert lin(X=D + 8) == 5 and lin(ws=E + 4, wsb=64) == 5
+    assert lin(Y=A + 64) == 6                       # Y overlaps the logits
+    assert lin(ws=C + 256, wsb=4096) == 6           # workspace overlaps Y
+    assert lin(T=0, X=0, logits=0, W=0, Y=0) == 0 and lin(rows=0, X=0, logits=0, W=0, Y=0) == 0
+    assert L.roi_masked_linear_workspace_size(0, 128, 64) == 0 and L.roi_masked_linear_workspace_size(300, 128, 64) == 0
     for s in range(10):
         assert L.roi_status_string(s)
 
