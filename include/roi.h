@@ -201,6 +201,25 @@ roi_status roi_masked_linear_fwd(const roi_bf16* X, const float* logits, const r
  * the current device (0: no split; also 0 for shapes the call rejects). */
 size_t roi_masked_linear_workspace_size(int64_t T, int64_t rows, int64_t cols);
 
+/* roi_masked_linear_fwd without a caller workspace.  The paper has no
+ * counterpart: this is the library's own convenience for callers that have no
+ * device allocator at hand.  The split-K partials go to one static device array
+ * of ROI_LINEAR_SCRATCH_BYTES (16 MiB) per device instead, so the call allocates
+ * nothing; arguments, results and errors are those of roi_masked_linear_fwd with
+ * a workspace of roi_masked_linear_workspace_size bytes, except:
+ *  - a call that needs more scratch than ROI_LINEAR_SCRATCH_BYTES returns
+ *    ROI_ERR_SHAPE (e.g. a 3584 x 18944 layer at 256 tokens needs 18.4 MB on a
+ *    152-SM GPU; pass a workspace to roi_masked_linear_fwd for those);
+ *  - the array is shared by every call on the device and keeps the last call's
+ *    partials; calls that overlap in time (other streams, other threads) race on
+ *    it and must be serialised by the caller;
+ *  - the first call on a device looks the array up (cudaGetSymbolAddress); when
+ *    calls are to be recorded by stream capture, make one call before it. */
+#define ROI_LINEAR_SCRATCH_BYTES (16u << 20)
+roi_status roi_masked_linear_fwd_noalloc(const roi_bf16* X, const float* logits, const roi_bf16* W, int N, int M,
+                                         float tau, const roi_noise_state* st, int64_t T, int64_t rows, int64_t cols,
+                                         float* out_Y, void* stream);
+
 /* Deployment mask (Sec. 4.2.3 anneals lambda towards 0; the limit of
  * Gumbel-top-N is the deterministic top-N of phi, which is also the most
  * probable subset of Eq. 8): argtop_N(phi) per group, NaN ranked as -inf,

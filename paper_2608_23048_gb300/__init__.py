@@ -70,6 +70,8 @@ def lib() -> ctypes.CDLL:
                                      ctypes.POINTER(AdamW), _P, _P, _P]
     L.roi_masked_linear_fwd.argtypes = [_P, _P, _P, i32, i32, f32, ctypes.POINTER(NoiseState), i64, i64, i64, _P,
                                         _P, ctypes.c_size_t, _P]
+    L.roi_masked_linear_fwd_noalloc.argtypes = [_P, _P, _P, i32, i32, f32, ctypes.POINTER(NoiseState), i64, i64,
+                                                i64, _P, _P]
     L.roi_masked_linear_workspace_size.argtypes = [i64, i64, i64]
     L.roi_masked_linear_workspace_size.restype = ctypes.c_size_t
     L.roi_anneal.argtypes = [f32, f32, u32, u32]
@@ -84,7 +86,8 @@ def lib() -> ctypes.CDLL:
     L.roi_launch_count.restype = ctypes.c_uint64
     for name in ("roi_mask_fwd", "roi_mask_fwd_ex", "roi_mask_bwd", "roi_hard_mask_export", "roi_device_status",
                  "roi_noise_words", "roi_gumbel_noise", "roi_mask_fwd_st", "roi_mask_bwd_st",
-                 "roi_export_compressed_2of4", "roi_mask_bwd_adamw", "roi_masked_linear_fwd"):
+                 "roi_export_compressed_2of4", "roi_mask_bwd_adamw", "roi_masked_linear_fwd",
+                 "roi_masked_linear_fwd_noalloc"):
         getattr(L, name).restype = i32
     _LIB = L
     return L
@@ -272,6 +275,21 @@ def roi_masked_linear_fwd(X, logits, W, N, M, tau, state: NoiseState, out_Y, wor
     s = lib().roi_masked_linear_fwd(_ptr(X), _ptr(logits), _ptr(W), int(N), int(M), float(tau), ctypes.byref(st), T,
                                     rows, cols, _ptr(out_Y), _ptr(workspace), ws_bytes, _stream(stream))
     _raise(s, "roi_masked_linear_fwd")
+
+
+def roi_masked_linear_fwd_noalloc(X, logits, W, N, M, tau, state: NoiseState, out_Y, stream=None):
+    """roi_masked_linear_fwd with the library's static split-K scratch (no workspace argument)."""
+    import torch
+    rows, cols = logits.shape
+    T = X.shape[0]
+    _check_tensor(logits, "logits", torch.float32)
+    _check_tensor(X, "X", torch.bfloat16, (T, cols))
+    _check_tensor(W, "W", torch.bfloat16, (rows, cols))
+    _check_tensor(out_Y, "out_Y", torch.float32, (T, rows))
+    st = state if isinstance(state, NoiseState) else NoiseState(*state)
+    s = lib().roi_masked_linear_fwd_noalloc(_ptr(X), _ptr(logits), _ptr(W), int(N), int(M), float(tau),
+                                            ctypes.byref(st), T, rows, cols, _ptr(out_Y), _stream(stream))
+    _raise(s, "roi_masked_linear_fwd_noalloc")
 
 
 def roi_hard_mask_export(logits, N, M, out_bits, W=None, out_Wpruned=None, stream=None):

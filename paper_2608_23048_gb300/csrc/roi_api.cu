@@ -309,6 +309,36 @@ size_t roi_masked_linear_workspace_size(int64_t T, int64_t rows, int64_t cols) {
   return linear_workspace_bytes(T, rows, cols);
 }
 
+}  // extern "C"
+
+namespace roi {
+namespace {
+
+// Split-K scratch of roi_masked_linear_fwd_noalloc: one static array per device,
+// ROI_LINEAR_SCRATCH_BYTES long.
+static __device__ __align__(256) unsigned char g_linear_scratch[ROI_LINEAR_SCRATCH_BYTES];
+
+// The array's device address on the current device, looked up once per device
+// (nullptr if the lookup fails or the address is not 256-byte aligned).
+void* linear_scratch() {
+  static std::atomic<void*> cache[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  void* p = cache[dev].load(std::memory_order_acquire);
+  if (p == nullptr) {
+    if (cudaGetSymbolAddress(&p, g_linear_scratch) != cudaSuccess || p == nullptr ||
+        (reinterpret_cast<uintptr_t>(p) & 255u) != 0)
+      return nullptr;
+    cache[dev].store(p, std::memory_order_release);
+  }
+  return p;
+}
+
+}  // namespace
+}  // namespace roi
+
+extern "C" {
+
 roi_status roi_masked_linear_fwd(const roi_bf16* X, const float* logits, const roi_bf16* W, int N, int M, float tau,
                                  const roi_noise_state* st, int64_t T, int64_t rows, int64_t cols, float* out_Y,
                                  void* workspace, size_t workspace_bytes, void* stream) {
@@ -344,6 +374,19 @@ roi_status roi_masked_linear_fwd(const roi_bf16* X, const float* logits, const r
   if (c.status == nullptr) return ROI_ERR_CUDA;
   c.stream = static_cast<cudaStream_t>(stream);
   return finish(launch_masked_linear(c));
+}
+
+roi_status roi_masked_linear_fwd_noalloc(const roi_bf16* X, const float* logits, const roi_bf16* W, int N, int M,
+                                         float tau, const roi_noise_state* st, int64_t T, int64_t rows, int64_t cols,
+                                         float* out_Y, void* stream) {
+  const size_t need = roi_masked_linear_workspace_size(T, rows, cols);
+  if (need > size_t(ROI_LINEAR_SCRATCH_BYTES)) return ROI_ERR_SHAPE;
+  void* ws = nullptr;
+  if (need > 0) {
+    ws = linear_scratch();
+    if (ws == nullptr) return ROI_ERR_CUDA;
+  }
+  return roi_masked_linear_fwd(X, logits, W, N, M, tau, st, T, rows, cols, out_Y, ws, need, stream);
 }
 
 static roi_status noise_call(const roi_noise_state* st, int64_t rows, int64_t cols, uint32_t* words, float* g,

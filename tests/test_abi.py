@@ -124,6 +124,11 @@ def test_validation_codes(L):
     assert lin(Y=A + 64) == 6                       # Y overlaps the logits
     assert lin(ws=C + 256, wsb=4096) == 6           # workspace overlaps Y
     assert lin(T=0, X=0, logits=0, W=0, Y=0) == 0 and lin(rows=0, X=0, logits=0, W=0, Y=0) == 0
+    # the no-workspace variant validates as the workspace call (invalid arguments only: nothing may launch)
+    assert L.roi_masked_linear_fwd_noalloc(None, _fake(A), _fake(B), 2, 4, 1.0, ctypes.byref(st), 4, 128, 64,
+                                           _fake(C), None) == 1
+    assert L.roi_masked_linear_fwd_noalloc(_fake(D), _fake(A), _fake(B), 2, 4, 1.0, ctypes.byref(st), 257, 128, 64,
+                                           _fake(C), None) == 2
     assert L.roi_masked_linear_workspace_size(0, 128, 64) == 0 and L.roi_masked_linear_workspace_size(300, 128, 64) == 0
     for s in range(10):
         assert L.roi_status_string(s)
