@@ -96,24 +96,28 @@ __device__ __forceinline__ float lane_of(V v, int h) {
 
 // L groups (one per lane of V) processed in lockstep by one thread; writes their
 // outputs and returns each group's hard bits in bits[h].
+// The keys of L groups from their staged logits (first half of fwd_groups).
+template <int M, class V>
+__device__ __forceinline__ void fwd_keys(const float* const* phi_g, const int64_t* e0, const FwdArgs& a,
+                                         V (&kap)[M]) {
+  constexpr int L = vlanes<V>();
+  float ph[L][M];
+#pragma unroll
+  for (int h = 0; h < L; ++h) {
+#pragma unroll
+    for (int s = 0; s < M / 4; ++s) {
+      const float4 p = reinterpret_cast<const float4*>(phi_g[h])[s];
+      ph[h][4 * s] = p.x, ph[h][4 * s + 1] = p.y, ph[h][4 * s + 2] = p.z, ph[h][4 * s + 3] = p.w;
+    }
+  }
+  group_keys<M, V>(ph, e0, a.np, kap);
+}
+
+// Relaxation, hard bits and outputs of L groups whose keys are `kap`.
 template <int N, int M, bool TAU1, class V, bool ST = false>
-__device__ __forceinline__ void fwd_groups(const float* const* phi_g, const uint16_t* const* W_g, const int64_t* e0,
+__device__ __forceinline__ void fwd_finish(const V (&kap)[M], const uint16_t* const* W_g, const int64_t* e0,
                                            const FwdArgs& a, uint32_t* bits) {
   constexpr int L = vlanes<V>();
-  V kap[M];
-  {
-    float ph[L][M];
-#pragma unroll
-    for (int h = 0; h < L; ++h) {
-#pragma unroll
-      for (int s = 0; s < M / 4; ++s) {
-        const float4 p = reinterpret_cast<const float4*>(phi_g[h])[s];
-        ph[h][4 * s] = p.x, ph[h][4 * s + 1] = p.y, ph[h][4 * s + 2] = p.z, ph[h][4 * s + 3] = p.w;
-      }
-    }
-    group_keys<M, V>(ph, e0, a.np, kap);
-  }
-
   FastGroup<N, M, TAU1, false, V> fg;
   fg.forward(kap, a.inv_tau);
   float S[L][M];
@@ -219,6 +223,14 @@ __device__ __forceinline__ void fwd_groups(const float* const* phi_g, const uint
   }
 }
 
+template <int N, int M, bool TAU1, class V, bool ST = false>
+__device__ __forceinline__ void fwd_groups(const float* const* phi_g, const uint16_t* const* W_g, const int64_t* e0,
+                                           const FwdArgs& a, uint32_t* bits) {
+  V kap[M];
+  fwd_keys<M, V>(phi_g, e0, a, kap);
+  fwd_finish<N, M, TAU1, V, ST>(kap, W_g, e0, a, bits);
+}
+
 // Combine the M-bit masks of 32 / M consecutive lanes into words and store.
 template <int M>
 __device__ __forceinline__ void store_hard(uint32_t* hard, int64_t e0, uint32_t bits, bool active) {
@@ -270,15 +282,30 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_fwd_
         const float* sphi = reinterpret_cast<const float*>(stage[0]);
         const uint16_t* sW = reinterpret_cast<const uint16_t*>(stage[1]);
         const int64_t base = tile * kT;
+        // pair p: groups t and t + kThreads of the p-th block of 2 kThreads groups.
+        // The keys of pair p + 1 (integer-heavy: Philox, range reduction) are
+        // formed before pair p is relaxed (floating-point-heavy), so the two
+        // streams share the issue slots of one basic block.
+        F2 kap[2][M];
+        {
+          const int g0 = threadIdx.x, g1 = g0 + C::kThreads;
+          const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
+          const int64_t e0[2] = {base + g0 * M, base + g1 * M};
+          fwd_keys<M, F2>(pp, e0, a, kap[0]);
+        }
 #pragma unroll
         for (int p = 0; p < C::kPairs; ++p) {
-          // pair p: groups t and t + kThreads of the p-th block of 2 kThreads groups
+          if (p + 1 < C::kPairs) {
+            const int g0 = threadIdx.x + 2 * (p + 1) * C::kThreads, g1 = g0 + C::kThreads;
+            const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
+            const int64_t e0[2] = {base + g0 * M, base + g1 * M};
+            fwd_keys<M, F2>(pp, e0, a, kap[(p + 1) & 1]);
+          }
           const int g0 = threadIdx.x + 2 * p * C::kThreads, g1 = g0 + C::kThreads;
-          const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
           const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
           const int64_t e0[2] = {base + g0 * M, base + g1 * M};
           uint32_t bits[2];
-          fwd_groups<N, M, TAU1, F2, ST>(pp, pw, e0, a, bits);
+          fwd_finish<N, M, TAU1, F2, ST>(kap[p & 1], pw, e0, a, bits);
           if (a.hard != nullptr) store_hard_pair<M>(a.hard, e0[0], e0[1], bits[0], bits[1]);
         }
       });
