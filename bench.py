@@ -740,9 +740,12 @@ def run_linear(args):
     gbs = bytes_step * args.steps / k_t / 1e9
     tflops = flops_step * args.steps / k_t / 1e12
     bound = "hbm" if bytes_step / (peak * 1e9) >= flops_step / (tpeak * 1e12) else "tensor"
+    tag = f"roi_masked_linear_kernel<{N},{M},{'tau1' if tau == 1.0 else 'tau'}>"
+    traffic = recorded_traffic(tag)  # DRAM bytes per weight element (one 256-token capture)
     roofline = {"bound": bound, "achieved": round(gbs, 1), "peak": peak, "unit": "GB/s",
-                "frac": round(gbs / peak, 4), "traffic": None,
-                "kernel": f"roi_masked_linear_kernel<{N},{M},{'tau1' if tau == 1.0 else 'tau'}>",
+                "frac": round(gbs / peak, 4),
+                "traffic": (None if traffic is None or T != 256 else traffic * E / len(tensors)),
+                "kernel": tag,
                 "peak_kind": peak_kind, "algorithmic_bytes_per_element": 6,
                 "algorithmic_bytes_per_step": bytes_step, "tensor_tflops": round(tflops, 1),
                 "tensor_peak_tflops": tpeak, "tensor_frac": round(tflops / tpeak, 4),
