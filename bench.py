@@ -59,6 +59,9 @@ def parse_args():
                         "export2of4: the compressed 2:4 export; linear: the masked linear forward "
                         "(mask formed in a tensor-core GEMM's prologue) over --tokens tokens (one GPU)")
     p.add_argument("--tokens", type=int, default=256, help="tokens per layer for --op linear (1..256)")
+    p.add_argument("--per-tensor", action="store_true",
+                   help="one roi_mask_fwd_ex / roi_mask_bwd call per tensor instead of one batched call per "
+                        "direction (adds the per-projection breakdown)")
     return p.parse_args()
 
 
@@ -93,6 +96,8 @@ def config_for(args):
         "layer_set": args.set, "N": N, "M": M, "tau": tau, "lambda": 1.0,
         "elements": E, "groups": E // M, "tensors": len(sel),
         "l2": "inputs larger than L2: every step streams the whole set (>90 GB for the 7B set)",
+        "calls": ("one roi_mask_fwd_ex + one roi_mask_bwd per tensor" if getattr(args, "per_tensor", False) else
+                  "one roi_mask_fwd_batch + one roi_mask_bwd_batch per step (all tensors)"),
     }
 
 
@@ -333,26 +338,39 @@ def run_ours(args):
     stream = torch.cuda.Stream(device=dev)
     states = {t["id"]: roi.NoiseState(0, 0, t["id"], 1.0, 0) for t in tensors}
 
+    # batched (default): every tensor's forward in one call, every backward in one
+    fwd_items = roi.make_fwd_items([(t["phi"], t["W"], states[t["id"]], t["Wm"], None, t["hard"]) for t in tensors])
+    bwd_items = roi.make_bwd_items([(t["phi"], t["W"], states[t["id"]], t["dWm"], t["dphi"], None)
+                                    for t in reversed(tensors)])
+
+    def mark(lst, ev):
+        if ev is not None:
+            lst.append(torch.cuda.Event(enable_timing=True))
+            lst[-1].record(stream)
+
     def step(s, ev=None):
+        if not args.per_tensor:
+            for arr in (fwd_items, bwd_items):
+                for k in range(len(arr)):
+                    arr[k].st.step = s
+            mark(ev[0] if ev else None, ev)
+            roi.roi_mask_fwd_batch(fwd_items, N, M, tau, stream=stream)
+            mark(ev[1] if ev else None, ev)
+            mark(ev[2] if ev else None, ev)
+            roi.roi_mask_bwd_batch(bwd_items, N, M, tau, stream=stream)
+            mark(ev[3] if ev else None, ev)
+            return
         for t in tensors:
             st = states[t["id"]]
             st.step = s
-            if ev is not None:
-                ev[0].append(torch.cuda.Event(enable_timing=True))
-                ev[0][-1].record(stream)
+            mark(ev[0] if ev else None, ev)
             roi.roi_mask_fwd_ex(t["phi"], t["W"], N, M, tau, st, t["Wm"], None, t["hard"], stream=stream)
-            if ev is not None:
-                ev[1].append(torch.cuda.Event(enable_timing=True))
-                ev[1][-1].record(stream)
+            mark(ev[1] if ev else None, ev)
         for t in reversed(tensors):
             st = states[t["id"]]
-            if ev is not None:
-                ev[2].append(torch.cuda.Event(enable_timing=True))
-                ev[2][-1].record(stream)
+            mark(ev[2] if ev else None, ev)
             roi.roi_mask_bwd(t["phi"], t["W"], st, N, M, t["dWm"], tau, t["dphi"], None, stream=stream)
-            if ev is not None:
-                ev[3].append(torch.cuda.Event(enable_timing=True))
-                ev[3][-1].record(stream)
+            mark(ev[3] if ev else None, ev)
 
     with torch.cuda.stream(stream):
         for w in range(args.warmup):
@@ -380,6 +398,18 @@ def run_ours(args):
     elapsed = start.elapsed_time(end) / 1e3
     fwd_t = sum(a.elapsed_time(b) for a, b in zip(ev[0], ev[1])) / 1e3
     bwd_t = sum(a.elapsed_time(b) for a, b in zip(ev[2], ev[3])) / 1e3
+    # per projection, summed over layers, per step: fwd ms, bwd ms, fraction of the roofline
+    # (per-tensor calls only)
+    per_proj = {}
+    nt = len(tensors) if args.per_tensor else 10 ** 9
+    for i, (a, b) in enumerate(zip(ev[0], ev[1]) if args.per_tensor else ()):
+        t = tensors[i % nt]
+        per_proj.setdefault(WL.PROJS[t["id"] % len(WL.PROJS)], [0.0, 0.0, 0])[0] += a.elapsed_time(b) / args.steps
+    for i, (a, b) in enumerate(zip(ev[2], ev[3]) if args.per_tensor else ()):
+        t = tensors[nt - 1 - i % nt]
+        per_proj[WL.PROJS[t["id"] % len(WL.PROJS)]][1] += a.elapsed_time(b) / args.steps
+    for t in tensors if args.per_tensor else ():
+        per_proj[WL.PROJS[t["id"] % len(WL.PROJS)]][2] += t["rows"] * t["cols"]
     if world > 1:
         tt = torch.tensor([elapsed], device=dev)
         dist.all_reduce(tt, op=dist.ReduceOp.MAX)
@@ -397,20 +427,27 @@ def run_ours(args):
     traffic = recorded_traffic(tag)
     per_elem = BWD_BYTES if dom == "bwd" else FWD_BYTES
     achieved = bwd_gbs if dom == "bwd" else fwd_gbs
-    launches_per_kernel = len(tensors)
+    launches_per_kernel = len(tensors) if args.per_tensor else -(-len(tensors) // 256)
+    pk = hbm_peak()[0]
+    per_projection = {k: {"fwd_ms": round(f, 3), "bwd_ms": round(b, 3),
+                          "frac": round(n * (FWD_BYTES + BWD_BYTES) / ((f + b) * 1e-3) / 1e9 / pk, 3)}
+                      for k, (f, b, n) in per_proj.items()}
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(achieved / peak, 4),
                 "traffic": (None if traffic is None else traffic * E / launches_per_kernel),
                 "kernel": tag, "peak_kind": peak_kind,
                 "algorithmic_bytes_per_element": per_elem,
-                "units_per_launch": f"{E / launches_per_kernel:.0f} elements (mean over the {launches_per_kernel} tensors)",
+                "units_per_launch": (f"{E / launches_per_kernel:.0f} elements (mean over the {launches_per_kernel} tensors)"
+                                     if args.per_tensor else
+                                     f"{E / launches_per_kernel:.0f} elements (all {len(tensors)} tensors of a step "
+                                     f"in {launches_per_kernel} batched launch per direction)"),
                 "fwd_gbs": round(fwd_gbs, 1), "bwd_gbs": round(bwd_gbs, 1),
                 "fwd_ms_per_step": round(1e3 * fwd_t / args.steps, 3),
                 "bwd_ms_per_step": round(1e3 * bwd_t / args.steps, 3),
-                "step_gbs": round(step_gbs / world, 1), "step_frac": round(step_gbs / world / peak, 4)}
+                "step_gbs": round(step_gbs / world, 1), "step_frac": round(step_gbs / world / peak, 4), "per_projection": per_projection}
 
     # per-step device time: first forward launch to last backward launch of each step
-    T = len(tensors)
+    T = len(ev[0]) // args.steps  # events per step and direction: one per call
     step_ms = sorted(ev[0][s * T].elapsed_time(ev[3][s * T + T - 1]) for s in range(args.steps))
     pct = lambda q: round(step_ms[min(len(step_ms) - 1, int(q * (len(step_ms) - 1) + 0.5))], 3)
     step_stats = {"p10": pct(0.1), "median": pct(0.5), "p90": pct(0.9)}

@@ -95,6 +95,37 @@ roi_status roi_mask_fwd_ex(const float* logits, const roi_bf16* W, int N, int M,
                            const roi_noise_state* st, int64_t rows, int64_t cols,
                            roi_bf16* out_Wm, float* out_soft, uint32_t* out_hard, void* stream);
 
+/* Many tensors in one call: the same results, bit for bit, as roi_mask_fwd_ex /
+ * roi_mask_bwd for each item in turn, with one (N, M, tau) and one stream for all.
+ * Each item is validated as the single call would be; in addition no output may
+ * overlap any input or output of any item (ROI_ERR_ALIAS), so the items are
+ * independent.  That lets the library chain their launches with programmatic
+ * dependent launch (for (N, M) = (2, 4), (4, 8), (2, 8)): a tensor's kernel may start
+ * on the SMs that the previous one frees as it drains, hiding the launch gap and
+ * the ragged last wave of small tensors, while each launch still completes after
+ * its predecessor, so the work queued after the call sees every item done.  Items
+ * with rows == 0 are skipped.  `items` is host memory, read during the call. */
+typedef struct {
+    const float* logits;  /* [rows, cols] */
+    const roi_bf16* W;    /* [rows, cols] */
+    roi_bf16* out_Wm;     /* [rows, cols] */
+    float* out_soft;      /* nullable, [rows, cols] */
+    uint32_t* out_hard;   /* nullable, [ceil(rows*cols/32)] */
+    int64_t rows, cols;
+    roi_noise_state st;
+} roi_fwd_item;
+typedef struct {
+    const float* logits;  /* [rows, cols] */
+    const roi_bf16* W;    /* [rows, cols] */
+    const roi_bf16* dWm;  /* [rows, cols] */
+    float* out_dlogits;   /* [rows, cols], overwritten */
+    roi_bf16* out_dW;     /* nullable, [rows, cols] */
+    int64_t rows, cols;
+    roi_noise_state st;
+} roi_bwd_item;
+roi_status roi_mask_fwd_batch(const roi_fwd_item* items, int count, int N, int M, float tau, void* stream);
+roi_status roi_mask_bwd_batch(const roi_bwd_item* items, int count, int N, int M, float tau, void* stream);
+
 /* Backward of the mask op: turns the upstream gradient of the masked weights
  * into logit gradients through the relaxation (Sec. 3.2: the map from logits
  * to the soft N-hot vector is differentiable).  The noise is regenerated from

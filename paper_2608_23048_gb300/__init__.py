@@ -46,6 +46,20 @@ class AdamW(ctypes.Structure):
                 ("eps", ctypes.c_float), ("weight_decay", ctypes.c_float), ("t", ctypes.c_uint32)]
 
 
+class FwdItem(ctypes.Structure):
+    """roi_fwd_item: one tensor of roi_mask_fwd_batch."""
+    _fields_ = [("logits", ctypes.c_void_p), ("W", ctypes.c_void_p), ("out_Wm", ctypes.c_void_p),
+                ("out_soft", ctypes.c_void_p), ("out_hard", ctypes.c_void_p), ("rows", ctypes.c_int64),
+                ("cols", ctypes.c_int64), ("st", NoiseState)]
+
+
+class BwdItem(ctypes.Structure):
+    """roi_bwd_item: one tensor of roi_mask_bwd_batch."""
+    _fields_ = [("logits", ctypes.c_void_p), ("W", ctypes.c_void_p), ("dWm", ctypes.c_void_p),
+                ("out_dlogits", ctypes.c_void_p), ("out_dW", ctypes.c_void_p), ("rows", ctypes.c_int64),
+                ("cols", ctypes.c_int64), ("st", NoiseState)]
+
+
 _LIB = None
 _P = ctypes.c_void_p
 
@@ -74,6 +88,8 @@ def lib() -> ctypes.CDLL:
                                                 i64, _P, _P]
     L.roi_masked_linear_workspace_size.argtypes = [i64, i64, i64]
     L.roi_masked_linear_workspace_size.restype = ctypes.c_size_t
+    L.roi_mask_fwd_batch.argtypes = [ctypes.POINTER(FwdItem), i32, i32, i32, f32, _P]
+    L.roi_mask_bwd_batch.argtypes = [ctypes.POINTER(BwdItem), i32, i32, i32, f32, _P]
     L.roi_anneal.argtypes = [f32, f32, u32, u32]
     L.roi_anneal.restype = f32
     L.roi_hard_mask_export.argtypes = [_P, i32, i32, i64, i64, _P, _P, _P, _P]
@@ -87,7 +103,7 @@ def lib() -> ctypes.CDLL:
     for name in ("roi_mask_fwd", "roi_mask_fwd_ex", "roi_mask_bwd", "roi_hard_mask_export", "roi_device_status",
                  "roi_noise_words", "roi_gumbel_noise", "roi_mask_fwd_st", "roi_mask_bwd_st",
                  "roi_export_compressed_2of4", "roi_mask_bwd_adamw", "roi_masked_linear_fwd",
-                 "roi_masked_linear_fwd_noalloc"):
+                 "roi_masked_linear_fwd_noalloc", "roi_mask_fwd_batch", "roi_mask_bwd_batch"):
         getattr(L, name).restype = i32
     _LIB = L
     return L
@@ -153,6 +169,59 @@ def roi_mask_fwd_ex(logits, W, N, M, tau, state: NoiseState, out_Wm, out_soft=No
     s = lib().roi_mask_fwd_ex(_ptr(logits), _ptr(W), int(N), int(M), float(tau), ctypes.byref(st), rows, cols,
                               _ptr(out_Wm), _ptr(out_soft), _ptr(out_hard), _stream(stream))
     _raise(s, "roi_mask_fwd_ex")
+
+
+def _addr(t):
+    return None if t is None else t.data_ptr()
+
+
+def make_fwd_items(items):
+    """ctypes array of FwdItem from (logits, W, state, out_Wm, out_soft, out_hard) tuples."""
+    import torch
+    arr = (FwdItem * len(items))()
+    for k, (logits, W, state, out_Wm, out_soft, out_hard) in enumerate(items):
+        rows, cols = logits.shape
+        _check_tensor(logits, "logits", torch.float32)
+        _check_tensor(W, "W", torch.bfloat16, (rows, cols))
+        _check_tensor(out_Wm, "out_Wm", torch.bfloat16, (rows, cols))
+        _check_tensor(out_soft, "out_soft", torch.float32, (rows, cols))
+        _check_tensor(out_hard, "out_hard", torch.int32, (hard_words(rows, cols),))
+        st = state if isinstance(state, NoiseState) else NoiseState(*state)
+        arr[k] = FwdItem(_addr(logits), _addr(W), _addr(out_Wm), _addr(out_soft), _addr(out_hard), rows, cols, st)
+    return arr
+
+
+def make_bwd_items(items):
+    """ctypes array of BwdItem from (logits, W, state, dWm, out_dlogits, out_dW) tuples."""
+    import torch
+    arr = (BwdItem * len(items))()
+    for k, (logits, W, state, dWm, out_dlogits, out_dW) in enumerate(items):
+        rows, cols = logits.shape
+        _check_tensor(logits, "logits", torch.float32)
+        _check_tensor(W, "W", torch.bfloat16, (rows, cols))
+        _check_tensor(dWm, "dWm", torch.bfloat16, (rows, cols))
+        _check_tensor(out_dlogits, "out_dlogits", torch.float32, (rows, cols))
+        _check_tensor(out_dW, "out_dW", torch.bfloat16, (rows, cols))
+        st = state if isinstance(state, NoiseState) else NoiseState(*state)
+        arr[k] = BwdItem(_addr(logits), _addr(W), _addr(dWm), _addr(out_dlogits), _addr(out_dW), rows, cols, st)
+    return arr
+
+
+def roi_mask_fwd_batch(items, N, M, tau, stream=None):
+    """Forward of many tensors in one call.  `items`: a FwdItem array from make_fwd_items
+    (reusable across calls while its tensors live; update .st.step per step) or a list
+    of (logits, W, state, out_Wm, out_soft, out_hard) tuples."""
+    arr = items if isinstance(items, ctypes.Array) else make_fwd_items(items)
+    s = lib().roi_mask_fwd_batch(arr, len(arr), int(N), int(M), float(tau), _stream(stream))
+    _raise(s, "roi_mask_fwd_batch")
+
+
+def roi_mask_bwd_batch(items, N, M, tau, stream=None):
+    """Backward of many tensors in one call (BwdItem array from make_bwd_items, or a list
+    of (logits, W, state, dWm, out_dlogits, out_dW) tuples)."""
+    arr = items if isinstance(items, ctypes.Array) else make_bwd_items(items)
+    s = lib().roi_mask_bwd_batch(arr, len(arr), int(N), int(M), float(tau), _stream(stream))
+    _raise(s, "roi_mask_bwd_batch")
 
 
 def roi_mask_fwd(logits, W, N, M, tau, seed, step, out_Wm, out_soft=None, out_hard=None, stream=None):

@@ -1,6 +1,8 @@
 // C ABI of libroi (see include/roi.h): host-side validation, then one launch.
+#include <algorithm>
 #include <atomic>
 #include <cmath>
+#include <vector>
 #include <cstdint>
 #include <cstring>
 
@@ -48,6 +50,29 @@ bool any_alias(const Range (&in)[NI], const Range (&out)[NO]) {
 }
 
 bool finite_positive(float x) { return std::isfinite(x) && x > 0.0f; }
+
+// Across a batch: true if an output range overlaps any other range (input or
+// output).  Sort by start; a range overlaps an earlier one iff it starts before
+// the largest end seen so far (of outputs, for an input; of all, for an output).
+struct Tagged {
+  uintptr_t lo, hi;
+  bool out;
+};
+bool batch_alias(std::vector<Tagged>& r) {
+  std::sort(r.begin(), r.end(), [](const Tagged& a, const Tagged& b) { return a.lo < b.lo; });
+  uintptr_t end_all = 0, end_out = 0;
+  for (const Tagged& x : r) {
+    if (x.out ? x.lo < end_all : x.lo < end_out) return true;
+    end_all = std::max(end_all, x.hi);
+    if (x.out) end_out = std::max(end_out, x.hi);
+  }
+  return false;
+}
+void add_range(std::vector<Tagged>& r, const void* p, uint64_t bytes, bool out) {
+  if (p == nullptr || bytes == 0) return;
+  const uintptr_t lo = reinterpret_cast<uintptr_t>(p);
+  r.push_back({lo, lo + uintptr_t(bytes), out});
+}
 
 roi_status check_common(int N, int M, float tau, int64_t rows, int64_t cols) {
   if (!(N >= 1 && N < M && M <= 32)) return ROI_ERR_NM;
@@ -128,6 +153,112 @@ static roi_status mask_fwd(const float* logits, const roi_bf16* W, int N, int M,
   if (c.status == nullptr) return ROI_ERR_CUDA;
   c.stream = static_cast<cudaStream_t>(stream);
   return finish(launch_fwd(c));
+}
+
+roi_status roi_mask_fwd_batch(const roi_fwd_item* items, int count, int N, int M, float tau, void* stream) {
+  if (count < 0) return ROI_ERR_SHAPE;
+  if (count > 0 && items == nullptr) return ROI_ERR_NULL;
+  roi_status s = check_common(N, M, tau, 0, M);
+  if (s != ROI_OK) return s;
+  std::vector<Tagged> ranges;
+  ranges.reserve(size_t(count) * 5);
+  for (int i = 0; i < count; ++i) {
+    const roi_fwd_item& it = items[i];
+    s = check_common(N, M, tau, it.rows, it.cols);
+    if (s != ROI_OK) return s;
+    if (it.st.row_offset < 0) return ROI_ERR_SHAPE;
+    if (!finite_positive(it.st.lambda)) return ROI_ERR_TAU;
+    if (it.rows == 0) continue;
+    if (it.logits == nullptr || it.W == nullptr || it.out_Wm == nullptr) return ROI_ERR_NULL;
+    if (!aligned16(it.logits) || !aligned16(it.W) || !aligned16(it.out_Wm) || !aligned16(it.out_soft) ||
+        !aligned16(it.out_hard))
+      return ROI_ERR_ALIGN;
+    const int64_t E = it.rows * it.cols;
+    add_range(ranges, it.logits, uint64_t(E) * 4, false);
+    add_range(ranges, it.W, uint64_t(E) * 2, false);
+    add_range(ranges, it.out_Wm, uint64_t(E) * 2, true);
+    add_range(ranges, it.out_soft, uint64_t(E) * 4, true);
+    add_range(ranges, it.out_hard, uint64_t((E + 31) / 32) * 4, true);
+  }
+  if (batch_alias(ranges)) return ROI_ERR_ALIAS;
+  if (ranges.empty()) return ROI_OK;  // only empty items: nothing is read or written
+  unsigned int* status = status_word();
+  if (status == nullptr) return ROI_ERR_CUDA;
+  std::vector<FwdCall> calls;
+  calls.reserve(size_t(count));
+  for (int i = 0; i < count; ++i) {
+    const roi_fwd_item& it = items[i];
+    if (it.rows == 0) continue;
+    FwdCall c;
+    c.phi = it.logits;
+    c.W = it.W;
+    c.Wm = it.out_Wm;
+    c.soft = it.out_soft;
+    c.hard = it.out_hard;
+    c.st = false;
+    c.E = it.rows * it.cols;
+    c.N = N;
+    c.M = M;
+    c.tau = tau;
+    c.np = make_noise(it.st, it.cols);
+    c.status = status;
+    c.stream = static_cast<cudaStream_t>(stream);
+    calls.push_back(c);
+  }
+  return finish(launch_fwd_batch(calls.data(), int(calls.size())));
+}
+
+roi_status roi_mask_bwd_batch(const roi_bwd_item* items, int count, int N, int M, float tau, void* stream) {
+  if (count < 0) return ROI_ERR_SHAPE;
+  if (count > 0 && items == nullptr) return ROI_ERR_NULL;
+  roi_status s = check_common(N, M, tau, 0, M);
+  if (s != ROI_OK) return s;
+  std::vector<Tagged> ranges;
+  ranges.reserve(size_t(count) * 5);
+  for (int i = 0; i < count; ++i) {
+    const roi_bwd_item& it = items[i];
+    s = check_common(N, M, tau, it.rows, it.cols);
+    if (s != ROI_OK) return s;
+    if (it.st.row_offset < 0) return ROI_ERR_SHAPE;
+    if (!finite_positive(it.st.lambda)) return ROI_ERR_TAU;
+    if (it.rows == 0) continue;
+    if (it.logits == nullptr || it.W == nullptr || it.dWm == nullptr || it.out_dlogits == nullptr)
+      return ROI_ERR_NULL;
+    if (!aligned16(it.logits) || !aligned16(it.W) || !aligned16(it.dWm) || !aligned16(it.out_dlogits) ||
+        !aligned16(it.out_dW))
+      return ROI_ERR_ALIGN;
+    const int64_t E = it.rows * it.cols;
+    add_range(ranges, it.logits, uint64_t(E) * 4, false);
+    add_range(ranges, it.W, uint64_t(E) * 2, false);
+    add_range(ranges, it.dWm, uint64_t(E) * 2, false);
+    add_range(ranges, it.out_dlogits, uint64_t(E) * 4, true);
+    add_range(ranges, it.out_dW, uint64_t(E) * 2, true);
+  }
+  if (batch_alias(ranges)) return ROI_ERR_ALIAS;
+  if (ranges.empty()) return ROI_OK;  // only empty items: nothing is read or written
+  unsigned int* status = status_word();
+  if (status == nullptr) return ROI_ERR_CUDA;
+  std::vector<BwdCall> calls;
+  calls.reserve(size_t(count));
+  for (int i = 0; i < count; ++i) {
+    const roi_bwd_item& it = items[i];
+    if (it.rows == 0) continue;
+    BwdCall c{};
+    c.phi = it.logits;
+    c.W = it.W;
+    c.dWm = it.dWm;
+    c.dphi = it.out_dlogits;
+    c.dW = it.out_dW;
+    c.E = it.rows * it.cols;
+    c.N = N;
+    c.M = M;
+    c.tau = tau;
+    c.np = make_noise(it.st, it.cols);
+    c.status = status;
+    c.stream = static_cast<cudaStream_t>(stream);
+    calls.push_back(c);
+  }
+  return finish(launch_bwd_batch(calls.data(), int(calls.size())));
 }
 
 roi_status roi_mask_fwd_ex(const float* logits, const roi_bf16* W, int N, int M, float tau,

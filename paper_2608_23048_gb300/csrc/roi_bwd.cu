@@ -337,13 +337,56 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
   }
 }
 
+// One full tile of a tensor (local tile index `tile`), inputs staged in shared
+// memory.
+template <int N, int M, bool TAU1, bool ST, bool OPT>
+__device__ __forceinline__ void bwd_tile(const uint8_t* const* stage, int64_t tile, const BwdArgs& a,
+                                         const BwdOptArgs& o, uint8_t* smem) {
+  using C = Cfg<M>;
+  const float* sphi = reinterpret_cast<const float*>(stage[0]);
+  const uint16_t* sW = reinterpret_cast<const uint16_t*>(stage[1]);
+  const uint16_t* sdW = reinterpret_cast<const uint16_t*>(stage[2]);
+  const int64_t base = tile * C::kTile;
+#pragma unroll
+  for (int p = 0; p < C::kPairs; ++p) {
+    const int g0 = threadIdx.x + 2 * p * C::kThreads, g1 = g0 + C::kThreads;
+    const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
+    const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
+    const uint16_t* pd[2] = {sdW + g0 * M, sdW + g1 * M};
+    const int64_t e0[2] = {base + g0 * M, base + g1 * M};
+    if constexpr (M == 4) {
+      bwd_groups<N, M, TAU1, F2, false, ST, OPT>(pp, pw, pd, e0, a, o);
+    } else {
+      // M = 8: the paired step history does not fit the register file; steps
+      // 0 .. N-2 go to shared memory behind the tile ring
+      F2* hist = reinterpret_cast<F2*>(smem + kHistOffset<M>) + threadIdx.x;
+      bwd_groups<N, M, TAU1, F2, true, ST, OPT>(pp, pw, pd, e0, a, o, hist);
+    }
+  }
+}
+
+// The ragged tail of a tensor (fewer than one tile after its full tiles), by one
+// CTA, straight from global memory.
+template <int N, int M, bool TAU1, bool ST, bool OPT>
+__device__ __forceinline__ void bwd_tail(const BwdArgs& a, const BwdOptArgs& o) {
+  using C = Cfg<M>;
+  const int64_t t0 = a.full_tiles * C::kTile;
+  const int64_t tail_groups = (a.E - t0) / M;
+  for (int64_t gi = threadIdx.x; gi < tail_groups; gi += C::kThreads) {
+    const float* pp[1] = {a.phi + t0 + gi * M};
+    const uint16_t* pw[1] = {a.W + t0 + gi * M};
+    const uint16_t* pd[1] = {a.dWm + t0 + gi * M};
+    const int64_t e0[1] = {t0 + gi * M};
+    bwd_groups<N, M, TAU1, float, false, ST, OPT>(pp, pw, pd, e0, a, o);
+  }
+}
+
 // ST: straight-through dW from the forward's hard bits; OPT: fused AdamW step on
 // the logits (separate instantiations, so the plain kernel's code is not touched)
 template <int N, int M, bool TAU1, bool ST, bool OPT>
 __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_kernel(BwdArgs a, BwdOptArgs o) {
   uint8_t* smem = roi_bwd_smem;
   using C = Cfg<M>;
-  constexpr int kT = C::kTile;
   TileSrc<3> src;
   src.ptr[0] = reinterpret_cast<const uint8_t*>(a.phi);
   src.esize[0] = 4;
@@ -351,43 +394,14 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_
   src.esize[1] = 2;
   src.ptr[2] = reinterpret_cast<const uint8_t*>(a.dWm);
   src.esize[2] = 2;
-
-  const bool ok = run_tiles<C::kThreads, kT, C::kStages, 3>(
-      smem, src, a.full_tiles, a.status, [&](const uint8_t* const* stage, int64_t tile) {
-        const float* sphi = reinterpret_cast<const float*>(stage[0]);
-        const uint16_t* sW = reinterpret_cast<const uint16_t*>(stage[1]);
-        const uint16_t* sdW = reinterpret_cast<const uint16_t*>(stage[2]);
-        const int64_t base = tile * kT;
-#pragma unroll
-        for (int p = 0; p < C::kPairs; ++p) {
-          const int g0 = threadIdx.x + 2 * p * C::kThreads, g1 = g0 + C::kThreads;
-          const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
-          const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
-          const uint16_t* pd[2] = {sdW + g0 * M, sdW + g1 * M};
-          const int64_t e0[2] = {base + g0 * M, base + g1 * M};
-          if constexpr (M == 4) {
-            bwd_groups<N, M, TAU1, F2, false, ST, OPT>(pp, pw, pd, e0, a, o);
-          } else {
-            // M = 8: the paired step history does not fit the register file; steps
-            // 0 .. N-2 go to shared memory behind the tile ring
-            F2* hist = reinterpret_cast<F2*>(smem + kHistOffset<M>) + threadIdx.x;
-            bwd_groups<N, M, TAU1, F2, true, ST, OPT>(pp, pw, pd, e0, a, o, hist);
-          }
-        }
-      });
-  if (!ok) return;
-
-  if (blockIdx.x == gridDim.x - 1) {
-    const int64_t t0 = a.full_tiles * kT;
-    const int64_t tail_groups = (a.E - t0) / M;
-    for (int64_t gi = threadIdx.x; gi < tail_groups; gi += C::kThreads) {
-      const float* pp[1] = {a.phi + t0 + gi * M};
-      const uint16_t* pw[1] = {a.W + t0 + gi * M};
-      const uint16_t* pd[1] = {a.dWm + t0 + gi * M};
-      const int64_t e0[1] = {t0 + gi * M};
-      bwd_groups<N, M, TAU1, float, false, ST, OPT>(pp, pw, pd, e0, a, o);
-    }
-  }
+  // a batch's next tensor may start on the SMs this launch frees (no-op otherwise)
+  pdl_launch_dependents();
+  const bool ok = run_tiles<C::kThreads, C::kTile, C::kStages, 3>(
+      smem, src, a.full_tiles, a.status,
+      [&](const uint8_t* const* stage, int64_t tile) { bwd_tile<N, M, TAU1, ST, OPT>(stage, tile, a, o, smem); });
+  if (ok && blockIdx.x == gridDim.x - 1) bwd_tail<N, M, TAU1, ST, OPT>(a, o);
+  // the launch completes only after the batch's previous one (stream order)
+  if (blockIdx.x == 0) pdl_wait();
 }
 
 __global__ void __launch_bounds__(128) roi_bwd_generic_kernel(BwdArgs a, BwdOptArgs o, int N, int M) {
@@ -431,7 +445,7 @@ struct LaunchCache {
 };
 
 template <int N, int M, bool TAU1, bool ST, bool OPT>
-int launch_tiles(const BwdArgs& a, const BwdOptArgs& o, cudaStream_t stream) {
+int launch_tiles(const BwdArgs& a, const BwdOptArgs& o, cudaStream_t stream, bool pdl = false) {
   using C = Cfg<M>;
   auto kern = roi_bwd_kernel<N, M, TAU1, ST, OPT>;
   const size_t smem = kHistBytes<N, M> == 0 ? tile_smem_bytes<C::kTile, C::kStages>(8)
@@ -450,13 +464,15 @@ int launch_tiles(const BwdArgs& a, const BwdOptArgs& o, cudaStream_t stream) {
   }
   const int64_t cap = int64_t(sm_count()) * cache.per_sm[dev];
   const int grid = int(a.full_tiles < 1 ? 1 : (a.full_tiles < cap ? a.full_tiles : cap));
-  kern<<<grid, C::kThreads, smem, stream>>>(a, o);
-  return cudaGetLastError() == cudaSuccess ? 1 : -1;
+  return launch_maybe_pdl(kern, grid, C::kThreads, smem, stream, pdl, a, o);
 }
 
 template <int N, int M>
-int launch_nm(const BwdArgs& a, const BwdOptArgs& o, cudaStream_t stream) {
+int launch_nm(const BwdArgs& a, const BwdOptArgs& o, cudaStream_t stream, bool pdl = false) {
   const bool t1 = a.tau == 1.0f;
+  if (pdl && o.phi_out == nullptr && !(a.hard_in != nullptr && a.dW != nullptr))
+    return t1 ? launch_tiles<N, M, true, false, false>(a, o, stream, true)
+              : launch_tiles<N, M, false, false, false>(a, o, stream, true);
   if (o.phi_out != nullptr)
     return t1 ? launch_tiles<N, M, true, false, true>(a, o, stream) : launch_tiles<N, M, false, false, true>(a, o, stream);
   if (a.hard_in != nullptr && a.dW != nullptr)
@@ -466,7 +482,8 @@ int launch_nm(const BwdArgs& a, const BwdOptArgs& o, cudaStream_t stream) {
 
 }  // namespace
 
-int launch_bwd(const BwdCall& c) {
+namespace {
+int launch_bwd_impl(const BwdCall& c, bool pdl) {
   BwdArgs a;
   a.phi = c.phi;
   a.W = c.W;
@@ -485,9 +502,9 @@ int launch_bwd(const BwdCall& c) {
   a.inv_tau = 1.0f / c.tau;
   a.np = c.np;
   a.status = c.status;
-  if (c.N == 2 && c.M == 4) return launch_nm<2, 4>(a, o, c.stream);
-  if (c.N == 4 && c.M == 8) return launch_nm<4, 8>(a, o, c.stream);
-  if (c.N == 2 && c.M == 8) return launch_nm<2, 8>(a, o, c.stream);
+  if (c.N == 2 && c.M == 4) return launch_nm<2, 4>(a, o, c.stream, pdl);
+  if (c.N == 4 && c.M == 8) return launch_nm<4, 8>(a, o, c.stream, pdl);
+  if (c.N == 2 && c.M == 8) return launch_nm<2, 8>(a, o, c.stream, pdl);
   if (slice_supported(c.N, c.M)) return launch_slice_bwd(c);
   const int64_t groups = c.E / c.M;
   int64_t blocks = (groups + 127) / 128;
@@ -496,6 +513,26 @@ int launch_bwd(const BwdCall& c) {
   if (blocks < 1) blocks = 1;
   roi_bwd_generic_kernel<<<int(blocks), 128, 0, c.stream>>>(a, o, c.N, c.M);
   return cudaGetLastError() == cudaSuccess ? 1 : -1;
+}
+}  // namespace
+
+int launch_bwd(const BwdCall& c) { return launch_bwd_impl(c, false); }
+
+// As launch_fwd_batch: the tensors are independent, so from the second one on the
+// plain tile kernels are launched with programmatic stream serialization.
+int launch_bwd_batch(const BwdCall* calls, int count) {
+  int launched = 0;
+  bool prev_tiled = false;
+  for (int i = 0; i < count; ++i) {
+    const BwdCall& c = calls[i];
+    const bool tiled = ((c.N == 2 && c.M == 4) || (c.N == 4 && c.M == 8) || (c.N == 2 && c.M == 8)) &&
+                       c.phi_out == nullptr && c.hard_in == nullptr;
+    const int r = launch_bwd_impl(c, tiled && prev_tiled);
+    if (r < 0) return -1;
+    launched += r;
+    prev_tiled = tiled && r > 0;
+  }
+  return launched;
 }
 
 }  // namespace roi

@@ -265,70 +265,83 @@ __device__ __forceinline__ void store_hard_pair(uint32_t* hard, int64_t e0a, int
   if (lane % kHalf == 0) hard[(upper ? e0b : e0a) >> 5] = word;
 }
 
+// One full tile of a tensor (local tile index `tile`), inputs staged in shared
+// memory.
+template <int N, int M, bool TAU1, bool ST>
+__device__ __forceinline__ void fwd_tile(const uint8_t* const* stage, int64_t tile, const FwdArgs& a) {
+  using C = Cfg<M>;
+  constexpr int kT = C::kTile;
+  const float* sphi = reinterpret_cast<const float*>(stage[0]);
+  const uint16_t* sW = reinterpret_cast<const uint16_t*>(stage[1]);
+  const int64_t base = tile * kT;
+  // pair p: groups t and t + kThreads of the p-th block of 2 kThreads groups.
+  // The keys of pair p + 1 (integer-heavy: Philox, range reduction) are
+  // formed before pair p is relaxed (floating-point-heavy), so the two
+  // streams share the issue slots of one basic block.
+  F2 kap[2][M];
+  {
+    const int g0 = threadIdx.x, g1 = g0 + C::kThreads;
+    const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
+    const int64_t e0[2] = {base + g0 * M, base + g1 * M};
+    fwd_keys<M, F2>(pp, e0, a, kap[0]);
+  }
+#pragma unroll
+  for (int p = 0; p < C::kPairs; ++p) {
+    if (p + 1 < C::kPairs) {
+      const int g0 = threadIdx.x + 2 * (p + 1) * C::kThreads, g1 = g0 + C::kThreads;
+      const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
+      const int64_t e0[2] = {base + g0 * M, base + g1 * M};
+      fwd_keys<M, F2>(pp, e0, a, kap[(p + 1) & 1]);
+    }
+    const int g0 = threadIdx.x + 2 * p * C::kThreads, g1 = g0 + C::kThreads;
+    const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
+    const int64_t e0[2] = {base + g0 * M, base + g1 * M};
+    uint32_t bits[2];
+    fwd_finish<N, M, TAU1, F2, ST>(kap[p & 1], pw, e0, a, bits);
+    if (a.hard != nullptr) store_hard_pair<M>(a.hard, e0[0], e0[1], bits[0], bits[1]);
+  }
+}
+
+// The ragged tail of a tensor (fewer than one tile after its full tiles), by one
+// CTA, straight from global memory.
+template <int N, int M, bool TAU1, bool ST>
+__device__ __forceinline__ void fwd_tail(const FwdArgs& a) {
+  using C = Cfg<M>;
+  const int64_t t0 = a.full_tiles * C::kTile;
+  const int64_t tail_groups = (a.E - t0) / M;
+  const int64_t rounds = (tail_groups + C::kThreads - 1) / C::kThreads;
+  for (int64_t r = 0; r < rounds; ++r) {
+    const int64_t gi = threadIdx.x + r * C::kThreads;
+    const bool active = gi < tail_groups;
+    uint32_t bits = 0;
+    if (active) {
+      const float* pp[1] = {a.phi + t0 + gi * M};
+      const uint16_t* pw[1] = {a.W + t0 + gi * M};
+      const int64_t e0[1] = {t0 + gi * M};
+      fwd_groups<N, M, TAU1, float, ST>(pp, pw, e0, a, &bits);
+    }
+    if (a.hard != nullptr) store_hard<M>(a.hard, t0 + gi * M, bits, active);
+  }
+}
+
 // ST: straight-through Wm (a separate instantiation)
 template <int N, int M, bool TAU1, bool ST>
 __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_fwd_kernel(FwdArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   using C = Cfg<M>;
-  constexpr int kT = C::kTile;
   TileSrc<2> src;
   src.ptr[0] = reinterpret_cast<const uint8_t*>(a.phi);
   src.esize[0] = 4;
   src.ptr[1] = reinterpret_cast<const uint8_t*>(a.W);
   src.esize[1] = 2;
-
-  const bool ok = run_tiles<C::kThreads, kT, C::kStages, 2>(
-      smem, src, a.full_tiles, a.status, [&](const uint8_t* const* stage, int64_t tile) {
-        const float* sphi = reinterpret_cast<const float*>(stage[0]);
-        const uint16_t* sW = reinterpret_cast<const uint16_t*>(stage[1]);
-        const int64_t base = tile * kT;
-        // pair p: groups t and t + kThreads of the p-th block of 2 kThreads groups.
-        // The keys of pair p + 1 (integer-heavy: Philox, range reduction) are
-        // formed before pair p is relaxed (floating-point-heavy), so the two
-        // streams share the issue slots of one basic block.
-        F2 kap[2][M];
-        {
-          const int g0 = threadIdx.x, g1 = g0 + C::kThreads;
-          const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
-          const int64_t e0[2] = {base + g0 * M, base + g1 * M};
-          fwd_keys<M, F2>(pp, e0, a, kap[0]);
-        }
-#pragma unroll
-        for (int p = 0; p < C::kPairs; ++p) {
-          if (p + 1 < C::kPairs) {
-            const int g0 = threadIdx.x + 2 * (p + 1) * C::kThreads, g1 = g0 + C::kThreads;
-            const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
-            const int64_t e0[2] = {base + g0 * M, base + g1 * M};
-            fwd_keys<M, F2>(pp, e0, a, kap[(p + 1) & 1]);
-          }
-          const int g0 = threadIdx.x + 2 * p * C::kThreads, g1 = g0 + C::kThreads;
-          const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
-          const int64_t e0[2] = {base + g0 * M, base + g1 * M};
-          uint32_t bits[2];
-          fwd_finish<N, M, TAU1, F2, ST>(kap[p & 1], pw, e0, a, bits);
-          if (a.hard != nullptr) store_hard_pair<M>(a.hard, e0[0], e0[1], bits[0], bits[1]);
-        }
-      });
-  if (!ok) return;
-
-  // ragged tail (fewer than one tile), last CTA, straight from global memory
-  if (blockIdx.x == gridDim.x - 1) {
-    const int64_t t0 = a.full_tiles * kT;
-    const int64_t tail_groups = (a.E - t0) / M;
-    const int64_t rounds = (tail_groups + C::kThreads - 1) / C::kThreads;
-    for (int64_t r = 0; r < rounds; ++r) {
-      const int64_t gi = threadIdx.x + r * C::kThreads;
-      const bool active = gi < tail_groups;
-      uint32_t bits = 0;
-      if (active) {
-        const float* pp[1] = {a.phi + t0 + gi * M};
-        const uint16_t* pw[1] = {a.W + t0 + gi * M};
-        const int64_t e0[1] = {t0 + gi * M};
-        fwd_groups<N, M, TAU1, float, ST>(pp, pw, e0, a, &bits);
-      }
-      if (a.hard != nullptr) store_hard<M>(a.hard, t0 + gi * M, bits, active);
-    }
-  }
+  // a batch's next tensor may start on the SMs this launch frees (no-op otherwise)
+  pdl_launch_dependents();
+  const bool ok = run_tiles<C::kThreads, C::kTile, C::kStages, 2>(
+      smem, src, a.full_tiles, a.status,
+      [&](const uint8_t* const* stage, int64_t tile) { fwd_tile<N, M, TAU1, ST>(stage, tile, a); });
+  if (ok && blockIdx.x == gridDim.x - 1) fwd_tail<N, M, TAU1, ST>(a);
+  // the launch completes only after the batch's previous one (stream order)
+  if (blockIdx.x == 0) pdl_wait();
 }
 
 // Any 1 <= N < M <= 32: one thread per group, exact log-space routine, direct
@@ -367,7 +380,7 @@ struct LaunchCache {
 };
 
 template <int N, int M, bool TAU1, bool ST>
-int launch_tiles(const FwdArgs& a, cudaStream_t stream) {
+int launch_tiles(const FwdArgs& a, cudaStream_t stream, bool pdl) {
   using C = Cfg<M>;
   auto kern = roi_fwd_kernel<N, M, TAU1, ST>;
   const size_t smem = tile_smem_bytes<C::kTile, C::kStages>(6);
@@ -383,19 +396,21 @@ int launch_tiles(const FwdArgs& a, cudaStream_t stream) {
   }
   const int64_t cap = int64_t(sm_count()) * cache.per_sm[dev];
   const int grid = int(a.full_tiles < 1 ? 1 : (a.full_tiles < cap ? a.full_tiles : cap));
-  kern<<<grid, C::kThreads, smem, stream>>>(a);
-  return cudaGetLastError() == cudaSuccess ? 1 : -1;
+  return launch_maybe_pdl(kern, grid, C::kThreads, smem, stream, pdl, a);
 }
 
 template <int N, int M>
-int launch_nm(const FwdArgs& a, cudaStream_t stream) {
-  if (a.st) return a.tau == 1.0f ? launch_tiles<N, M, true, true>(a, stream) : launch_tiles<N, M, false, true>(a, stream);
-  return a.tau == 1.0f ? launch_tiles<N, M, true, false>(a, stream) : launch_tiles<N, M, false, false>(a, stream);
+int launch_nm(const FwdArgs& a, cudaStream_t stream, bool pdl = false) {
+  if (a.st)
+    return a.tau == 1.0f ? launch_tiles<N, M, true, true>(a, stream, pdl) : launch_tiles<N, M, false, true>(a, stream, pdl);
+  return a.tau == 1.0f ? launch_tiles<N, M, true, false>(a, stream, pdl)
+                       : launch_tiles<N, M, false, false>(a, stream, pdl);
 }
 
 }  // namespace
 
-int launch_fwd(const FwdCall& c) {
+namespace {
+int launch_fwd_impl(const FwdCall& c, bool pdl) {
   FwdArgs a;
   a.phi = c.phi;
   a.W = c.W;
@@ -409,9 +424,9 @@ int launch_fwd(const FwdCall& c) {
   a.inv_tau = 1.0f / c.tau;
   a.np = c.np;
   a.status = c.status;
-  if (c.N == 2 && c.M == 4) return launch_nm<2, 4>(a, c.stream);
-  if (c.N == 4 && c.M == 8) return launch_nm<4, 8>(a, c.stream);
-  if (c.N == 2 && c.M == 8) return launch_nm<2, 8>(a, c.stream);
+  if (c.N == 2 && c.M == 4) return launch_nm<2, 4>(a, c.stream, pdl);
+  if (c.N == 4 && c.M == 8) return launch_nm<4, 8>(a, c.stream, pdl);
+  if (c.N == 2 && c.M == 8) return launch_nm<2, 8>(a, c.stream, pdl);
   if (slice_supported(c.N, c.M)) return launch_slice_fwd(c);
   // generic path
   int launched = 0;
@@ -426,6 +441,27 @@ int launch_fwd(const FwdCall& c) {
   roi_fwd_generic_kernel<<<int(blocks), 128, 0, c.stream>>>(a, c.N, c.M);
   launched += 1;
   return cudaGetLastError() == cudaSuccess ? launched : -1;
+}
+}  // namespace
+
+int launch_fwd(const FwdCall& c) { return launch_fwd_impl(c, false); }
+
+// The tensors of a batch are independent (the caller checked that no output
+// overlaps another range), so from the second one on the tile kernels are launched
+// with programmatic stream serialization: each may start while the previous one
+// drains, and completes only after it (see roi_fwd_kernel).
+int launch_fwd_batch(const FwdCall* calls, int count) {
+  int launched = 0;
+  bool prev_tiled = false;
+  for (int i = 0; i < count; ++i) {
+    const FwdCall& c = calls[i];
+    const bool tiled = (c.N == 2 && c.M == 4) || (c.N == 4 && c.M == 8) || (c.N == 2 && c.M == 8);
+    const int r = launch_fwd_impl(c, tiled && prev_tiled);
+    if (r < 0) return -1;
+    launched += r;
+    prev_tiled = tiled && r > 0;
+  }
+  return launched;
 }
 
 }  // namespace roi

@@ -79,6 +79,11 @@ struct LinearCall {
 // Each returns the number of kernels launched (>= 0) or -1 after a CUDA error.
 int launch_fwd(const FwdCall& c);
 int launch_bwd(const BwdCall& c);
+// Many independent tensors on one stream: one launch per tensor, the tile kernels
+// chained by programmatic dependent launch so each may start while the previous
+// one drains (stream order is kept: each completes after its predecessor).
+int launch_fwd_batch(const FwdCall* calls, int count);
+int launch_bwd_batch(const BwdCall* calls, int count);
 int launch_export(const ExportCall& c);
 int launch_export_compressed_2of4(const CompressCall& c);
 // Warp-slice kernels for M = 16, 32 (roi_slice.cu).
@@ -92,6 +97,29 @@ bool linear_supported(int N, int M);
 int linear_splits(int64_t T, int64_t rows, int64_t cols);
 size_t linear_workspace_bytes(int64_t T, int64_t rows, int64_t cols);
 int launch_masked_linear(const LinearCall& c);
+
+// Launches kern<<<grid, threads, smem, stream>>>(args...), with programmatic stream
+// serialization allowed when `pdl` (the kernel then may start before the stream's
+// previous kernel has finished).  Returns 1, or -1 after a CUDA error.
+template <class... KArgs, class... Args>
+int launch_maybe_pdl(void (*kern)(KArgs...), int grid, int threads, size_t smem, cudaStream_t stream, bool pdl,
+                     const Args&... args) {
+  if (!pdl) {
+    kern<<<grid, threads, smem, stream>>>(args...);
+    return cudaGetLastError() == cudaSuccess ? 1 : -1;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(unsigned(grid));
+  cfg.blockDim = dim3(unsigned(threads));
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, args...) == cudaSuccess ? 1 : -1;
+}
 
 // Streaming multiprocessors of the current device (cached).
 int sm_count();

@@ -24,11 +24,13 @@ constexpr size_t tile_smem_bytes(uint32_t bytes_per_element) {
   return ((size_t(STAGES) * TILE * bytes_per_element + 7) & ~size_t(7)) + size_t(STAGES) * 16;
 }
 
-// Runs `compute(stage_ptrs, tile)` for every full tile of this CTA.  Returns
-// false if a wait timed out (status recorded, copies drained).
-template <int THREADS, int TILE, int STAGES, int NARR, class Compute>
-__device__ __forceinline__ bool run_tiles(uint8_t* smem, const TileSrc<NARR>& src, int64_t full_tiles,
-                                          unsigned int* status, Compute&& compute) {
+// Runs `compute(stage_ptrs, tile)` for every tile of this CTA among tiles
+// 0 .. full_tiles - 1; `src_of(tile, a)` gives the global address of input array
+// a's part of the tile (TILE * esize[a] contiguous bytes, 16-byte aligned).
+// Returns false if a wait timed out (status recorded, copies drained).
+template <int THREADS, int TILE, int STAGES, int NARR, class SrcOf, class Compute>
+__device__ __forceinline__ bool run_tiles_src(uint8_t* smem, const uint32_t (&esize)[NARR], int64_t full_tiles,
+                                              unsigned int* status, SrcOf&& src_of, Compute&& compute) {
   constexpr int kWarps = THREADS / 32;
   const int tid = threadIdx.x;
   const int lane = tid & 31;
@@ -38,8 +40,8 @@ __device__ __forceinline__ bool run_tiles(uint8_t* smem, const TileSrc<NARR>& sr
 #pragma unroll
   for (int a = 0; a < NARR; ++a) {
     arr_off[a] = off;
-    off += size_t(STAGES) * TILE * src.esize[a];
-    stage_bytes += TILE * src.esize[a];
+    off += size_t(STAGES) * TILE * esize[a];
+    stage_bytes += TILE * esize[a];
   }
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + ((off + 7) & ~size_t(7)));
   uint32_t* done = reinterpret_cast<uint32_t*>(bars + STAGES);   // warps finished with the current fill
@@ -55,9 +57,8 @@ __device__ __forceinline__ bool run_tiles(uint8_t* smem, const TileSrc<NARR>& sr
     mbar_arrive_expect_tx(&bars[s], stage_bytes);
 #pragma unroll
     for (int a = 0; a < NARR; ++a) {
-      const uint32_t es = src.esize[a];
-      bulk_g2s(smem + arr_off[a] + size_t(s) * TILE * es, src.ptr[a] + size_t(t) * TILE * es, TILE * es,
-               &bars[s]);
+      const uint32_t es = esize[a];
+      bulk_g2s(smem + arr_off[a] + size_t(s) * TILE * es, src_of(t, a), TILE * es, &bars[s]);
     }
   };
 
@@ -92,7 +93,7 @@ __device__ __forceinline__ bool run_tiles(uint8_t* smem, const TileSrc<NARR>& sr
     }
     const uint8_t* stage[NARR];
 #pragma unroll
-    for (int a = 0; a < NARR; ++a) stage[a] = smem + arr_off[a] + size_t(s) * TILE * src.esize[a];
+    for (int a = 0; a < NARR; ++a) stage[a] = smem + arr_off[a] + size_t(s) * TILE * esize[a];
     compute(stage, tile);
     __syncwarp();
     if (lane == 0) {
@@ -112,6 +113,15 @@ __device__ __forceinline__ bool run_tiles(uint8_t* smem, const TileSrc<NARR>& sr
     }
   }
   return true;
+}
+
+// One tensor per input array: tile t of array a starts at ptr[a] + t * TILE * esize[a].
+template <int THREADS, int TILE, int STAGES, int NARR, class Compute>
+__device__ __forceinline__ bool run_tiles(uint8_t* smem, const TileSrc<NARR>& src, int64_t full_tiles,
+                                          unsigned int* status, Compute&& compute) {
+  return run_tiles_src<THREADS, TILE, STAGES, NARR>(
+      smem, src.esize, full_tiles, status,
+      [&](int64_t t, int a) { return src.ptr[a] + size_t(t) * TILE * src.esize[a]; }, compute);
 }
 
 }  // namespace roi

@@ -130,6 +130,31 @@ def test_validation_codes(L):
     assert L.roi_masked_linear_fwd_noalloc(_fake(D), _fake(A), _fake(B), 2, 4, 1.0, ctypes.byref(st), 257, 128, 64,
                                            _fake(C), None) == 2
     assert L.roi_masked_linear_workspace_size(0, 128, 64) == 0 and L.roi_masked_linear_workspace_size(300, 128, 64) == 0
+    # batches: every item validated as the single call, plus no output overlapping any other range
+    def fitem(logits=A, W=B, Wm=C, soft=None, hard=None, rows=4, cols=8, state=None):
+        return roi.FwdItem(logits, W, Wm, soft, hard, rows, cols, state or roi.NoiseState(0, 0, 0, 1.0, 0))
+    def fbatch(*its, N=2, M=4, tau=1.0):
+        arr = (roi.FwdItem * len(its))(*its)
+        return L.roi_mask_fwd_batch(arr, len(its), N, M, tau, None)
+    assert L.roi_mask_fwd_batch(None, 2, 2, 4, 1.0, None) == 1
+    assert L.roi_mask_fwd_batch(None, -1, 2, 4, 1.0, None) == 2
+    assert L.roi_mask_fwd_batch(None, 0, 2, 4, 1.0, None) == 0
+    assert fbatch(fitem(), fitem(logits=0x60000000, W=0x61000000, Wm=0)) == 1
+    assert fbatch(fitem(), N=4) == 3 and fbatch(fitem(cols=6)) == 2 and fbatch(fitem(), tau=0.0) == 4
+    assert fbatch(fitem(state=roi.NoiseState(0, 0, 0, 0.0, 0))) == 4
+    assert fbatch(fitem(hard=D + 4)) == 5
+    # item 2's output overlaps item 1's logits; item 2's output overlaps item 1's output
+    assert fbatch(fitem(), fitem(logits=0x60000000, W=0x61000000, Wm=A + 16)) == 6
+    assert fbatch(fitem(), fitem(logits=0x60000000, W=0x61000000, Wm=C + 32)) == 6
+    # inputs may be shared between items; empty items only: nothing to do
+    assert fbatch(fitem(rows=0, logits=0, W=0, Wm=0), fitem(rows=0, logits=0, W=0, Wm=0)) == 0
+    def bitem(logits=A, W=B, dWm=C, dl=D, dW=None, rows=4, cols=8):
+        return roi.BwdItem(logits, W, dWm, dl, dW, rows, cols, roi.NoiseState(0, 0, 0, 1.0, 0))
+    def bbatch(*its, N=2, M=4):
+        arr = (roi.BwdItem * len(its))(*its)
+        return L.roi_mask_bwd_batch(arr, len(its), N, M, 1.0, None)
+    assert bbatch(bitem(dl=0)) == 1 and bbatch(bitem(dW=E + 2)) == 5
+    assert bbatch(bitem(), bitem(logits=0x60000000, W=0x61000000, dWm=0x62000000, dl=B + 16)) == 6
     for s in range(10):
         assert L.roi_status_string(s)
 

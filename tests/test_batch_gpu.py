@@ -1,0 +1,151 @@
+"""Batched calls (roi_mask_fwd_batch / roi_mask_bwd_batch): many tensors per call,
+their launches chained by programmatic dependent launch, must give, bit for bit,
+what the single-tensor calls give, and match the oracle.  Sets mix tensors with and
+without full tiles, ragged tails,
+per-item noise states (seed, step, tensor_id, lambda, row_offset), optional outputs,
+empty items, 300 items, and an (N, M) without a tile kernel (no chaining)."""
+import numpy as np
+import pytest
+
+import workloads as WL
+from oracle import roi_oracle as O
+import _compare as C
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def roi():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2608_23048_gb300 import _build
+    _build.build()
+    import paper_2608_23048_gb300 as roi
+    return roi
+
+
+def _u16(t):
+    import torch
+    return t.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+
+
+def make_set(shapes, seed0):
+    import torch
+    dev = torch.device("cuda")
+    out = []
+    for k, (rows, cols) in enumerate(shapes):
+        W, phi, dWm = WL.make_inputs(rows, cols, "normal" if k % 2 else "logw", seed0 + k)
+        st = (seed0 * 7 + k, 3 + k % 5, k, [1.0, 0.7, 1.3][k % 3], (k * 37) % 11)
+        out.append({"W": W.to(dev), "phi": phi.to(dev), "dWm": dWm.to(dev), "st": st, "rows": rows, "cols": cols})
+    return out
+
+
+def outputs(roi, t, soft, hard, dW):
+    import torch
+    rows, cols = t["rows"], t["cols"]
+    return {"Wm": torch.full((rows, cols), -1, dtype=torch.int16, device="cuda").view(torch.bfloat16),
+            "soft": torch.full((rows, cols), float("nan"), device="cuda") if soft else None,
+            "hard": torch.full((roi.hard_words(rows, cols),), -1, dtype=torch.int32, device="cuda") if hard else None,
+            "dphi": torch.full((rows, cols), float("nan"), device="cuda"),
+            "dW": torch.full((rows, cols), -1, dtype=torch.int16, device="cuda").view(torch.bfloat16) if dW else None}
+
+
+def run_single(roi, ts, N, M, tau, flags):
+    res = []
+    for t, (soft, hard, dW) in zip(ts, flags):
+        o = outputs(roi, t, soft, hard, dW)
+        roi.roi_mask_fwd_ex(t["phi"], t["W"], N, M, tau, t["st"], o["Wm"], o["soft"], o["hard"])
+        roi.roi_mask_bwd(t["phi"], t["W"], t["st"], N, M, t["dWm"], tau, o["dphi"], o["dW"])
+        res.append(o)
+    roi.roi_device_status()
+    return res
+
+
+def run_batch(roi, ts, N, M, tau, flags):
+    res = [outputs(roi, t, *f) for t, f in zip(ts, flags)]
+    roi.roi_mask_fwd_batch([(t["phi"], t["W"], t["st"], o["Wm"], o["soft"], o["hard"]) for t, o in zip(ts, res)],
+                           N, M, tau)
+    roi.roi_mask_bwd_batch([(t["phi"], t["W"], t["st"], t["dWm"], o["dphi"], o["dW"]) for t, o in zip(ts, res)],
+                           N, M, tau)
+    roi.roi_device_status()
+    return res
+
+
+def assert_same(a, b):
+    import torch
+    for k in a:
+        if a[k] is None:
+            assert b[k] is None
+            continue
+        x, y = a[k], b[k]
+        if x.dtype == torch.bfloat16:
+            x, y = x.view(torch.int16), y.view(torch.int16)
+        assert torch.equal(x, y) if x.dtype != torch.float32 else torch.equal(x.view(torch.int32), y.view(torch.int32)), k
+
+
+# shapes: tails of every size, tensors smaller than one tile, large ones spanning many tiles
+SHAPES = [(37, 1000), (3, 64), (64, 3584), (512, 256), (1, 32), (129, 2048), (8, 8), (300, 520), (16, 24576)]
+
+
+@pytest.mark.parametrize("N,M,tau", [(2, 4, 1.0), (2, 4, 0.5), (4, 8, 1.0), (4, 8, 0.3), (2, 8, 1.0), (3, 4, 0.8)])
+def test_batch_equals_single_calls(roi, N, M, tau):
+    shapes = [(r, c) for r, c in SHAPES if c % M == 0]
+    ts = make_set(shapes, 40 + M + int(10 * tau))
+    flags = [(k % 3 == 0, k % 2 == 0, k % 4 == 1) for k in range(len(ts))]
+    single = run_single(roi, ts, N, M, tau, flags)
+    batch = run_batch(roi, ts, N, M, tau, flags)
+    for a, b in zip(single, batch):
+        assert_same(a, b)
+
+
+def test_batch_matches_oracle(roi):
+    N, M, tau = 2, 4, 1.0
+    shapes = [(37, 1000), (5, 96), (64, 3584), (1, 32)]
+    ts = make_set(shapes, 90)
+    flags = [(True, True, True)] * len(ts)
+    res = run_batch(roi, ts, N, M, tau, flags)
+    for t, o in zip(ts, res):
+        seed, step, tid, lam, roff = t["st"]
+        ph, Wb, dWb = t["phi"].cpu().numpy(), _u16(t["W"]), _u16(t["dWm"])
+        kw = dict(tensor_id=tid, lam=lam, row_offset=roff)
+        f64 = O.mask_fwd(ph, Wb, N, M, tau, seed, step, **kw)
+        f32 = O.mask_fwd(ph, Wb, N, M, tau, seed, step, dtype=np.float32, **kw)
+        b64 = O.mask_bwd(ph, Wb, dWb, N, M, tau, seed, step, **kw)
+        E = t["rows"] * t["cols"]
+        outside, _ = C.hard_mismatches(o["hard"].cpu().numpy().view(np.uint32), f64["hard_bits"], f64["keys"], N, M, E)
+        assert outside == 0
+        tolS = (C.soft_tolerance(f64["soft"], f64["keys"], N, M, tau).ravel()
+                + 4.0 * np.abs(f32["soft"].astype(np.float64) - f64["soft"]).ravel())
+        assert np.all(np.abs(o["soft"].cpu().numpy().ravel() - f64["soft"].ravel()) <= tolS)
+        c = (O.bf16_to_f32(dWb).astype(np.float64) * O.bf16_to_f32(Wb)).ravel()
+        assert C.plain_relative(o["dphi"].cpu().numpy(), b64["dlogits"], c, M, tau, lam) <= 1e-5
+
+
+def test_more_items_than_one_launch_and_empty_items(roi):
+    """300 items with empty ones mixed in."""
+    import torch
+    N, M, tau = 2, 4, 1.0
+    shapes = [((k * 7) % 13 + 1, 32 * ((k % 5) + 1)) for k in range(300)]
+    ts = make_set(shapes, 7)
+    flags = [(False, True, False)] * len(ts)
+    empty = {"W": torch.empty(0, 32, dtype=torch.bfloat16, device="cuda"),
+             "phi": torch.empty(0, 32, device="cuda"), "dWm": torch.empty(0, 32, dtype=torch.bfloat16, device="cuda"),
+             "st": (0, 0, 0, 1.0, 0), "rows": 0, "cols": 32}
+    ts = ts[:100] + [empty] + ts[100:] + [empty]
+    flags = flags[:100] + [(False, True, False)] + flags[100:] + [(False, True, False)]
+    single = run_single(roi, [t for t in ts if t["rows"]], N, M, tau, [f for t, f in zip(ts, flags) if t["rows"]])
+    batch = run_batch(roi, ts, N, M, tau, flags)
+    batch = [b for t, b in zip(ts, batch) if t["rows"]]
+    for a, b in zip(single, batch):
+        assert_same(a, b)
+
+
+def test_batch_launches_one_kernel_per_tensor_and_direction(roi):
+    N, M, tau = 2, 4, 1.0
+    ts = make_set([(64, 3584), (16, 512), (37, 1000)], 3)
+    flags = [(False, True, False)] * len(ts)
+    run_batch(roi, ts, N, M, tau, flags)
+    before = roi.roi_launch_count()
+    run_batch(roi, ts, N, M, tau, flags)
+    assert roi.roi_launch_count() - before == 2 * len(ts)
