@@ -149,3 +149,31 @@ def test_batch_launches_one_kernel_per_tensor_and_direction(roi):
     before = roi.roi_launch_count()
     run_batch(roi, ts, N, M, tau, flags)
     assert roi.roi_launch_count() - before == 2 * len(ts)
+
+
+def test_work_queued_after_a_batch_sees_every_item(roi):
+    """Launch chaining keeps stream order: a reduction queued on the same stream right
+    after the batched calls (no synchronisation in between) reads every item's
+    finished outputs, including those of early items whose successors started
+    before they ended."""
+    import torch
+    N, M, tau = 2, 4, 1.0
+    shapes = [(1024, 3584), (64, 512), (8, 256)] * 6 + [(2048, 3584)]
+    ts = make_set(shapes, 11)
+    flags = [(False, True, False)] * len(ts)
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        for rep in range(3):
+            res = [outputs(roi, t, *f) for t, f in zip(ts, flags)]
+            torch.cuda.current_stream().wait_stream(torch.cuda.default_stream())
+            roi.roi_mask_fwd_batch([(t["phi"], t["W"], t["st"], o["Wm"], None, o["hard"])
+                                    for t, o in zip(ts, res)], N, M, tau, stream=stream)
+            roi.roi_mask_bwd_batch([(t["phi"], t["W"], t["st"], t["dWm"], o["dphi"], None)
+                                    for t, o in zip(ts, res)], N, M, tau, stream=stream)
+            # queued behind the batch: every output must already be final
+            nan_dphi = torch.stack([o["dphi"].isnan().any() for o in res]).any()
+            sums = torch.stack([o["Wm"].float().sum() for o in res])
+            stream.synchronize()
+            assert not bool(nan_dphi)
+            again = torch.stack([o["Wm"].float().sum() for o in res])
+            assert torch.equal(sums, again)
