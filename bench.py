@@ -590,12 +590,31 @@ def run_variant(args):
                      meta=torch.empty(rows * cols // 32, dtype=torch.int32, device=dev))
         tensors.append(t)
     stream = torch.cuda.Stream(device=dev)
+    if args.op == "adamw":
+        adamw_fwd = roi.make_fwd_items([(t["phi"], t["W"], roi.NoiseState(0, 0, t["id"], 1.0, 0), t["Wm"], None,
+                                         t["hard"]) for t in tensors])
+        adamw_bwd = roi.make_adamw_items([(t["phi"], t["W"], roi.NoiseState(0, 0, t["id"], 1.0, 0), t["dWm"], t["m"],
+                                           t["v"], None, None) for t in reversed(tensors)])
 
     def launches(s, ev):
         def rec(lst):
             if ev is not None:
                 lst.append(torch.cuda.Event(enable_timing=True))
                 lst[-1].record(stream)
+        if args.op == "adamw" and not args.per_tensor:
+            # the training step's two calls: every forward, then every backward fused
+            # with the logits' AdamW step (chained launches)
+            for arr in (adamw_fwd, adamw_bwd):
+                for k in range(len(arr)):
+                    arr[k].st.step = s
+            rec(ev[0] if ev else None)
+            roi.roi_mask_fwd_batch(adamw_fwd, N, M, tau, stream=stream)
+            rec(ev[1] if ev else None)
+            rec(ev[2] if ev else None)
+            roi.roi_mask_bwd_adamw_batch(adamw_bwd, N, M, tau, roi.AdamW(1e-3, 0.9, 0.95, 1e-8, 0.05, s + 1),
+                                         stream=stream)
+            rec(ev[3] if ev else None)
+            return
         for t in tensors:
             st = roi.NoiseState(0, s, t["id"], 1.0, 0)
             rec(ev[0] if ev else None)

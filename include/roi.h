@@ -189,6 +189,25 @@ roi_status roi_mask_bwd_adamw(float* logits, const roi_bf16* W, const roi_noise_
                               float* m, float* v, const roi_adamw* opt,
                               float* out_dlogits, roi_bf16* out_dW, void* stream);
 
+/* roi_mask_bwd_adamw for many tensors in one call (one optimizer step, one
+ * (N, M, tau), one stream): the same results, bit for bit, as the single call per
+ * item, with the launches chained as in roi_mask_bwd_batch.  Each item is
+ * validated as the single call; no output (logits, m, v, gradient, dW) may
+ * overlap any other range of any item (ROI_ERR_ALIAS). */
+typedef struct {
+    float* logits;        /* [rows, cols], phi_t on entry, phi_{t+1} on return */
+    const roi_bf16* W;    /* [rows, cols] */
+    const roi_bf16* dWm;  /* [rows, cols] */
+    float* m;             /* [rows, cols], updated */
+    float* v;             /* [rows, cols], updated */
+    float* out_dlogits;   /* nullable, [rows, cols] */
+    roi_bf16* out_dW;     /* nullable, [rows, cols] */
+    int64_t rows, cols;
+    roi_noise_state st;
+} roi_adamw_item;
+roi_status roi_mask_bwd_adamw_batch(const roi_adamw_item* items, int count, int N, int M, float tau,
+                                    const roi_adamw* opt, void* stream);
+
 /* Exponential annealing of tau and lambda (Sec. 4.2.3, Eq. 9), on the host:
  *     x_t = max(x_end, x_init (x_end / x_init)^(t / T_anneal))
  * (the paper: tau 1.0 -> 0.05, lambda 1.0 -> 0.002, T_anneal = 1500).

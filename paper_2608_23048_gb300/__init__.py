@@ -60,6 +60,14 @@ class BwdItem(ctypes.Structure):
                 ("cols", ctypes.c_int64), ("st", NoiseState)]
 
 
+class AdamWItem(ctypes.Structure):
+    """roi_adamw_item: one tensor of roi_mask_bwd_adamw_batch."""
+    _fields_ = [("logits", ctypes.c_void_p), ("W", ctypes.c_void_p), ("dWm", ctypes.c_void_p),
+                ("m", ctypes.c_void_p), ("v", ctypes.c_void_p), ("out_dlogits", ctypes.c_void_p),
+                ("out_dW", ctypes.c_void_p), ("rows", ctypes.c_int64), ("cols", ctypes.c_int64),
+                ("st", NoiseState)]
+
+
 _LIB = None
 _P = ctypes.c_void_p
 
@@ -90,6 +98,7 @@ def lib() -> ctypes.CDLL:
     L.roi_masked_linear_workspace_size.restype = ctypes.c_size_t
     L.roi_mask_fwd_batch.argtypes = [ctypes.POINTER(FwdItem), i32, i32, i32, f32, _P]
     L.roi_mask_bwd_batch.argtypes = [ctypes.POINTER(BwdItem), i32, i32, i32, f32, _P]
+    L.roi_mask_bwd_adamw_batch.argtypes = [ctypes.POINTER(AdamWItem), i32, i32, i32, f32, ctypes.POINTER(AdamW), _P]
     L.roi_anneal.argtypes = [f32, f32, u32, u32]
     L.roi_anneal.restype = f32
     L.roi_hard_mask_export.argtypes = [_P, i32, i32, i64, i64, _P, _P, _P, _P]
@@ -103,7 +112,8 @@ def lib() -> ctypes.CDLL:
     for name in ("roi_mask_fwd", "roi_mask_fwd_ex", "roi_mask_bwd", "roi_hard_mask_export", "roi_device_status",
                  "roi_noise_words", "roi_gumbel_noise", "roi_mask_fwd_st", "roi_mask_bwd_st",
                  "roi_export_compressed_2of4", "roi_mask_bwd_adamw", "roi_masked_linear_fwd",
-                 "roi_masked_linear_fwd_noalloc", "roi_mask_fwd_batch", "roi_mask_bwd_batch"):
+                 "roi_masked_linear_fwd_noalloc", "roi_mask_fwd_batch", "roi_mask_bwd_batch",
+                 "roi_mask_bwd_adamw_batch"):
         getattr(L, name).restype = i32
     _LIB = L
     return L
@@ -205,6 +215,31 @@ def make_bwd_items(items):
         st = state if isinstance(state, NoiseState) else NoiseState(*state)
         arr[k] = BwdItem(_addr(logits), _addr(W), _addr(dWm), _addr(out_dlogits), _addr(out_dW), rows, cols, st)
     return arr
+
+
+def make_adamw_items(items):
+    """ctypes array of AdamWItem from (logits, W, state, dWm, m, v, out_dlogits, out_dW) tuples."""
+    import torch
+    arr = (AdamWItem * len(items))()
+    for k, (logits, W, state, dWm, m, v, out_dlogits, out_dW) in enumerate(items):
+        rows, cols = logits.shape
+        _check_tensor(logits, "logits", torch.float32)
+        for name, t, dt in (("W", W, torch.bfloat16), ("dWm", dWm, torch.bfloat16), ("m", m, torch.float32),
+                            ("v", v, torch.float32), ("out_dlogits", out_dlogits, torch.float32),
+                            ("out_dW", out_dW, torch.bfloat16)):
+            _check_tensor(t, name, dt, (rows, cols))
+        st = state if isinstance(state, NoiseState) else NoiseState(*state)
+        arr[k] = AdamWItem(_addr(logits), _addr(W), _addr(dWm), _addr(m), _addr(v), _addr(out_dlogits),
+                           _addr(out_dW), rows, cols, st)
+    return arr
+
+
+def roi_mask_bwd_adamw_batch(items, N, M, tau, opt: AdamW, stream=None):
+    """Backward fused with the logits' AdamW step for many tensors (AdamWItem array from
+    make_adamw_items, or a list of (logits, W, state, dWm, m, v, out_dlogits, out_dW) tuples)."""
+    arr = items if isinstance(items, ctypes.Array) else make_adamw_items(items)
+    s = lib().roi_mask_bwd_adamw_batch(arr, len(arr), int(N), int(M), float(tau), ctypes.byref(opt), _stream(stream))
+    _raise(s, "roi_mask_bwd_adamw_batch")
 
 
 def roi_mask_fwd_batch(items, N, M, tau, stream=None):

@@ -355,29 +355,99 @@ roi_status roi_mask_bwd_st(const float* logits, const roi_bf16* W, const roi_noi
                   out_dW, nullptr, stream);
 }
 
-roi_status roi_mask_bwd_adamw(float* logits, const roi_bf16* W, const roi_noise_state* st, int N, int M,
-                              const roi_bf16* dWm, float tau, int64_t rows, int64_t cols, float* m, float* v,
-                              const roi_adamw* opt, float* out_dlogits, roi_bf16* out_dW, void* stream) {
+// Checks the optimizer settings and forms the step's constants, rounded to float
+// as the float32 statement of the step forms them.
+static roi_status adamw_constants(const roi_adamw* opt, AdamW* out) {
   if (opt == nullptr) return ROI_ERR_NULL;
   const bool ok = std::isfinite(opt->lr) && opt->lr >= 0.0f && opt->beta1 >= 0.0f && opt->beta1 < 1.0f &&
                   opt->beta2 >= 0.0f && opt->beta2 < 1.0f && finite_positive(opt->eps) &&
                   std::isfinite(opt->weight_decay) && opt->weight_decay >= 0.0f && opt->t >= 1;
   if (!ok) return ROI_ERR_OPT;
+  out->b1 = opt->beta1;
+  out->omb1 = 1.0f - opt->beta1;
+  out->b2 = opt->beta2;
+  out->omb2 = 1.0f - opt->beta2;
+  out->eps = opt->eps;
+  out->decay = 1.0f - opt->lr * opt->weight_decay;
+  const double t = static_cast<double>(opt->t);
+  out->step = static_cast<float>(static_cast<double>(opt->lr) / (1.0 - std::pow(static_cast<double>(opt->beta1), t)));
+  out->r = static_cast<float>(1.0 / std::sqrt(1.0 - std::pow(static_cast<double>(opt->beta2), t)));
+  return ROI_OK;
+}
+
+roi_status roi_mask_bwd_adamw(float* logits, const roi_bf16* W, const roi_noise_state* st, int N, int M,
+                              const roi_bf16* dWm, float tau, int64_t rows, int64_t cols, float* m, float* v,
+                              const roi_adamw* opt, float* out_dlogits, roi_bf16* out_dW, void* stream) {
   FusedAdamW fo;
+  const roi_status s = adamw_constants(opt, &fo.opt);
+  if (s != ROI_OK) return s;
   fo.phi = logits;
   fo.m = m;
   fo.v = v;
-  // constants rounded to float as the float32 statement of the step forms them
-  fo.opt.b1 = opt->beta1;
-  fo.opt.omb1 = 1.0f - opt->beta1;
-  fo.opt.b2 = opt->beta2;
-  fo.opt.omb2 = 1.0f - opt->beta2;
-  fo.opt.eps = opt->eps;
-  fo.opt.decay = 1.0f - opt->lr * opt->weight_decay;
-  const double t = static_cast<double>(opt->t);
-  fo.opt.step = static_cast<float>(static_cast<double>(opt->lr) / (1.0 - std::pow(static_cast<double>(opt->beta1), t)));
-  fo.opt.r = static_cast<float>(1.0 / std::sqrt(1.0 - std::pow(static_cast<double>(opt->beta2), t)));
   return mask_bwd(logits, W, st, N, M, dWm, nullptr, tau, rows, cols, out_dlogits, out_dW, &fo, stream);
+}
+
+roi_status roi_mask_bwd_adamw_batch(const roi_adamw_item* items, int count, int N, int M, float tau,
+                                    const roi_adamw* opt, void* stream) {
+  if (count < 0) return ROI_ERR_SHAPE;
+  if (count > 0 && items == nullptr) return ROI_ERR_NULL;
+  AdamW k;
+  roi_status s = adamw_constants(opt, &k);
+  if (s != ROI_OK) return s;
+  s = check_common(N, M, tau, 0, M);
+  if (s != ROI_OK) return s;
+  std::vector<Tagged> ranges;
+  ranges.reserve(size_t(count) * 7);
+  for (int i = 0; i < count; ++i) {
+    const roi_adamw_item& it = items[i];
+    s = check_common(N, M, tau, it.rows, it.cols);
+    if (s != ROI_OK) return s;
+    if (it.st.row_offset < 0) return ROI_ERR_SHAPE;
+    if (!finite_positive(it.st.lambda)) return ROI_ERR_TAU;
+    if (it.rows == 0) continue;
+    if (it.logits == nullptr || it.W == nullptr || it.dWm == nullptr || it.m == nullptr || it.v == nullptr)
+      return ROI_ERR_NULL;
+    if (!aligned16(it.logits) || !aligned16(it.W) || !aligned16(it.dWm) || !aligned16(it.m) || !aligned16(it.v) ||
+        !aligned16(it.out_dlogits) || !aligned16(it.out_dW))
+      return ROI_ERR_ALIGN;
+    const int64_t E = it.rows * it.cols;
+    add_range(ranges, it.W, uint64_t(E) * 2, false);
+    add_range(ranges, it.dWm, uint64_t(E) * 2, false);
+    add_range(ranges, it.logits, uint64_t(E) * 4, true);  // read and written
+    add_range(ranges, it.m, uint64_t(E) * 4, true);
+    add_range(ranges, it.v, uint64_t(E) * 4, true);
+    add_range(ranges, it.out_dlogits, uint64_t(E) * 4, true);
+    add_range(ranges, it.out_dW, uint64_t(E) * 2, true);
+  }
+  if (batch_alias(ranges)) return ROI_ERR_ALIAS;
+  if (ranges.empty()) return ROI_OK;
+  unsigned int* status = status_word();
+  if (status == nullptr) return ROI_ERR_CUDA;
+  std::vector<BwdCall> calls;
+  calls.reserve(size_t(count));
+  for (int i = 0; i < count; ++i) {
+    const roi_adamw_item& it = items[i];
+    if (it.rows == 0) continue;
+    BwdCall c{};
+    c.phi = it.logits;
+    c.W = it.W;
+    c.dWm = it.dWm;
+    c.dphi = it.out_dlogits;
+    c.dW = it.out_dW;
+    c.phi_out = it.logits;
+    c.m = it.m;
+    c.v = it.v;
+    c.opt = k;
+    c.E = it.rows * it.cols;
+    c.N = N;
+    c.M = M;
+    c.tau = tau;
+    c.np = make_noise(it.st, it.cols);
+    c.status = status;
+    c.stream = static_cast<cudaStream_t>(stream);
+    calls.push_back(c);
+  }
+  return finish(launch_bwd_batch(calls.data(), int(calls.size())));
 }
 
 float roi_anneal(float init, float end, uint32_t t, uint32_t T_anneal) {

@@ -470,14 +470,14 @@ int launch_tiles(const BwdArgs& a, const BwdOptArgs& o, cudaStream_t stream, boo
 template <int N, int M>
 int launch_nm(const BwdArgs& a, const BwdOptArgs& o, cudaStream_t stream, bool pdl = false) {
   const bool t1 = a.tau == 1.0f;
-  if (pdl && o.phi_out == nullptr && !(a.hard_in != nullptr && a.dW != nullptr))
-    return t1 ? launch_tiles<N, M, true, false, false>(a, o, stream, true)
-              : launch_tiles<N, M, false, false, false>(a, o, stream, true);
   if (o.phi_out != nullptr)
-    return t1 ? launch_tiles<N, M, true, false, true>(a, o, stream) : launch_tiles<N, M, false, false, true>(a, o, stream);
+    return t1 ? launch_tiles<N, M, true, false, true>(a, o, stream, pdl)
+              : launch_tiles<N, M, false, false, true>(a, o, stream, pdl);
   if (a.hard_in != nullptr && a.dW != nullptr)
-    return t1 ? launch_tiles<N, M, true, true, false>(a, o, stream) : launch_tiles<N, M, false, true, false>(a, o, stream);
-  return t1 ? launch_tiles<N, M, true, false, false>(a, o, stream) : launch_tiles<N, M, false, false, false>(a, o, stream);
+    return t1 ? launch_tiles<N, M, true, true, false>(a, o, stream, pdl)
+              : launch_tiles<N, M, false, true, false>(a, o, stream, pdl);
+  return t1 ? launch_tiles<N, M, true, false, false>(a, o, stream, pdl)
+            : launch_tiles<N, M, false, false, false>(a, o, stream, pdl);
 }
 
 }  // namespace
@@ -519,14 +519,14 @@ int launch_bwd_impl(const BwdCall& c, bool pdl) {
 int launch_bwd(const BwdCall& c) { return launch_bwd_impl(c, false); }
 
 // As launch_fwd_batch: the tensors are independent, so from the second one on the
-// plain tile kernels are launched with programmatic stream serialization.
+// tile kernels (plain or fused with AdamW) are launched with programmatic stream
+// serialization.
 int launch_bwd_batch(const BwdCall* calls, int count) {
   int launched = 0;
   bool prev_tiled = false;
   for (int i = 0; i < count; ++i) {
     const BwdCall& c = calls[i];
-    const bool tiled = ((c.N == 2 && c.M == 4) || (c.N == 4 && c.M == 8) || (c.N == 2 && c.M == 8)) &&
-                       c.phi_out == nullptr && c.hard_in == nullptr;
+    const bool tiled = (c.N == 2 && c.M == 4) || (c.N == 4 && c.M == 8) || (c.N == 2 && c.M == 8);
     const int r = launch_bwd_impl(c, tiled && prev_tiled);
     if (r < 0) return -1;
     launched += r;

@@ -155,6 +155,16 @@ def test_validation_codes(L):
         return L.roi_mask_bwd_batch(arr, len(its), N, M, 1.0, None)
     assert bbatch(bitem(dl=0)) == 1 and bbatch(bitem(dW=E + 2)) == 5
     assert bbatch(bitem(), bitem(logits=0x60000000, W=0x61000000, dWm=0x62000000, dl=B + 16)) == 6
+    # AdamW batch: settings first, then every item; logits, m, v are outputs
+    def aitem(logits=A, W=B, dWm=C, m=D, v=E, dl=None, rows=4, cols=8):
+        return roi.AdamWItem(logits, W, dWm, m, v, dl, None, rows, cols, roi.NoiseState(0, 0, 0, 1.0, 0))
+    def abatch(*its, o=opt):
+        arr = (roi.AdamWItem * len(its))(*its)
+        return L.roi_mask_bwd_adamw_batch(arr, len(its), 2, 4, 1.0, ctypes.byref(o) if o is not None else None, None)
+    assert abatch(aitem(), o=None) == 1 and abatch(aitem(), o=bad) == 9
+    assert abatch(aitem(m=0)) == 1 and abatch(aitem(v=E + 4)) == 5
+    assert abatch(aitem(), aitem(logits=0x60000000, W=0x61000000, dWm=0x62000000, m=0x63000000, v=D + 64)) == 6
+    assert abatch(aitem(rows=0, logits=0, W=0, dWm=0, m=0, v=0)) == 0
     for s in range(10):
         assert L.roi_status_string(s)
 

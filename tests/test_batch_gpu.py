@@ -177,3 +177,35 @@ def test_work_queued_after_a_batch_sees_every_item(roi):
             assert not bool(nan_dphi)
             again = torch.stack([o["Wm"].float().sum() for o in res])
             assert torch.equal(sums, again)
+
+
+def test_adamw_batch_equals_single_calls(roi):
+    """roi_mask_bwd_adamw_batch: logits, moments, gradients and dW after the step equal
+    the single calls' bit for bit (2:4 and 4:8, mixed shapes and noise states)."""
+    import torch
+    for N, M, tau in ((2, 4, 1.0), (4, 8, 0.5)):
+        shapes = [(r, c) for r, c in SHAPES if c % M == 0][:6]
+        ts = make_set(shapes, 70 + M)
+        opt = roi.AdamW(1e-3, 0.9, 0.95, 1e-8, 0.05, 4)
+        def state():
+            out = []
+            for k, t in enumerate(ts):
+                g = torch.Generator(device="cuda").manual_seed(k)
+                out.append({"phi": t["phi"].clone(),
+                            "m": 1e-3 * torch.randn(t["phi"].shape, generator=g, device="cuda"),
+                            "v": 1e-6 * torch.rand(t["phi"].shape, generator=g, device="cuda"),
+                            "dphi": torch.empty_like(t["phi"]),
+                            "dW": torch.empty_like(t["W"]) if k % 2 else None})
+            return out
+        single, batch = state(), state()
+        for t, s_ in zip(ts, single):
+            roi.roi_mask_bwd_adamw(s_["phi"], t["W"], t["st"], N, M, t["dWm"], tau, s_["m"], s_["v"], opt,
+                                   s_["dphi"], s_["dW"])
+        roi.roi_mask_bwd_adamw_batch([(b["phi"], t["W"], t["st"], t["dWm"], b["m"], b["v"], b["dphi"], b["dW"])
+                                      for t, b in zip(ts, batch)], N, M, tau, opt)
+        roi.roi_device_status()
+        for a, b in zip(single, batch):
+            for k in ("phi", "m", "v", "dphi"):
+                assert torch.equal(a[k].view(torch.int32), b[k].view(torch.int32)), k
+            if a["dW"] is not None:
+                assert torch.equal(a["dW"].view(torch.int16), b["dW"].view(torch.int16))
