@@ -590,6 +590,11 @@ def run_variant(args):
                      meta=torch.empty(rows * cols // 32, dtype=torch.int32, device=dev))
         tensors.append(t)
     stream = torch.cuda.Stream(device=dev)
+    if args.op == "st":
+        st_fwd = roi.make_fwd_items([(t["phi"], t["W"], roi.NoiseState(0, 0, t["id"], 1.0, 0), t["Wm"], None,
+                                      t["hard"]) for t in tensors])
+        st_bwd = roi.make_bwd_st_items([(t["phi"], t["W"], roi.NoiseState(0, 0, t["id"], 1.0, 0), t["dWm"], t["hard"],
+                                         t["dphi"], t["dW"]) for t in reversed(tensors)])
     if args.op == "adamw":
         adamw_fwd = roi.make_fwd_items([(t["phi"], t["W"], roi.NoiseState(0, 0, t["id"], 1.0, 0), t["Wm"], None,
                                          t["hard"]) for t in tensors])
@@ -601,6 +606,17 @@ def run_variant(args):
             if ev is not None:
                 lst.append(torch.cuda.Event(enable_timing=True))
                 lst[-1].record(stream)
+        if args.op == "st" and not args.per_tensor:
+            for arr in (st_fwd, st_bwd):
+                for k in range(len(arr)):
+                    arr[k].st.step = s
+            rec(ev[0] if ev else None)
+            roi.roi_mask_fwd_st_batch(st_fwd, N, M, tau, stream=stream)
+            rec(ev[1] if ev else None)
+            rec(ev[2] if ev else None)
+            roi.roi_mask_bwd_st_batch(st_bwd, N, M, tau, stream=stream)
+            rec(ev[3] if ev else None)
+            return
         if args.op == "adamw" and not args.per_tensor:
             # the training step's two calls: every forward, then every backward fused
             # with the logits' AdamW step (chained launches)

@@ -214,6 +214,23 @@ roi_status roi_mask_bwd_adamw_batch(const roi_adamw_item* items, int count, int 
  * init, end > 0; T_anneal == 0 gives end. */
 float roi_anneal(float init, float end, uint32_t t, uint32_t T_anneal);
 
+/* The straight-through pair for many tensors in one call (items as for
+ * roi_mask_fwd_batch; for the backward, each item adds the forward's hard bits,
+ * needed when out_dW is given): the same results, bit for bit, as the single
+ * straight-through calls per item, launches chained as in roi_mask_fwd_batch. */
+typedef struct {
+    const float* logits;  /* [rows, cols] */
+    const roi_bf16* W;    /* [rows, cols] */
+    const roi_bf16* dWm;  /* [rows, cols] */
+    const uint32_t* hard; /* the forward's out_hard; nullable when out_dW is NULL */
+    float* out_dlogits;   /* [rows, cols], overwritten */
+    roi_bf16* out_dW;     /* nullable, [rows, cols] */
+    int64_t rows, cols;
+    roi_noise_state st;
+} roi_bwd_st_item;
+roi_status roi_mask_fwd_st_batch(const roi_fwd_item* items, int count, int N, int M, float tau, void* stream);
+roi_status roi_mask_bwd_st_batch(const roi_bwd_st_item* items, int count, int N, int M, float tau, void* stream);
+
 /* Compressed 2:4 export for semi-structured sparse inference (the deployment the
  * paper targets, Sec. 1 and the Throughput appendix; it gives no format, so this
  * is the library's): the deployment mask argtop_2(phi) of every group of four

@@ -68,6 +68,13 @@ class AdamWItem(ctypes.Structure):
                 ("st", NoiseState)]
 
 
+class BwdStItem(ctypes.Structure):
+    """roi_bwd_st_item: one tensor of roi_mask_bwd_st_batch."""
+    _fields_ = [("logits", ctypes.c_void_p), ("W", ctypes.c_void_p), ("dWm", ctypes.c_void_p),
+                ("hard", ctypes.c_void_p), ("out_dlogits", ctypes.c_void_p), ("out_dW", ctypes.c_void_p),
+                ("rows", ctypes.c_int64), ("cols", ctypes.c_int64), ("st", NoiseState)]
+
+
 _LIB = None
 _P = ctypes.c_void_p
 
@@ -98,6 +105,8 @@ def lib() -> ctypes.CDLL:
     L.roi_masked_linear_workspace_size.restype = ctypes.c_size_t
     L.roi_mask_fwd_batch.argtypes = [ctypes.POINTER(FwdItem), i32, i32, i32, f32, _P]
     L.roi_mask_bwd_batch.argtypes = [ctypes.POINTER(BwdItem), i32, i32, i32, f32, _P]
+    L.roi_mask_fwd_st_batch.argtypes = [ctypes.POINTER(FwdItem), i32, i32, i32, f32, _P]
+    L.roi_mask_bwd_st_batch.argtypes = [ctypes.POINTER(BwdStItem), i32, i32, i32, f32, _P]
     L.roi_mask_bwd_adamw_batch.argtypes = [ctypes.POINTER(AdamWItem), i32, i32, i32, f32, ctypes.POINTER(AdamW), _P]
     L.roi_anneal.argtypes = [f32, f32, u32, u32]
     L.roi_anneal.restype = f32
@@ -113,7 +122,7 @@ def lib() -> ctypes.CDLL:
                  "roi_noise_words", "roi_gumbel_noise", "roi_mask_fwd_st", "roi_mask_bwd_st",
                  "roi_export_compressed_2of4", "roi_mask_bwd_adamw", "roi_masked_linear_fwd",
                  "roi_masked_linear_fwd_noalloc", "roi_mask_fwd_batch", "roi_mask_bwd_batch",
-                 "roi_mask_bwd_adamw_batch"):
+                 "roi_mask_bwd_adamw_batch", "roi_mask_fwd_st_batch", "roi_mask_bwd_st_batch"):
         getattr(L, name).restype = i32
     _LIB = L
     return L
@@ -240,6 +249,39 @@ def roi_mask_bwd_adamw_batch(items, N, M, tau, opt: AdamW, stream=None):
     arr = items if isinstance(items, ctypes.Array) else make_adamw_items(items)
     s = lib().roi_mask_bwd_adamw_batch(arr, len(arr), int(N), int(M), float(tau), ctypes.byref(opt), _stream(stream))
     _raise(s, "roi_mask_bwd_adamw_batch")
+
+
+def make_bwd_st_items(items):
+    """ctypes array of BwdStItem from (logits, W, state, dWm, hard, out_dlogits, out_dW) tuples."""
+    import torch
+    arr = (BwdStItem * len(items))()
+    for k, (logits, W, state, dWm, hard, out_dlogits, out_dW) in enumerate(items):
+        rows, cols = logits.shape
+        _check_tensor(logits, "logits", torch.float32)
+        _check_tensor(W, "W", torch.bfloat16, (rows, cols))
+        _check_tensor(dWm, "dWm", torch.bfloat16, (rows, cols))
+        _check_tensor(hard, "hard", torch.int32, (hard_words(rows, cols),))
+        _check_tensor(out_dlogits, "out_dlogits", torch.float32, (rows, cols))
+        _check_tensor(out_dW, "out_dW", torch.bfloat16, (rows, cols))
+        st = state if isinstance(state, NoiseState) else NoiseState(*state)
+        arr[k] = BwdStItem(_addr(logits), _addr(W), _addr(dWm), _addr(hard), _addr(out_dlogits), _addr(out_dW),
+                           rows, cols, st)
+    return arr
+
+
+def roi_mask_fwd_st_batch(items, N, M, tau, stream=None):
+    """Straight-through forward of many tensors (items as for roi_mask_fwd_batch)."""
+    arr = items if isinstance(items, ctypes.Array) else make_fwd_items(items)
+    s = lib().roi_mask_fwd_st_batch(arr, len(arr), int(N), int(M), float(tau), _stream(stream))
+    _raise(s, "roi_mask_fwd_st_batch")
+
+
+def roi_mask_bwd_st_batch(items, N, M, tau, stream=None):
+    """Straight-through backward of many tensors (BwdStItem array from make_bwd_st_items,
+    or a list of (logits, W, state, dWm, hard, out_dlogits, out_dW) tuples)."""
+    arr = items if isinstance(items, ctypes.Array) else make_bwd_st_items(items)
+    s = lib().roi_mask_bwd_st_batch(arr, len(arr), int(N), int(M), float(tau), _stream(stream))
+    _raise(s, "roi_mask_bwd_st_batch")
 
 
 def roi_mask_fwd_batch(items, N, M, tau, stream=None):

@@ -155,7 +155,8 @@ static roi_status mask_fwd(const float* logits, const roi_bf16* W, int N, int M,
   return finish(launch_fwd(c));
 }
 
-roi_status roi_mask_fwd_batch(const roi_fwd_item* items, int count, int N, int M, float tau, void* stream) {
+static roi_status fwd_batch(const roi_fwd_item* items, int count, int N, int M, float tau, bool straight_through,
+                            void* stream) {
   if (count < 0) return ROI_ERR_SHAPE;
   if (count > 0 && items == nullptr) return ROI_ERR_NULL;
   roi_status s = check_common(N, M, tau, 0, M);
@@ -195,7 +196,7 @@ roi_status roi_mask_fwd_batch(const roi_fwd_item* items, int count, int N, int M
     c.Wm = it.out_Wm;
     c.soft = it.out_soft;
     c.hard = it.out_hard;
-    c.st = false;
+    c.st = straight_through;
     c.E = it.rows * it.cols;
     c.N = N;
     c.M = M;
@@ -206,6 +207,70 @@ roi_status roi_mask_fwd_batch(const roi_fwd_item* items, int count, int N, int M
     calls.push_back(c);
   }
   return finish(launch_fwd_batch(calls.data(), int(calls.size())));
+}
+
+roi_status roi_mask_fwd_batch(const roi_fwd_item* items, int count, int N, int M, float tau, void* stream) {
+  return fwd_batch(items, count, N, M, tau, false, stream);
+}
+
+roi_status roi_mask_fwd_st_batch(const roi_fwd_item* items, int count, int N, int M, float tau, void* stream) {
+  return fwd_batch(items, count, N, M, tau, true, stream);
+}
+
+roi_status roi_mask_bwd_st_batch(const roi_bwd_st_item* items, int count, int N, int M, float tau, void* stream) {
+  if (count < 0) return ROI_ERR_SHAPE;
+  if (count > 0 && items == nullptr) return ROI_ERR_NULL;
+  roi_status s = check_common(N, M, tau, 0, M);
+  if (s != ROI_OK) return s;
+  std::vector<Tagged> ranges;
+  ranges.reserve(size_t(count) * 6);
+  for (int i = 0; i < count; ++i) {
+    const roi_bwd_st_item& it = items[i];
+    s = check_common(N, M, tau, it.rows, it.cols);
+    if (s != ROI_OK) return s;
+    if (it.st.row_offset < 0) return ROI_ERR_SHAPE;
+    if (!finite_positive(it.st.lambda)) return ROI_ERR_TAU;
+    if (it.rows == 0) continue;
+    if (it.logits == nullptr || it.W == nullptr || it.dWm == nullptr || it.out_dlogits == nullptr ||
+        (it.out_dW != nullptr && it.hard == nullptr))
+      return ROI_ERR_NULL;
+    if (!aligned16(it.logits) || !aligned16(it.W) || !aligned16(it.dWm) || !aligned16(it.hard) ||
+        !aligned16(it.out_dlogits) || !aligned16(it.out_dW))
+      return ROI_ERR_ALIGN;
+    const int64_t E = it.rows * it.cols;
+    add_range(ranges, it.logits, uint64_t(E) * 4, false);
+    add_range(ranges, it.W, uint64_t(E) * 2, false);
+    add_range(ranges, it.dWm, uint64_t(E) * 2, false);
+    add_range(ranges, it.hard, uint64_t((E + 31) / 32) * 4, false);
+    add_range(ranges, it.out_dlogits, uint64_t(E) * 4, true);
+    add_range(ranges, it.out_dW, uint64_t(E) * 2, true);
+  }
+  if (batch_alias(ranges)) return ROI_ERR_ALIAS;
+  if (ranges.empty()) return ROI_OK;
+  unsigned int* status = status_word();
+  if (status == nullptr) return ROI_ERR_CUDA;
+  std::vector<BwdCall> calls;
+  calls.reserve(size_t(count));
+  for (int i = 0; i < count; ++i) {
+    const roi_bwd_st_item& it = items[i];
+    if (it.rows == 0) continue;
+    BwdCall c{};
+    c.phi = it.logits;
+    c.W = it.W;
+    c.dWm = it.dWm;
+    c.dphi = it.out_dlogits;
+    c.dW = it.out_dW;
+    c.hard_in = it.out_dW != nullptr ? it.hard : nullptr;
+    c.E = it.rows * it.cols;
+    c.N = N;
+    c.M = M;
+    c.tau = tau;
+    c.np = make_noise(it.st, it.cols);
+    c.status = status;
+    c.stream = static_cast<cudaStream_t>(stream);
+    calls.push_back(c);
+  }
+  return finish(launch_bwd_batch(calls.data(), int(calls.size())));
 }
 
 roi_status roi_mask_bwd_batch(const roi_bwd_item* items, int count, int N, int M, float tau, void* stream) {

@@ -165,6 +165,13 @@ def test_validation_codes(L):
     assert abatch(aitem(m=0)) == 1 and abatch(aitem(v=E + 4)) == 5
     assert abatch(aitem(), aitem(logits=0x60000000, W=0x61000000, dWm=0x62000000, m=0x63000000, v=D + 64)) == 6
     assert abatch(aitem(rows=0, logits=0, W=0, dWm=0, m=0, v=0)) == 0
+    # straight-through batches: dW needs the forward's bits
+    def sitem(hard=None, dW=E, dl=D, rows=4, cols=8):
+        return roi.BwdStItem(A, B, C, hard, dl, dW, rows, cols, roi.NoiseState(0, 0, 0, 1.0, 0))
+    sarr = lambda *its: (roi.BwdStItem * len(its))(*its)
+    assert L.roi_mask_bwd_st_batch(sarr(sitem()), 1, 2, 4, 1.0, None) == 1
+    assert L.roi_mask_bwd_st_batch(sarr(sitem(hard=0x64000004)), 1, 2, 4, 1.0, None) == 5
+    assert L.roi_mask_fwd_st_batch(None, 1, 2, 4, 1.0, None) == 1
     for s in range(10):
         assert L.roi_status_string(s)
 

@@ -209,3 +209,24 @@ def test_adamw_batch_equals_single_calls(roi):
                 assert torch.equal(a[k].view(torch.int32), b[k].view(torch.int32)), k
             if a["dW"] is not None:
                 assert torch.equal(a["dW"].view(torch.int16), b["dW"].view(torch.int16))
+
+
+def test_straight_through_batch_equals_single_calls(roi):
+    import torch
+    for N, M, tau in ((2, 4, 1.0), (4, 8, 0.5)):
+        shapes = [(r, c) for r, c in SHAPES if c % M == 0][:6]
+        ts = make_set(shapes, 50 + M)
+        res = []
+        for k, t in enumerate(ts):
+            o = outputs(roi, t, False, True, True)
+            roi.roi_mask_fwd_st(t["phi"], t["W"], N, M, tau, t["st"], o["Wm"], None, o["hard"])
+            roi.roi_mask_bwd_st(t["phi"], t["W"], t["st"], N, M, t["dWm"], o["hard"], tau, o["dphi"], o["dW"])
+            res.append(o)
+        bat = [outputs(roi, t, False, True, True) for t in ts]
+        roi.roi_mask_fwd_st_batch([(t["phi"], t["W"], t["st"], o["Wm"], None, o["hard"]) for t, o in zip(ts, bat)],
+                                  N, M, tau)
+        roi.roi_mask_bwd_st_batch([(t["phi"], t["W"], t["st"], t["dWm"], o["hard"], o["dphi"], o["dW"])
+                                   for t, o in zip(ts, bat)], N, M, tau)
+        roi.roi_device_status()
+        for a, b in zip(res, bat):
+            assert_same(a, b)
