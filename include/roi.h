@@ -208,7 +208,7 @@ typedef struct {
 roi_status roi_mask_bwd_adamw_batch(const roi_adamw_item* items, int count, int N, int M, float tau,
                                     const roi_adamw* opt, void* stream);
 
-/* Exponential annealing of tau and lambda (Sec. 4.2.3, Eq. 9), on the host:
+/* Exponential annealing of tau and lambda (Sec. 4.2.3, Eq. 13), on the host:
  *     x_t = max(x_end, x_init (x_end / x_init)^(t / T_anneal))
  * (the paper: tau 1.0 -> 0.05, lambda 1.0 -> 0.002, T_anneal = 1500).
  * init, end > 0; T_anneal == 0 gives end. */

@@ -396,7 +396,7 @@ def decompress_2of4(values, meta, rows, cols):
 
 
 def anneal(init: float, end: float, t, T_anneal: float):
-    """Exponential annealing of tau and lambda (Sec. 4.2.3, Eq. 9):
+    """Exponential annealing of tau and lambda (Sec. 4.2.3, Eq. 13):
     x_t = max(x_end, x_init * (x_end / x_init) ** (t / T_anneal))."""
     t = np.asarray(t, dtype=np.float64)
     return np.maximum(end, init * (end / init) ** (t / T_anneal))

@@ -382,7 +382,7 @@ def roi_mask_bwd_adamw(logits, W, state: NoiseState, N, M, dWm, tau, m, v, opt: 
 
 
 def roi_anneal(init, end, t, T_anneal):
-    """Eq. 9: max(end, init * (end / init) ** (t / T_anneal)), evaluated by the library."""
+    """Eq. 13: max(end, init * (end / init) ** (t / T_anneal)), evaluated by the library."""
     return float(lib().roi_anneal(float(init), float(end), int(t), int(T_anneal)))
 
 

@@ -2,7 +2,7 @@
 
 * AdamW (the optimizer of Sec. 5.1, beta = (0.9, 0.95), weight decay 0.05): three
   steps against torch.optim.AdamW in float64, a library implementation.
-* Eq. 9 annealing: endpoints, the clamp at the final value, the geometric midpoint.
+* Eq. 13 annealing: endpoints, the clamp at the final value, the geometric midpoint.
 """
 import numpy as np
 import pytest
