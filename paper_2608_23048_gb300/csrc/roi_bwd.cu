@@ -505,7 +505,7 @@ int launch_bwd_impl(const BwdCall& c, bool pdl) {
   if (c.N == 2 && c.M == 4) return launch_nm<2, 4>(a, o, c.stream, pdl);
   if (c.N == 4 && c.M == 8) return launch_nm<4, 8>(a, o, c.stream, pdl);
   if (c.N == 2 && c.M == 8) return launch_nm<2, 8>(a, o, c.stream, pdl);
-  if (slice_supported(c.N, c.M)) return launch_slice_bwd(c);
+  if (slice_supported(c.N, c.M)) return launch_slice_bwd(c, pdl);
   const int64_t groups = c.E / c.M;
   int64_t blocks = (groups + 127) / 128;
   const int64_t cap = int64_t(sm_count()) * 16;
@@ -526,7 +526,8 @@ int launch_bwd_batch(const BwdCall* calls, int count) {
   bool prev_tiled = false;
   for (int i = 0; i < count; ++i) {
     const BwdCall& c = calls[i];
-    const bool tiled = (c.N == 2 && c.M == 4) || (c.N == 4 && c.M == 8) || (c.N == 2 && c.M == 8);
+    const bool tiled =
+        (c.N == 2 && c.M == 4) || (c.N == 4 && c.M == 8) || (c.N == 2 && c.M == 8) || slice_supported(c.N, c.M);
     const int r = launch_bwd_impl(c, tiled && prev_tiled);
     if (r < 0) return -1;
     launched += r;

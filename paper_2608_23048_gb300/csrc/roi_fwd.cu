@@ -427,7 +427,7 @@ int launch_fwd_impl(const FwdCall& c, bool pdl) {
   if (c.N == 2 && c.M == 4) return launch_nm<2, 4>(a, c.stream, pdl);
   if (c.N == 4 && c.M == 8) return launch_nm<4, 8>(a, c.stream, pdl);
   if (c.N == 2 && c.M == 8) return launch_nm<2, 8>(a, c.stream, pdl);
-  if (slice_supported(c.N, c.M)) return launch_slice_fwd(c);
+  if (slice_supported(c.N, c.M)) return launch_slice_fwd(c, pdl);
   // generic path
   int launched = 0;
   if (c.hard != nullptr) {
@@ -455,7 +455,8 @@ int launch_fwd_batch(const FwdCall* calls, int count) {
   bool prev_tiled = false;
   for (int i = 0; i < count; ++i) {
     const FwdCall& c = calls[i];
-    const bool tiled = (c.N == 2 && c.M == 4) || (c.N == 4 && c.M == 8) || (c.N == 2 && c.M == 8);
+    const bool tiled =
+        (c.N == 2 && c.M == 4) || (c.N == 4 && c.M == 8) || (c.N == 2 && c.M == 8) || slice_supported(c.N, c.M);
     const int r = launch_fwd_impl(c, tiled && prev_tiled);
     if (r < 0) return -1;
     launched += r;

@@ -88,8 +88,8 @@ int launch_export(const ExportCall& c);
 int launch_export_compressed_2of4(const CompressCall& c);
 // Warp-slice kernels for M = 16, 32 (roi_slice.cu).
 bool slice_supported(int N, int M);
-int launch_slice_fwd(const FwdCall& c);
-int launch_slice_bwd(const BwdCall& c);
+int launch_slice_fwd(const FwdCall& c, bool pdl = false);
+int launch_slice_bwd(const BwdCall& c, bool pdl = false);
 int launch_noise(const NoiseParams& np, int64_t E, uint32_t* words, float* g, cudaStream_t stream);
 
 // Masked linear forward on the tensor cores (roi_linear.cu).

@@ -525,6 +525,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksFwd) roi_slice_fwd_kernel(
   src.esize[0] = 4;
   src.ptr[1] = reinterpret_cast<const uint8_t*>(a.W);
   src.esize[1] = 2;
+  // a batch's next tensor may start on the SMs this launch frees (no-op otherwise)
+  pdl_launch_dependents();
   const bool ok = run_tiles<kThreads, kTile, kStagesFwd, 2>(
       smem, src, a.full_tiles, a.status, [&](const uint8_t* const* stage, int64_t tile) {
         const float* sphi = reinterpret_cast<const float*>(stage[0]);
@@ -547,8 +549,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksFwd) roi_slice_fwd_kernel(
         }
         if (a.hard != nullptr) store_hard_slot_pair(a.hard, e0[0], e0[1], bits[0], bits[1]);
       });
-  if (!ok) return;
-  if (blockIdx.x == gridDim.x - 1) {
+  if (ok && blockIdx.x == gridDim.x - 1) {
     const int64_t t0 = a.full_tiles * kTile;
     const int64_t slots = (a.E - t0) / 4;
     for (int64_t r = 0; r * kThreads < slots; ++r) {
@@ -563,6 +564,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksFwd) roi_slice_fwd_kernel(
       if (a.hard != nullptr) store_hard_slot(a.hard, e0[0], bits[0], active);
     }
   }
+  // the launch completes only after the batch's previous one (stream order)
+  if (blockIdx.x == 0) pdl_wait();
 }
 
 template <int N, int M, bool TAU1>
@@ -575,6 +578,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksBwd<M>) roi_slice_bwd_kern
   src.esize[1] = 2;
   src.ptr[2] = reinterpret_cast<const uint8_t*>(a.dWm);
   src.esize[2] = 2;
+  pdl_launch_dependents();
   const bool ok = run_tiles<kThreads, kTile, kStagesBwd, 3>(
       smem, src, a.full_tiles, a.status, [&](const uint8_t* const* stage, int64_t tile) {
         const float* sphi = reinterpret_cast<const float*>(stage[0]);
@@ -589,8 +593,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksBwd<M>) roi_slice_bwd_kern
 #pragma unroll 1
         for (int j = 0; j < 2; ++j) bwd_slots<N, M, TAU1, float>(pp + j, pw + j, pd + j, e0 + j, true, a);
       });
-  if (!ok) return;
-  if (blockIdx.x == gridDim.x - 1) {
+  if (ok && blockIdx.x == gridDim.x - 1) {
     const int64_t t0 = a.full_tiles * kTile;
     const int64_t slots = (a.E - t0) / 4;
     for (int64_t r = 0; r * kThreads < slots; ++r) {
@@ -604,6 +607,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksBwd<M>) roi_slice_bwd_kern
       bwd_slots<N, M, TAU1, float>(pp, pw, pd, e0, active, a);
     }
   }
+  if (blockIdx.x == 0) pdl_wait();
 }
 
 struct LaunchCache {
@@ -611,7 +615,8 @@ struct LaunchCache {
 };
 
 template <class Kern>
-int launch_persistent(Kern kern, LaunchCache& cache, size_t smem, const SliceArgs& a, cudaStream_t stream) {
+int launch_persistent(Kern kern, LaunchCache& cache, size_t smem, const SliceArgs& a, cudaStream_t stream,
+                      bool pdl) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return -1;
   if (cache.per_sm[dev] == 0) {
@@ -623,35 +628,36 @@ int launch_persistent(Kern kern, LaunchCache& cache, size_t smem, const SliceArg
   }
   const int64_t cap = int64_t(sm_count()) * cache.per_sm[dev];
   const int grid = int(a.full_tiles < 1 ? 1 : (a.full_tiles < cap ? a.full_tiles : cap));
-  kern<<<grid, kThreads, smem, stream>>>(a);
-  return cudaGetLastError() == cudaSuccess ? 1 : -1;
+  return launch_maybe_pdl(kern, grid, kThreads, smem, stream, pdl, a);
 }
 
 template <int N, int M, bool TAU1>
-int slice_fwd(const SliceArgs& a, cudaStream_t stream) {
+int slice_fwd(const SliceArgs& a, cudaStream_t stream, bool pdl) {
   static LaunchCache cache;
-  return launch_persistent(roi_slice_fwd_kernel<N, M, TAU1>, cache, tile_smem_bytes<kTile, kStagesFwd>(6), a, stream);
+  return launch_persistent(roi_slice_fwd_kernel<N, M, TAU1>, cache, tile_smem_bytes<kTile, kStagesFwd>(6), a, stream,
+                           pdl);
 }
 template <int N, int M, bool TAU1>
-int slice_bwd(const SliceArgs& a, cudaStream_t stream) {
+int slice_bwd(const SliceArgs& a, cudaStream_t stream, bool pdl) {
   static LaunchCache cache;
-  return launch_persistent(roi_slice_bwd_kernel<N, M, TAU1>, cache, tile_smem_bytes<kTile, kStagesBwd>(8), a, stream);
+  return launch_persistent(roi_slice_bwd_kernel<N, M, TAU1>, cache, tile_smem_bytes<kTile, kStagesBwd>(8), a, stream,
+                           pdl);
 }
 
 template <int N, int M>
-int slice_fwd_nm(const SliceArgs& a, cudaStream_t stream) {
-  return a.tau == 1.0f ? slice_fwd<N, M, true>(a, stream) : slice_fwd<N, M, false>(a, stream);
+int slice_fwd_nm(const SliceArgs& a, cudaStream_t stream, bool pdl) {
+  return a.tau == 1.0f ? slice_fwd<N, M, true>(a, stream, pdl) : slice_fwd<N, M, false>(a, stream, pdl);
 }
 template <int N, int M>
-int slice_bwd_nm(const SliceArgs& a, cudaStream_t stream) {
-  return a.tau == 1.0f ? slice_bwd<N, M, true>(a, stream) : slice_bwd<N, M, false>(a, stream);
+int slice_bwd_nm(const SliceArgs& a, cudaStream_t stream, bool pdl) {
+  return a.tau == 1.0f ? slice_bwd<N, M, true>(a, stream, pdl) : slice_bwd<N, M, false>(a, stream, pdl);
 }
 
 }  // namespace
 
 bool slice_supported(int N, int M) { return (N == 8 && M == 16) || (N == 16 && M == 32); }
 
-int launch_slice_fwd(const FwdCall& c) {
+int launch_slice_fwd(const FwdCall& c, bool pdl) {
   SliceArgs a{};
   a.phi = c.phi;
   a.W = c.W;
@@ -665,12 +671,12 @@ int launch_slice_fwd(const FwdCall& c) {
   a.inv_tau = 1.0f / c.tau;
   a.np = c.np;
   a.status = c.status;
-  if (c.N == 8 && c.M == 16) return slice_fwd_nm<8, 16>(a, c.stream);
-  if (c.N == 16 && c.M == 32) return slice_fwd_nm<16, 32>(a, c.stream);
+  if (c.N == 8 && c.M == 16) return slice_fwd_nm<8, 16>(a, c.stream, pdl);
+  if (c.N == 16 && c.M == 32) return slice_fwd_nm<16, 32>(a, c.stream, pdl);
   return -1;
 }
 
-int launch_slice_bwd(const BwdCall& c) {
+int launch_slice_bwd(const BwdCall& c, bool pdl) {
   SliceArgs a{};
   a.phi = c.phi;
   a.W = c.W;
@@ -688,8 +694,8 @@ int launch_slice_bwd(const BwdCall& c) {
   a.inv_tau = 1.0f / c.tau;
   a.np = c.np;
   a.status = c.status;
-  if (c.N == 8 && c.M == 16) return slice_bwd_nm<8, 16>(a, c.stream);
-  if (c.N == 16 && c.M == 32) return slice_bwd_nm<16, 32>(a, c.stream);
+  if (c.N == 8 && c.M == 16) return slice_bwd_nm<8, 16>(a, c.stream, pdl);
+  if (c.N == 16 && c.M == 32) return slice_bwd_nm<16, 32>(a, c.stream, pdl);
   return -1;
 }
 

@@ -88,7 +88,8 @@ def assert_same(a, b):
 SHAPES = [(37, 1000), (3, 64), (64, 3584), (512, 256), (1, 32), (129, 2048), (8, 8), (300, 520), (16, 24576)]
 
 
-@pytest.mark.parametrize("N,M,tau", [(2, 4, 1.0), (2, 4, 0.5), (4, 8, 1.0), (4, 8, 0.3), (2, 8, 1.0), (3, 4, 0.8)])
+@pytest.mark.parametrize("N,M,tau", [(2, 4, 1.0), (2, 4, 0.5), (4, 8, 1.0), (4, 8, 0.3), (2, 8, 1.0), (3, 4, 0.8),
+                                     (8, 16, 0.2), (16, 32, 1.0)])
 def test_batch_equals_single_calls(roi, N, M, tau):
     shapes = [(r, c) for r, c in SHAPES if c % M == 0]
     ts = make_set(shapes, 40 + M + int(10 * tau))
