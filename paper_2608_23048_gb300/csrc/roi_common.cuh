@@ -292,12 +292,22 @@ __device__ __forceinline__ void topn_bits4_signs(const F2 (&k)[4], int N, uint32
   }
 }
 
-// M = 8, two groups at once, for groups whose keys are all finite: the N-th
-// largest key of each group comes out of a sorting network (Batcher's odd-even
-// merge sort, 19 compare-exchanges), and member l is selected iff its key is at
-// least that threshold, read off the sign bit of the packed difference.  When
-// the threshold is tied with another member more than N members pass; such a
-// group gets 0xffffffff and the caller re-ranks it with topn_bits<8>.
+// Three-input maximum / minimum (one instruction on sm_100 and later).
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// M = 8, two groups at once, for groups whose keys are all finite: member l is
+// selected iff its key is at least the group's N-th largest key, read off the
+// sign bit of the packed difference.  The N-th largest comes from the two sorted
+// halves: with a_1 >= .. >= a_4 and b_1 >= .. >= b_4 (five compare-exchanges
+// each), the N-th largest of all eight is the largest min(a_i, b_j) over
+// i + j = N (a_0 = b_0 = +inf): some such pair lies within the top N, and of
+// any such pair one member lies outside the top N - 1.  When the threshold is
+// tied with another member more than N members pass; such a group gets
+// 0xffffffff and the caller re-ranks it with topn_bits<8>.
 template <int N>
 __device__ __forceinline__ void topn_bits8_threshold(const F2 (&k)[8], uint32_t (&bits)[2]) {
   static_assert(N >= 1 && N < 8, "1 <= N < 8");
@@ -313,13 +323,22 @@ __device__ __forceinline__ void topn_bits8_threshold(const F2 (&k)[8], uint32_t 
       s[a] = fmaxf(x, y);
       s[b] = fminf(x, y);
     };
-    ce(0, 1), ce(2, 3), ce(4, 5), ce(6, 7);
-    ce(0, 2), ce(1, 3), ce(4, 6), ce(5, 7);
-    ce(1, 2), ce(5, 6);
-    ce(0, 4), ce(1, 5), ce(2, 6), ce(3, 7);
-    ce(2, 4), ce(3, 5);
-    ce(1, 2), ce(3, 4), ce(5, 6);
-    thr[h] = s[N - 1];
+    ce(0, 1), ce(2, 3), ce(0, 2), ce(1, 3), ce(1, 2);  // s[0..3] = a_1..a_4
+    ce(4, 5), ce(6, 7), ce(4, 6), ce(5, 7), ce(5, 6);  // s[4..7] = b_1..b_4
+    float c[5];
+    int nc = 0;
+#pragma unroll
+    for (int i = 0; i <= N; ++i) {
+      const int j = N - i;
+      if (i > 4 || j > 4) continue;
+      c[nc++] = i == 0 ? s[3 + j] : j == 0 ? s[i - 1] : fminf(s[i - 1], s[3 + j]);
+    }
+    float t = c[0];
+    int q = 1;
+#pragma unroll
+    for (; q + 1 < nc; q += 2) t = fmax3(t, c[q], c[q + 1]);
+    if (q < nc) t = fmaxf(t, c[q]);
+    thr[h] = t;
   }
   const F2 t = f2(thr[0], thr[1]);
   uint32_t sg[2][8];
@@ -701,8 +720,12 @@ struct FastGroup {
       exclusive_sums(h, H);
 #pragma unroll
       for (int l = 0; l < M; ++l) {
-        const V mu_l = TAU1 ? mk[l] : vmul(mk[l], itau);
-        b[l] = vfma(mu_l, vsub(vadd(c[l], H[l]), K), b[l]);
+        if constexpr (TAU1) {
+          // b + mu (c + H - K) = (c mu + b) + mu (H - K), and c mu + b is cm
+          b[l] = vfma(mk[l], vsub(H[l], K), cm[l]);
+        } else {
+          b[l] = vfma(vmul(mk[l], itau), vsub(vadd(c[l], H[l]), K), b[l]);
+        }
       }
     };
 #pragma unroll
