@@ -85,9 +85,9 @@ __device__ __forceinline__ float lane_of(V v, int h) {
 
 // Keys (log2 units) of L groups (one per lane of V): logits from the tile stage,
 // noise regenerated four members (one Philox block) at a time.
-template <int M, class V>
-__device__ __forceinline__ void bwd_keys(const float* const* phi_g, const int64_t* e0, const NoiseParams& np,
-                                         V (&kap)[M]) {
+template <int M, class V, bool NARROW = false>
+__device__ __forceinline__ void bwd_keys(const float* const* phi_g, const int64_t* e0, const uint32_t* q0,
+                                         const NoiseParams& np, V (&kap)[M]) {
   constexpr int L = vlanes<V>();
 #pragma unroll
   for (int s = 0; s < M / 4; ++s) {
@@ -97,7 +97,8 @@ __device__ __forceinline__ void bwd_keys(const float* const* phi_g, const int64_
     for (int h = 0; h < L; ++h) {
       const float4 p = reinterpret_cast<const float4*>(phi_g[h])[s];
       ph[h][0] = p.x, ph[h][1] = p.y, ph[h][2] = p.z, ph[h][3] = p.w;
-      const uint4 q = noise_block_q(np, ((np.e_base + uint64_t(e0[h])) >> 2) + s);
+      const uint4 q = NARROW ? noise_block_lo(np, q0[h] + s)
+                             : noise_block_q(np, ((np.e_base + uint64_t(e0[h])) >> 2) + s);
       x[h][0] = q.x, x[h][1] = q.y, x[h][2] = q.z, x[h][3] = q.w;
     }
 #pragma unroll
@@ -140,10 +141,10 @@ __device__ __forceinline__ void bwd_upstream(const uint16_t* const* W_g, const u
 }
 
 // Keys and upstream gradients together, reading each stage word once.
-template <int M, class V>
+template <int M, class V, bool NARROW = false>
 __device__ __forceinline__ void bwd_inputs(const float* const* phi_g, const uint16_t* const* W_g,
-                                           const uint16_t* const* dWm_g, const int64_t* e0, const NoiseParams& np,
-                                           V (&kap)[M], V (&c)[M]) {
+                                           const uint16_t* const* dWm_g, const int64_t* e0, const uint32_t* q0,
+                                           const NoiseParams& np, V (&kap)[M], V (&c)[M]) {
   constexpr int L = vlanes<V>();
 #pragma unroll
   for (int s = 0; s < M / 4; ++s) {
@@ -155,7 +156,8 @@ __device__ __forceinline__ void bwd_inputs(const float* const* phi_g, const uint
       ph[h][0] = p.x, ph[h][1] = p.y, ph[h][2] = p.z, ph[h][3] = p.w;
       unpack4(reinterpret_cast<const uint2*>(W_g[h])[s], w[h]);
       unpack4(reinterpret_cast<const uint2*>(dWm_g[h])[s], dw[h]);
-      const uint4 q = noise_block_q(np, ((np.e_base + uint64_t(e0[h])) >> 2) + s);
+      const uint4 q = NARROW ? noise_block_lo(np, q0[h] + s)
+                             : noise_block_q(np, ((np.e_base + uint64_t(e0[h])) >> 2) + s);
       x[h][0] = q.x, x[h][1] = q.y, x[h][2] = q.z, x[h][3] = q.w;
     }
 #pragma unroll
@@ -181,19 +183,29 @@ __device__ __forceinline__ void bwd_inputs(const float* const* phi_g, const uint
 // whole history stays in registers.  With HIST (M = 8) registers are tight:
 // the keys die after the forward relaxation (a flagged group re-forms them) and
 // the upstream gradients are formed only for the sweep.
-template <int N, int M, bool TAU1, class V, bool HIST = false, bool ST = false, bool OPT = false>
+template <int N, int M, bool TAU1, class V, bool HIST = false, bool ST = false, bool OPT = false,
+          bool NARROW = false>
 __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint16_t* const* W_g,
-                                           const uint16_t* const* dWm_g, const int64_t* e0, const BwdArgs& a,
-                                           const BwdOptArgs& o, V* hist = nullptr) {
+                                           const uint16_t* const* dWm_g, const int64_t* e0, const uint32_t* q0,
+                                           const BwdArgs& a, const BwdOptArgs& o, V* hist = nullptr) {
   constexpr int L = vlanes<V>();
   // straight-through: the forward's hard bits of these groups, loaded now so the
-  // load's latency hides behind the relaxation
+  // load's latency hides behind the relaxation.  With HIST (registers tight) dW,
+  // which needs nothing else, is written at once and the bits die here.
   uint32_t keep[ST ? L : 1][ST ? M / 4 : 1];
   if constexpr (ST) {
 #pragma unroll
     for (int h = 0; h < L; ++h)
 #pragma unroll
       for (int s = 0; s < M / 4; ++s) keep[h][s] = hard4(a.hard_in, e0[h] + 4 * s);
+    if (HIST && a.dW != nullptr) {
+#pragma unroll
+      for (int s = 0; s < M / 4; ++s)
+#pragma unroll
+        for (int h = 0; h < L; ++h)
+          reinterpret_cast<uint2*>(a.dW + e0[h])[s] =
+              keep4(reinterpret_cast<const uint2*>(dWm_g[h])[s], keep[h][s]);
+    }
   }
   // fused optimizer: the moments, fetched now for the epilogue, into registers
   // (M = 4) or into this thread's shared-memory slot `mom` (with HIST)
@@ -228,13 +240,13 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
   V kap[HIST ? 1 : M], c[M], dkv[M];
   if constexpr (HIST) {
     V k[M];
-    bwd_keys<M, V>(phi_g, e0, a.np, k);
+    bwd_keys<M, V, NARROW>(phi_g, e0, q0, a.np, k);
     fg.forward(k, a.inv_tau);
   } else {
-    bwd_inputs<M, V>(phi_g, W_g, dWm_g, e0, a.np, kap, c);
+    bwd_inputs<M, V, NARROW>(phi_g, W_g, dWm_g, e0, q0, a.np, kap, c);
     fg.forward(kap, a.inv_tau);
   }
-  if (a.dW != nullptr) {
+  if (a.dW != nullptr && !(ST && HIST)) {
     // dW = bf16(dWm * S) now, while the relaxation is live anyway (dWm is re-read);
     // straight-through: dWm where the forward's hard mask is set, +0 elsewhere
 #pragma unroll
@@ -285,7 +297,7 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
       if constexpr (HIST) {
         NoiseParams np = a.np;
         asm volatile("" : "+r"(np.k0));
-        bwd_keys<M, float>(phi_g + h, e0 + h, np, k);
+        bwd_keys<M, float>(phi_g + h, e0 + h, nullptr, np, k);
       } else {
 #pragma unroll
         for (int l = 0; l < M; ++l) k[l] = lane_of(kap[l], h);
@@ -338,8 +350,8 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
 }
 
 // One full tile of a tensor (local tile index `tile`), inputs staged in shared
-// memory.
-template <int N, int M, bool TAU1, bool ST, bool OPT>
+// memory.  NARROW: the call's counters are below 2^32 (a.np.narrow).
+template <int N, int M, bool TAU1, bool ST, bool OPT, bool NARROW>
 __device__ __forceinline__ void bwd_tile(const uint8_t* const* stage, int64_t tile, const BwdArgs& a,
                                          const BwdOptArgs& o, uint8_t* smem) {
   using C = Cfg<M>;
@@ -347,6 +359,8 @@ __device__ __forceinline__ void bwd_tile(const uint8_t* const* stage, int64_t ti
   const uint16_t* sW = reinterpret_cast<const uint16_t*>(stage[1]);
   const uint16_t* sdW = reinterpret_cast<const uint16_t*>(stage[2]);
   const int64_t base = tile * C::kTile;
+  // low word of the tile's first counter (uniform); group g adds g M / 4
+  const uint32_t qt = uint32_t((a.np.e_base + uint64_t(base)) >> 2);
 #pragma unroll
   for (int p = 0; p < C::kPairs; ++p) {
     const int g0 = threadIdx.x + 2 * p * C::kThreads, g1 = g0 + C::kThreads;
@@ -354,13 +368,14 @@ __device__ __forceinline__ void bwd_tile(const uint8_t* const* stage, int64_t ti
     const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
     const uint16_t* pd[2] = {sdW + g0 * M, sdW + g1 * M};
     const int64_t e0[2] = {base + g0 * M, base + g1 * M};
+    const uint32_t q0[2] = {qt + uint32_t(g0 * (M / 4)), qt + uint32_t(g1 * (M / 4))};
     if constexpr (M == 4) {
-      bwd_groups<N, M, TAU1, F2, false, ST, OPT>(pp, pw, pd, e0, a, o);
+      bwd_groups<N, M, TAU1, F2, false, ST, OPT, NARROW>(pp, pw, pd, e0, q0, a, o);
     } else {
       // M = 8: the paired step history does not fit the register file; steps
       // 0 .. N-2 go to shared memory behind the tile ring
       F2* hist = reinterpret_cast<F2*>(smem + kHistOffset<M>) + threadIdx.x;
-      bwd_groups<N, M, TAU1, F2, true, ST, OPT>(pp, pw, pd, e0, a, o, hist);
+      bwd_groups<N, M, TAU1, F2, true, ST, OPT, NARROW>(pp, pw, pd, e0, q0, a, o, hist);
     }
   }
 }
@@ -377,7 +392,7 @@ __device__ __forceinline__ void bwd_tail(const BwdArgs& a, const BwdOptArgs& o) 
     const uint16_t* pw[1] = {a.W + t0 + gi * M};
     const uint16_t* pd[1] = {a.dWm + t0 + gi * M};
     const int64_t e0[1] = {t0 + gi * M};
-    bwd_groups<N, M, TAU1, float, false, ST, OPT>(pp, pw, pd, e0, a, o);
+    bwd_groups<N, M, TAU1, float, false, ST, OPT>(pp, pw, pd, e0, nullptr, a, o);
   }
 }
 
@@ -398,7 +413,17 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_
   pdl_launch_dependents();
   const bool ok = run_tiles<C::kThreads, C::kTile, C::kStages, 3>(
       smem, src, a.full_tiles, a.status,
-      [&](const uint8_t* const* stage, int64_t tile) { bwd_tile<N, M, TAU1, ST, OPT>(stage, tile, a, o, smem); });
+      [&](const uint8_t* const* stage, int64_t tile) {
+        // 32-bit counters for M = 4 only (at M = 8 the second copy of the tile body
+        // spills)
+        if constexpr (M == 4) {
+          if (a.np.narrow) {
+            bwd_tile<N, M, TAU1, ST, OPT, true>(stage, tile, a, o, smem);
+            return;
+          }
+        }
+        bwd_tile<N, M, TAU1, ST, OPT, false>(stage, tile, a, o, smem);
+      });
   if (ok && blockIdx.x == gridDim.x - 1) bwd_tail<N, M, TAU1, ST, OPT>(a, o);
   // the launch completes only after the batch's previous one (stream order)
   if (blockIdx.x == 0) pdl_wait();
@@ -501,6 +526,7 @@ int launch_bwd_impl(const BwdCall& c, bool pdl) {
   a.tau = c.tau;
   a.inv_tau = 1.0f / c.tau;
   a.np = c.np;
+  a.np.narrow = counters_narrow(c.np, c.E);
   a.status = c.status;
   if (c.N == 2 && c.M == 4) return launch_nm<2, 4>(a, o, c.stream, pdl);
   if (c.N == 4 && c.M == 8) return launch_nm<4, 8>(a, o, c.stream, pdl);

@@ -129,11 +129,20 @@ struct NoiseParams {
   float inv_lam;         // 1 / lambda
   float l2e_inv_lam;     // log2(e) / lambda: keys in log2 units, t = phi log2(e) / lambda - log2(E)
   uint64_t e_base;       // row_offset * cols: flat index of this call's element 0
+  // every counter of the call is below 2^32 (e_base + E <= 2^34): the tile kernels
+  // then form the counter's low word in 32-bit arithmetic and its high word is 0
+  bool narrow = false;
 };
 
 // The four noise words of block q (elements 4q .. 4q+3).
 __device__ __forceinline__ uint4 noise_block_q(const NoiseParams& np, uint64_t q) {
   return philox4x32_10(make_uint4(uint32_t(q), uint32_t(q >> 32), np.step, np.tensor_id), np.k0, np.k1);
+}
+// Block q of a call whose counters are all below 2^32 (the same words as
+// noise_block_q(np, q)); the high word is the constant 0, so the first two rounds
+// take their other inputs (step, tensor id, key) from kernel parameters.
+__device__ __forceinline__ uint4 noise_block_lo(const NoiseParams& np, uint32_t q) {
+  return philox4x32_10(make_uint4(q, 0u, np.step, np.tensor_id), np.k0, np.k1);
 }
 // Four consecutive noise words for elements e4 .. e4+3 (e4 % 4 == 0).
 __device__ __forceinline__ uint4 noise_block(const NoiseParams& np, uint64_t e4) {
@@ -165,7 +174,8 @@ __device__ __forceinline__ float uniform_from_word(uint32_t x) {
 // ln u = e ln2 + ln m; ln m = 2 atanh(s), s = (m - 1) / (m + 1), |s| < 0.172,
 // 2 atanh(s) = 2s + (2/3)s^3 + (2/5)s^5 + (2/7)s^7 + (2/9)s^9 + O(s^11)
 // (truncation below 2^-28 relative).  m - 1 is exact (Sterbenz).  The Horner
-// chain runs on negated coefficients so the result needs no final negation.
+// chain in s^2 runs on the negated coefficients down to -2, so one product with
+// s gives -ln m (no final negation).
 __device__ __forceinline__ int rounded_exponent(float x) {
   return int(__float_as_uint(x) - 0x3f3504f3u) >> 23;  // 0x3f3504f3: sqrt(1/2)
 }
@@ -183,7 +193,8 @@ __device__ __forceinline__ V neg_log_unit(V u) {
   V q = vfma(s2, vconst<V>(-0.22222222f), vconst<V>(-0.28571429f));
   q = vfma(s2, q, vconst<V>(-0.4f));
   q = vfma(s2, q, vconst<V>(-0.66666667f));
-  const V nlnm = vfma(vmul(s, s2), q, vmul(s, vconst<V>(-2.0f)));  // -ln m
+  q = vfma(s2, q, vconst<V>(-2.0f));
+  const V nlnm = vmul(s, q);  // -ln m
   return vfma(ef, vconst<V>(-kLn2), nlnm);
 }
 
@@ -681,7 +692,10 @@ struct FastGroup {
   // Reverse sweep (requires KEEP): dk = dL/dkappa for c = dL/dS.
   //   abar_l = b_l + (mu_l / tau) (c_l - <c, mu> + H_l - B),
   //   H_l = sum_{i != l} b_i / om_i,  B = sum_i b_i,
-  // with om_i = 1 - mu_i formed as the sum of the other members' mu.
+  // with om_i = 1 - mu_i formed as the sum of the other members' mu.  REUSE (tau = 1):
+  // the update reads c mu + b from the K terms (one operation less per member and
+  // step, one more array live).
+  template <bool REUSE = true>
   __device__ __forceinline__ void backward(const V (&c)[M], float inv_tau, V (&dk)[M]) const {
     static_assert(KEEP, "backward needs the stored steps");
     const V itau = vconst<V>(inv_tau);
@@ -720,9 +734,11 @@ struct FastGroup {
       exclusive_sums(h, H);
 #pragma unroll
       for (int l = 0; l < M; ++l) {
-        if constexpr (TAU1) {
+        if constexpr (TAU1 && REUSE) {
           // b + mu (c + H - K) = (c mu + b) + mu (H - K), and c mu + b is cm
           b[l] = vfma(mk[l], vsub(H[l], K), cm[l]);
+        } else if constexpr (TAU1) {
+          b[l] = vfma(mk[l], vsub(vadd(c[l], H[l]), K), b[l]);
         } else {
           b[l] = vfma(vmul(mk[l], itau), vsub(vadd(c[l], H[l]), K), b[l]);
         }

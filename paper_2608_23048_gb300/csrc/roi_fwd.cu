@@ -54,18 +54,23 @@ __device__ __forceinline__ void load_group(const float* phi_g, const uint16_t* W
 
 // Perturbed keys of L groups (one per lane of V), in log2 units
 // (t = (phi / lambda + g) log2 e), whose first elements have call-flat indices
-// e0[h]; ph[h] holds each group's logits.
-template <int M, class V>
-__device__ __forceinline__ void group_keys(const float (&ph)[vlanes<V>()][M], const int64_t* e0,
+// e0[h]; ph[h] holds each group's logits.  NARROW: the call's counters are below
+// 2^32 and q0[h] holds the low word of group h's first counter.
+template <int M, class V, bool NARROW>
+__device__ __forceinline__ void group_keys(const float (&ph)[vlanes<V>()][M], const int64_t* e0, const uint32_t* q0,
                                            const NoiseParams& np, V (&kap)[M]) {
   constexpr int L = vlanes<V>();
   uint32_t x[L][M];
 #pragma unroll
   for (int h = 0; h < L; ++h) {
-    const uint64_t q0 = (np.e_base + uint64_t(e0[h])) >> 2;
 #pragma unroll
     for (int s = 0; s < M / 4; ++s) {
-      const uint4 w = noise_block_q(np, q0 + s);
+      uint4 w;
+      if constexpr (NARROW) {
+        w = noise_block_lo(np, q0[h] + s);
+      } else {
+        w = noise_block_q(np, ((np.e_base + uint64_t(e0[h])) >> 2) + s);
+      }
       x[h][4 * s] = w.x, x[h][4 * s + 1] = w.y, x[h][4 * s + 2] = w.z, x[h][4 * s + 3] = w.w;
     }
   }
@@ -97,9 +102,9 @@ __device__ __forceinline__ float lane_of(V v, int h) {
 // L groups (one per lane of V) processed in lockstep by one thread; writes their
 // outputs and returns each group's hard bits in bits[h].
 // The keys of L groups from their staged logits (first half of fwd_groups).
-template <int M, class V>
-__device__ __forceinline__ void fwd_keys(const float* const* phi_g, const int64_t* e0, const FwdArgs& a,
-                                         V (&kap)[M]) {
+template <int M, class V, bool NARROW = false>
+__device__ __forceinline__ void fwd_keys(const float* const* phi_g, const int64_t* e0, const uint32_t* q0,
+                                         const FwdArgs& a, V (&kap)[M]) {
   constexpr int L = vlanes<V>();
   float ph[L][M];
 #pragma unroll
@@ -110,7 +115,7 @@ __device__ __forceinline__ void fwd_keys(const float* const* phi_g, const int64_
       ph[h][4 * s] = p.x, ph[h][4 * s + 1] = p.y, ph[h][4 * s + 2] = p.z, ph[h][4 * s + 3] = p.w;
     }
   }
-  group_keys<M, V>(ph, e0, a.np, kap);
+  group_keys<M, V, NARROW>(ph, e0, q0, a.np, kap);
 }
 
 // Relaxation, hard bits and outputs of L groups whose keys are `kap`.
@@ -227,7 +232,7 @@ template <int N, int M, bool TAU1, class V, bool ST = false>
 __device__ __forceinline__ void fwd_groups(const float* const* phi_g, const uint16_t* const* W_g, const int64_t* e0,
                                            const FwdArgs& a, uint32_t* bits) {
   V kap[M];
-  fwd_keys<M, V>(phi_g, e0, a, kap);
+  fwd_keys<M, V>(phi_g, e0, nullptr, a, kap);
   fwd_finish<N, M, TAU1, V, ST>(kap, W_g, e0, a, bits);
 }
 
@@ -266,14 +271,16 @@ __device__ __forceinline__ void store_hard_pair(uint32_t* hard, int64_t e0a, int
 }
 
 // One full tile of a tensor (local tile index `tile`), inputs staged in shared
-// memory.
-template <int N, int M, bool TAU1, bool ST>
+// memory.  NARROW: the call's counters are below 2^32 (a.np.narrow).
+template <int N, int M, bool TAU1, bool ST, bool NARROW>
 __device__ __forceinline__ void fwd_tile(const uint8_t* const* stage, int64_t tile, const FwdArgs& a) {
   using C = Cfg<M>;
   constexpr int kT = C::kTile;
   const float* sphi = reinterpret_cast<const float*>(stage[0]);
   const uint16_t* sW = reinterpret_cast<const uint16_t*>(stage[1]);
   const int64_t base = tile * kT;
+  // low word of the tile's first counter (uniform); group g adds g M / 4
+  const uint32_t qt = uint32_t((a.np.e_base + uint64_t(base)) >> 2);
   // pair p: groups t and t + kThreads of the p-th block of 2 kThreads groups.
   // The keys of pair p + 1 (integer-heavy: Philox, range reduction) are
   // formed before pair p is relaxed (floating-point-heavy), so the two
@@ -283,7 +290,8 @@ __device__ __forceinline__ void fwd_tile(const uint8_t* const* stage, int64_t ti
     const int g0 = threadIdx.x, g1 = g0 + C::kThreads;
     const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
     const int64_t e0[2] = {base + g0 * M, base + g1 * M};
-    fwd_keys<M, F2>(pp, e0, a, kap[0]);
+    const uint32_t q0[2] = {qt + uint32_t(g0 * (M / 4)), qt + uint32_t(g1 * (M / 4))};
+    fwd_keys<M, F2, NARROW>(pp, e0, q0, a, kap[0]);
   }
 #pragma unroll
   for (int p = 0; p < C::kPairs; ++p) {
@@ -291,7 +299,8 @@ __device__ __forceinline__ void fwd_tile(const uint8_t* const* stage, int64_t ti
       const int g0 = threadIdx.x + 2 * (p + 1) * C::kThreads, g1 = g0 + C::kThreads;
       const float* pp[2] = {sphi + g0 * M, sphi + g1 * M};
       const int64_t e0[2] = {base + g0 * M, base + g1 * M};
-      fwd_keys<M, F2>(pp, e0, a, kap[(p + 1) & 1]);
+      const uint32_t q0[2] = {qt + uint32_t(g0 * (M / 4)), qt + uint32_t(g1 * (M / 4))};
+      fwd_keys<M, F2, NARROW>(pp, e0, q0, a, kap[(p + 1) & 1]);
     }
     const int g0 = threadIdx.x + 2 * p * C::kThreads, g1 = g0 + C::kThreads;
     const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
@@ -338,7 +347,17 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_fwd_
   pdl_launch_dependents();
   const bool ok = run_tiles<C::kThreads, C::kTile, C::kStages, 2>(
       smem, src, a.full_tiles, a.status,
-      [&](const uint8_t* const* stage, int64_t tile) { fwd_tile<N, M, TAU1, ST>(stage, tile, a); });
+      [&](const uint8_t* const* stage, int64_t tile) {
+        // 32-bit counters for M = 4 only: at M = 8 the second copy of the tile
+        // body measured slower (register allocation), so those keep one
+        if constexpr (M == 4) {
+          if (a.np.narrow) {
+            fwd_tile<N, M, TAU1, ST, true>(stage, tile, a);
+            return;
+          }
+        }
+        fwd_tile<N, M, TAU1, ST, false>(stage, tile, a);
+      });
   if (ok && blockIdx.x == gridDim.x - 1) fwd_tail<N, M, TAU1, ST>(a);
   // the launch completes only after the batch's previous one (stream order)
   if (blockIdx.x == 0) pdl_wait();
@@ -423,6 +442,7 @@ int launch_fwd_impl(const FwdCall& c, bool pdl) {
   a.tau = c.tau;
   a.inv_tau = 1.0f / c.tau;
   a.np = c.np;
+  a.np.narrow = counters_narrow(c.np, c.E);
   a.status = c.status;
   if (c.N == 2 && c.M == 4) return launch_nm<2, 4>(a, c.stream, pdl);
   if (c.N == 4 && c.M == 8) return launch_nm<4, 8>(a, c.stream, pdl);

@@ -8,6 +8,13 @@
 
 namespace roi {
 
+// Every Philox counter (e_base + e) / 4 of a call of E elements is below 2^32
+// (its flat element indices stay below 2^34).
+inline bool counters_narrow(const NoiseParams& np, int64_t E) {
+  const uint64_t lim = uint64_t(1) << 34;
+  return np.e_base <= lim && uint64_t(E) <= lim - np.e_base;
+}
+
 struct FwdCall {
   const float* phi;
   const uint16_t* W;

@@ -181,6 +181,27 @@ def test_row_slices_reproduce_whole_tensor(roi, N, M, tau):
     assert np.array_equal(np.concatenate([a["hard_bits"], b["hard_bits"]]), whole["hard_bits"])
 
 
+@pytest.mark.parametrize("N,M,tau", [(2, 4, 1.0), (2, 4, 0.3), (4, 8, 1.0), (8, 16, 0.2)])
+def test_counters_past_2_to_32(roi, N, M, tau):
+    """Rows whose flat element indices cross 2^34, where the Philox counter (index / 4)
+    gains a non-zero high word: the whole call, and the same rows split at the
+    crossing (the first part's counters all below 2^32, which the tile kernels form
+    in 32-bit arithmetic; the second's all above), agree bit for bit and match the
+    oracle."""
+    rows, cols = 64, 1024
+    split = 24
+    r0 = 2 ** 34 // cols - split  # rows r0 + split onwards start at index 2^34
+    W, phi, dWm, ph, Wb, dWb = make(rows, cols, "normal", data_seed=8)
+    whole = gpu_run(roi, phi, W, dWm, N, M, tau, roi.NoiseState(31, 2, 6, 1.0, r0))
+    a = gpu_run(roi, phi[:split].contiguous(), W[:split].contiguous(), dWm[:split].contiguous(), N, M, tau,
+                roi.NoiseState(31, 2, 6, 1.0, r0))
+    b = gpu_run(roi, phi[split:].contiguous(), W[split:].contiguous(), dWm[split:].contiguous(), N, M, tau,
+                roi.NoiseState(31, 2, 6, 1.0, r0 + split))
+    for key in ("Wm", "soft", "dlogits", "dW", "hard_bits"):
+        assert np.array_equal(np.concatenate([a[key], b[key]]), whole[key]), key
+    check_against_oracle(whole, ph, Wb, dWb, N, M, tau, 31, 2, 6, 1.0, r0)
+
+
 def test_deterministic_and_noise_keyed(roi):
     W, phi, dWm, *_ = make(32, 1024, "normal", data_seed=6)
     r1 = gpu_run(roi, phi, W, dWm, 2, 4, 1.0, roi.NoiseState(1, 3, 0, 1.0, 0))
