@@ -160,6 +160,27 @@ class ClockSampler:
 # --------------------------------------------------------------------------
 # roofline denominators and counters
 # --------------------------------------------------------------------------
+# Special-function-unit work per element of the general-tau path, in ex2 issue slots
+# (lg2 and rcp take two: 32 ex2 or 16 lg2 / rcp per clock per SM on this part).
+# Algorithmic counts: the Gumbel sample needs two logs; each of the N relaxation
+# steps one exp per element and one reciprocal per group, each step but the last a
+# log per element; the backward re-forms all of it and divides by 1 - mu once per
+# element in each of its N - 1 earlier steps.
+SFU_SLOTS_PER_CLK_SM = 32
+SFU_CLOCK_MHZ = 2070  # maximum SM clock
+
+
+def sfu_slots(N, M):
+    fwd = 2 * 2 + N + 2 * (N - 1) + 2 * N / M
+    return fwd, fwd + 2 * (N - 1)
+
+
+def sfu_peak(dev):
+    import torch
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    return SFU_SLOTS_PER_CLK_SM * sms * SFU_CLOCK_MHZ * 1e6 / 1e9  # G slots/s
+
+
 def hbm_peak():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -445,6 +466,24 @@ def run_ours(args):
                 "fwd_ms_per_step": round(1e3 * fwd_t / args.steps, 3),
                 "bwd_ms_per_step": round(1e3 * bwd_t / args.steps, 3),
                 "step_gbs": round(step_gbs / world, 1), "step_frac": round(step_gbs / world / peak, 4), "per_projection": per_projection}
+    if M >= 16 and tau != 1.0:
+        # the warp-slice configurations bind on the special-function units, not HBM:
+        # the binding roofline is the SFU issue rate (the HBM figures stay beside it)
+        sf, sb = sfu_slots(N, M)
+        sp = sfu_peak(dev)
+        t_dom = bwd_t if dom == "bwd" else fwd_t
+        ach = E * (sb if dom == "bwd" else sf) * args.steps / t_dom / 1e9
+        step_ach = E * (sf + sb) * args.steps / (fwd_t + bwd_t) / 1e9
+        roofline = {"bound": "alu", "achieved": round(ach, 1), "peak": round(sp, 1), "unit": "G SFU slots/s",
+                    "frac": round(ach / sp, 4), "traffic": roofline["traffic"], "kernel": tag,
+                    "peak_kind": (f"derived: {SFU_SLOTS_PER_CLK_SM} ex2 slots per clock per SM x SMs x "
+                                  f"{SFU_CLOCK_MHZ} MHz (lg2 / rcp take two slots)"),
+                    "sfu_slots_per_element": {"fwd": sf, "bwd": sb},
+                    "units_per_launch": roofline["units_per_launch"],
+                    "fwd_ms_per_step": roofline["fwd_ms_per_step"], "bwd_ms_per_step": roofline["bwd_ms_per_step"],
+                    "step_sfu_frac": round(step_ach / sp, 4), "hbm": {k: roofline[k] for k in (
+                        "achieved", "peak", "unit", "frac", "algorithmic_bytes_per_element", "fwd_gbs", "bwd_gbs",
+                        "step_gbs", "step_frac")}, "per_projection": per_projection}
 
     # per-step device time: first forward launch to last backward launch of each step
     T = len(ev[0]) // args.steps  # events per step and direction: one per call

@@ -16,8 +16,10 @@
 // groups per chunk from shared memory (the same keys, noise and rounding as
 // roi_mask_fwd, so Wm is bit-identical to its output), writes their bf16
 // products into the chunk's A tile and arrives.  Layers with few row blocks
-// split K across CTAs; the last CTA of a row block (an atomic ticket) adds the
-// fp32 partials in split order, so Y does not depend on timing.
+// split K across CTAs, which write fp32 partials; a second launch, dependent on
+// the first (programmatic dependent launch: it is scheduled while the GEMM drains
+// and reads once the GEMM has completed), adds them in split order across the
+// whole GPU, so Y does not depend on timing.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -35,7 +37,10 @@ constexpr uint32_t kSBO = (kBK / 8) * 128;      // A tile: adjacent 8-row groups
 constexpr uint32_t kTileA = kRows * kBK * 2;    // 8 KB
 constexpr uint32_t kTilePhi = kRows * kBK * 4;  // 16 KB, [128][32] fp32 (one TMA box)
 constexpr uint32_t kTileW = kRows * kBK * 2;    // 8 KB, [128][32] bf16 (one TMA box)
-constexpr int kMinChunksPerSplit = 16;
+#ifndef ROI_LIN_MIN_CHUNKS
+#define ROI_LIN_MIN_CHUNKS 4
+#endif
+constexpr int kMinChunksPerSplit = ROI_LIN_MIN_CHUNKS;  // K chunks per split, at least
 
 template <int M>
 struct LinCfg {
@@ -46,7 +51,6 @@ struct LinCfg {
 struct LinArgs {
   float* Y;               // [T, rows]
   float* part;            // [splits, T, rows] (splits > 1)
-  unsigned int* tickets;  // [row blocks], zero at launch (splits > 1)
   int64_t T, rows, cols;
   int T_pad;              // T rounded up to 16 (the MMA's N)
   int splits, nchunks;
@@ -207,9 +211,11 @@ __global__ void __launch_bounds__(LinCfg<M>::kThreads + 32, 1)
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + L.full);    // TMA of a stage landed
   uint64_t* ready = reinterpret_cast<uint64_t*>(smem + L.ready);  // every compute thread wrote its A part
   uint64_t* mma = reinterpret_cast<uint64_t*>(smem + L.mma);      // the stage's MMAs completed
-  uint32_t* misc = reinterpret_cast<uint32_t*>(smem + L.misc);    // [0] TMEM base, [1] last-CTA flag, [2] ok
+  uint32_t* misc = reinterpret_cast<uint32_t*>(smem + L.misc);    // [0] TMEM base, [2] ok
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const bool producer = warp == kComputeWarps;  // TMA and MMA issue (one elected lane)
+  // the split-K reduction launch may be scheduled now (it waits for this grid)
+  pdl_launch_dependents();
 
   const int rb = blockIdx.x / a.splits, sp = blockIdx.x % a.splits;
   const int row0 = rb * kRows;
@@ -316,34 +322,27 @@ __global__ void __launch_bounds__(LinCfg<M>::kThreads + 32, 1)
   tc_fence_before();
   __syncthreads();
   if (warp == 0) tc_dealloc(tmem, a.tmem_cols);
-  if (!ok || a.splits == 1) return;
+}
 
-  // split K: the last CTA of this row block adds the partials in split order
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) misc[1] = atomicAdd(a.tickets + rb, 1u) == unsigned(a.splits - 1) ? 1u : 0u;
-  __syncthreads();
-  if (misc[1] == 0u) return;
-  __threadfence();
-  const int64_t rows_here = a.rows - row0 < kRows ? a.rows - row0 : kRows;
-  const int64_t split_stride = a.T * a.rows;
-  if ((a.rows & 3) == 0) {
-    // four rows per thread (float4), the loads of up to eight splits in flight
-    // before they are added, in split order
-    const int64_t n4 = a.T * (kRows / 4);
-    for (int64_t i = tid; i < n4; i += blockDim.x) {
-      const int64_t t = i / (kRows / 4), r4 = 4 * (i % (kRows / 4));
-      if (r4 >= rows_here) continue;
-      const int64_t o = t * a.rows + row0 + r4;
-      float4 acc = __ldcg(reinterpret_cast<const float4*>(a.part + o));
-      for (int q0 = 1; q0 < a.splits; q0 += 8) {
+// Split K: Y = the splits' fp32 partials ([splits][n] after one another) added in
+// split order, four consecutive outputs per thread when n % 4 == 0 (part and Y are
+// 16-byte aligned), the loads of up to eight splits in flight.
+__global__ void __launch_bounds__(256) roi_linear_reduce_kernel(const float* part, float* Y, int splits, int64_t n) {
+  pdl_wait();  // the partials of the GEMM launched before
+  const int64_t stride = int64_t(gridDim.x) * blockDim.x;
+  if ((n & 3) == 0) {
+    const int64_t n4 = n / 4;
+    const float4* p = reinterpret_cast<const float4*>(part);
+    for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < n4; i += stride) {
+      float4 acc = __ldcs(p + i);
+      for (int q0 = 1; q0 < splits; q0 += 8) {
         float4 v[8];
 #pragma unroll
         for (int j = 0; j < 8; ++j)
-          if (q0 + j < a.splits) v[j] = __ldcg(reinterpret_cast<const float4*>(a.part + (q0 + j) * split_stride + o));
+          if (q0 + j < splits) v[j] = __ldcs(p + (q0 + j) * n4 + i);
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-          if (q0 + j < a.splits) {
+          if (q0 + j < splits) {
             acc.x = __fadd_rn(acc.x, v[j].x);
             acc.y = __fadd_rn(acc.y, v[j].y);
             acc.z = __fadd_rn(acc.z, v[j].z);
@@ -351,17 +350,13 @@ __global__ void __launch_bounds__(LinCfg<M>::kThreads + 32, 1)
           }
         }
       }
-      *reinterpret_cast<float4*>(a.Y + o) = acc;
+      reinterpret_cast<float4*>(Y)[i] = acc;
     }
   } else {
-    const int64_t n = a.T * kRows;
-    for (int64_t i = tid; i < n; i += blockDim.x) {
-      const int64_t t = i / kRows, rr = i % kRows;
-      if (rr >= rows_here) continue;
-      const int64_t o = t * a.rows + row0 + rr;
-      float acc = __ldcg(a.part + o);
-      for (int q = 1; q < a.splits; ++q) acc = __fadd_rn(acc, __ldcg(a.part + q * split_stride + o));
-      a.Y[o] = acc;
+    for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < n; i += stride) {
+      float acc = __ldcs(part + i);
+      for (int q = 1; q < splits; ++q) acc = __fadd_rn(acc, __ldcs(part + q * n + i));
+      Y[i] = acc;
     }
   }
 }
@@ -419,7 +414,17 @@ int launch_nm(const LinearCall& c, const LinArgs& a) {
   }
   const int64_t row_blocks = (a.rows + kRows - 1) / kRows;
   kern<<<int(row_blocks * a.splits), LinCfg<M>::kThreads + 32, smem, c.stream>>>(tm_phi, tm_w, tm_x, a);
-  return cudaGetLastError() == cudaSuccess ? 1 : -1;
+  if (cudaGetLastError() != cudaSuccess) return -1;
+  if (a.splits == 1) return 1;
+  const int64_t n = a.T * a.rows;
+  const int64_t items = (n & 3) == 0 ? n / 4 : n;
+  int64_t blocks = (items + 255) / 256;
+  const int64_t cap = int64_t(sm_count()) * 8;
+  if (blocks > cap) blocks = cap;
+  if (blocks < 1) blocks = 1;
+  if (launch_maybe_pdl(roi_linear_reduce_kernel, int(blocks), 256, 0, c.stream, true, a.part, a.Y, a.splits, n) < 0)
+    return -1;
+  return 2;
 }
 
 }  // namespace
@@ -438,8 +443,7 @@ int linear_splits(int64_t T, int64_t rows, int64_t cols) {
 size_t linear_workspace_bytes(int64_t T, int64_t rows, int64_t cols) {
   const int s = linear_splits(T, rows, cols);
   if (s <= 1) return 0;
-  const int64_t row_blocks = (rows + kRows - 1) / kRows;
-  return size_t(s) * size_t(T) * size_t(rows) * 4 + size_t(row_blocks) * 4;
+  return size_t(s) * size_t(T) * size_t(rows) * 4;
 }
 
 bool linear_supported(int N, int M) { return (N == 2 && M == 4) || (N == 4 && M == 8) || (N == 2 && M == 8); }
@@ -461,18 +465,10 @@ int launch_masked_linear(const LinearCall& c) {
   a.status = c.status;
   // split K only as far as the caller's workspace holds the partials
   int splits = linear_splits(c.T, c.rows, c.cols);
-  const int64_t row_blocks = (c.rows + kRows - 1) / kRows;
   const size_t per_split = size_t(c.T) * size_t(c.rows) * 4;
-  const size_t tickets = size_t(row_blocks) * 4;
-  while (splits > 1 && (c.workspace == nullptr || size_t(splits) * per_split + tickets > c.workspace_bytes)) --splits;
+  while (splits > 1 && (c.workspace == nullptr || size_t(splits) * per_split > c.workspace_bytes)) --splits;
   a.splits = splits;
-  a.part = nullptr;
-  a.tickets = nullptr;
-  if (splits > 1) {
-    a.part = reinterpret_cast<float*>(c.workspace);
-    a.tickets = reinterpret_cast<unsigned int*>(reinterpret_cast<uint8_t*>(c.workspace) + size_t(splits) * per_split);
-    if (cudaMemsetAsync(a.tickets, 0, tickets, c.stream) != cudaSuccess) return -1;
-  }
+  a.part = splits > 1 ? reinterpret_cast<float*>(c.workspace) : nullptr;
   int r = -1;
   if (c.N == 2 && c.M == 4) r = launch_nm<2, 4>(c, a);
   else if (c.N == 4 && c.M == 8) r = launch_nm<4, 8>(c, a);
