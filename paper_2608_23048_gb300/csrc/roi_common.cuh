@@ -173,9 +173,11 @@ __device__ __forceinline__ float uniform_from_word(uint32_t x) {
 // round log2 u to the nearest integer at the sqrt(2) boundaries), so
 // ln u = e ln2 + ln m; ln m = 2 atanh(s), s = (m - 1) / (m + 1), |s| < 0.172,
 // 2 atanh(s) = 2s + (2/3)s^3 + (2/5)s^5 + (2/7)s^7 + (2/9)s^9 + O(s^11)
-// (truncation below 2^-28 relative).  m - 1 is exact (Sterbenz).  The Horner
-// chain in s^2 runs on the negated coefficients down to -2, so one product with
-// s gives -ln m (no final negation).
+// (truncation below 2^-28 relative).  m - 1 is exact (Sterbenz).  In t = -2s,
+// formed with one reciprocal as (m - 1) / (-(m + 1) / 2) (the halving folded into
+// the fma that forms the denominator), -ln m = t + t^3/12 + t^5/80 + t^7/448 +
+// t^9/2304: the leading term is added last and exactly in a fused multiply-add,
+// with no separate negation or doubling.
 __device__ __forceinline__ int rounded_exponent(float x) {
   return int(__float_as_uint(x) - 0x3f3504f3u) >> 23;  // 0x3f3504f3: sqrt(1/2)
 }
@@ -188,13 +190,12 @@ __device__ __forceinline__ V neg_log_unit(V u) {
                     vconst<V>(12582912.0f));
   const V one = vconst<V>(1.0f);
   const V f = vsub(m, one);
-  const V s = vmul(f, vmap(vadd(m, one), rcp_approx));
-  const V s2 = vmul(s, s);
-  V q = vfma(s2, vconst<V>(-0.22222222f), vconst<V>(-0.28571429f));
-  q = vfma(s2, q, vconst<V>(-0.4f));
-  q = vfma(s2, q, vconst<V>(-0.66666667f));
-  q = vfma(s2, q, vconst<V>(-2.0f));
-  const V nlnm = vmul(s, q);  // -ln m
+  const V t = vmul(f, vmap(vfma(m, vconst<V>(-0.5f), vconst<V>(-0.5f)), rcp_approx));
+  const V t2 = vmul(t, t);
+  V q = vfma(t2, vconst<V>(1.0f / 2304.0f), vconst<V>(1.0f / 448.0f));
+  q = vfma(t2, q, vconst<V>(1.0f / 80.0f));
+  q = vfma(t2, q, vconst<V>(1.0f / 12.0f));
+  const V nlnm = vfma(vmul(t, t2), q, t);  // -ln m
   return vfma(ef, vconst<V>(-kLn2), nlnm);
 }
 

@@ -142,13 +142,31 @@ __device__ __forceinline__ void chunk_masked_weights(const LinArgs& a, uint8_t* 
   F2 kap[M];
   {
     uint32_t x[2][M];
+    // M = 4 with every counter of the call below 2^32: the counter's low word in
+    // 32-bit arithmetic and a zero high word (as the mask kernels; rows past the
+    // last may wrap, but their outputs are never stored)
+    bool narrow = false;
+    if constexpr (M == 4) narrow = a.np.narrow;
+    if (narrow) {
+      const uint32_t qk = uint32_t(a.np.e_base >> 2) + uint32_t(k >> 2);
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const uint64_t q0 = (a.np.e_base + uint64_t(e0[h])) >> 2;
+      for (int h = 0; h < 2; ++h) {
+        const uint32_t q0 = qk + uint32_t(row0 + r + 64 * h) * uint32_t(a.cols >> 2);
 #pragma unroll
-      for (int s = 0; s < M / 4; ++s) {
-        const uint4 w = noise_block_q(a.np, q0 + s);
-        x[h][4 * s] = w.x, x[h][4 * s + 1] = w.y, x[h][4 * s + 2] = w.z, x[h][4 * s + 3] = w.w;
+        for (int s = 0; s < M / 4; ++s) {
+          const uint4 w = noise_block_lo(a.np, q0 + s);
+          x[h][4 * s] = w.x, x[h][4 * s + 1] = w.y, x[h][4 * s + 2] = w.z, x[h][4 * s + 3] = w.w;
+        }
+      }
+    } else {
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const uint64_t q0 = (a.np.e_base + uint64_t(e0[h])) >> 2;
+#pragma unroll
+        for (int s = 0; s < M / 4; ++s) {
+          const uint4 w = noise_block_q(a.np, q0 + s);
+          x[h][4 * s] = w.x, x[h][4 * s + 1] = w.y, x[h][4 * s + 2] = w.z, x[h][4 * s + 3] = w.w;
+        }
       }
     }
 #pragma unroll
@@ -462,6 +480,7 @@ int launch_masked_linear(const LinearCall& c) {
   a.tau = c.tau;
   a.inv_tau = 1.0f / c.tau;
   a.np = c.np;
+  a.np.narrow = counters_narrow(c.np, c.rows * c.cols);
   a.status = c.status;
   // split K only as far as the caller's workspace holds the partials
   int splits = linear_splits(c.T, c.rows, c.cols);
