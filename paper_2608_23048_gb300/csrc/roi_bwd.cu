@@ -398,7 +398,9 @@ __device__ __forceinline__ void bwd_tail(const BwdArgs& a, const BwdOptArgs& o) 
 
 // ST: straight-through dW from the forward's hard bits; OPT: fused AdamW step on
 // the logits (separate instantiations, so the plain kernel's code is not touched)
-template <int N, int M, bool TAU1, bool ST, bool OPT>
+// NARROW_ONLY: launched only for calls whose counters are all below 2^32 (one tile
+// body, 32-bit counters; the 4:8 tau = 1 backward fused with AdamW)
+template <int N, int M, bool TAU1, bool ST, bool OPT, bool NARROW_ONLY = false>
 __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_kernel(BwdArgs a, BwdOptArgs o) {
   uint8_t* smem = roi_bwd_smem;
   using C = Cfg<M>;
@@ -414,8 +416,14 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_
   const bool ok = run_tiles<C::kThreads, C::kTile, C::kStages, 3>(
       smem, src, a.full_tiles, a.status,
       [&](const uint8_t* const* stage, int64_t tile) {
-        // 32-bit counters for M = 4 only (at M = 8 the second copy of the tile body
-        // spills)
+        // 32-bit counters in a second copy of the tile body for M = 4 (at M = 8 that
+        // copy spills; a narrow-only 4:8 kernel measured faster only when fused with
+        // AdamW: 386 against 418 us per 18944 x 3584 tensor, while the plain one
+        // spilled, 225 against 192 us)
+        if constexpr (NARROW_ONLY) {
+          bwd_tile<N, M, TAU1, ST, OPT, true>(stage, tile, a, o, smem);
+          return;
+        }
         if constexpr (M == 4) {
           if (a.np.narrow) {
             bwd_tile<N, M, TAU1, ST, OPT, true>(stage, tile, a, o, smem);
@@ -469,10 +477,10 @@ struct LaunchCache {
   int per_sm[64] = {0};
 };
 
-template <int N, int M, bool TAU1, bool ST, bool OPT>
+template <int N, int M, bool TAU1, bool ST, bool OPT, bool NARROW_ONLY = false>
 int launch_tiles(const BwdArgs& a, const BwdOptArgs& o, cudaStream_t stream, bool pdl = false) {
   using C = Cfg<M>;
-  auto kern = roi_bwd_kernel<N, M, TAU1, ST, OPT>;
+  auto kern = roi_bwd_kernel<N, M, TAU1, ST, OPT, NARROW_ONLY>;
   const size_t smem = kHistBytes<N, M> == 0 ? tile_smem_bytes<C::kTile, C::kStages>(8)
                       : OPT               ? kMomOffset<N, M> + kMomBytes<M>
                                           : kHistOffset<M> + kHistBytes<N, M>;
@@ -495,6 +503,9 @@ int launch_tiles(const BwdArgs& a, const BwdOptArgs& o, cudaStream_t stream, boo
 template <int N, int M>
 int launch_nm(const BwdArgs& a, const BwdOptArgs& o, cudaStream_t stream, bool pdl = false) {
   const bool t1 = a.tau == 1.0f;
+  if constexpr (N == 4 && M == 8) {
+    if (t1 && a.np.narrow && o.phi_out != nullptr) return launch_tiles<N, M, true, false, true, true>(a, o, stream, pdl);
+  }
   if (o.phi_out != nullptr)
     return t1 ? launch_tiles<N, M, true, false, true>(a, o, stream, pdl)
               : launch_tiles<N, M, false, false, true>(a, o, stream, pdl);

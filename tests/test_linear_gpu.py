@@ -74,6 +74,7 @@ LIN_CASES = [
     (128, 2048, 64, 4, 8, 0.3, "logw"),
     (64, 1000, 40, 2, 8, 1.0, "normal"),    # fewer rows than one block
     (384, 4096, 48, 2, 4, 1.0, "logw"),     # split K (three row blocks, long K)
+    (130, 4096, 3, 2, 4, 1.0, "normal"),    # split K with T * rows not a multiple of 4
 ]
 
 
@@ -106,6 +107,33 @@ def test_wide_key_gaps_take_exact_path(roi, N, M, tau):
     st = roi.NoiseState(4, 1, 0, 1.0, 0)
     Y = gpu_linear(roi, X, phi, W, N, M, tau, st)
     check(Y, WL.bf16_bits(X), phi.numpy(), WL.bf16_bits(W), N, M, tau, 4, 1)
+
+
+@pytest.mark.parametrize("N,M,tau", [(2, 4, 1.0), (4, 8, 0.5)])
+def test_nonfinite_logits(roi, N, M, tau):
+    """NaN or +inf logits make their group's Wm NaN (as in the mask forward), so the
+    rows holding them come out NaN for every token; a -inf member only gets zero
+    weight; every other output matches the oracle."""
+    import torch
+    rows, cols, T = 200, 256, 24
+    W, phi, _ = WL.make_inputs(rows, cols, "normal", 41)
+    phi = phi.clone()
+    phi[3, 5] = float("nan")
+    phi[7, 100] = float("inf")
+    phi[150, 33] = float("-inf")
+    phi[199, 255] = float("nan")        # last row of the ragged second row block
+    X = WL.make_tokens(T, cols, 41)
+    st = roi.NoiseState(6, 1, 0, 1.0, 0)
+    Y = gpu_linear(roi, X, phi, W, N, M, tau, st)
+    with np.errstate(invalid="ignore"):
+        o = O.masked_linear_fwd(WL.bf16_bits(X), phi.numpy(), WL.bf16_bits(W), N, M, tau, 6, 1)
+    bad = np.isnan(o["Y"])
+    assert bad[:, 3].all() and bad[:, 7].all() and bad[:, 199].all() and not bad[:, 150].any()
+    assert np.array_equal(np.isnan(Y), bad)
+    Wm = O.bf16_to_f32(o["Wm"]).astype(np.float64)
+    fin = ~np.isnan(Wm).any(axis=1)
+    tol, _ = linear_tolerance(WL.bf16_bits(X)[:, :], o["Wm"][fin], cols)
+    assert np.all(np.abs(Y[:, fin] - o["Y"][:, fin]) <= tol)
 
 
 def test_prologue_wm_is_the_mask_forward(roi):
