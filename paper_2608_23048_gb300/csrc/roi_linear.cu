@@ -142,12 +142,10 @@ __device__ __forceinline__ void chunk_masked_weights(const LinArgs& a, uint8_t* 
   F2 kap[M];
   {
     uint32_t x[2][M];
-    // M = 4 with every counter of the call below 2^32: the counter's low word in
-    // 32-bit arithmetic and a zero high word (as the mask kernels; rows past the
-    // last may wrap, but their outputs are never stored)
-    bool narrow = false;
-    if constexpr (M == 4) narrow = a.np.narrow;
-    if (narrow) {
+    // every counter of the call below 2^32: the counter's low word in 32-bit
+    // arithmetic and a zero high word (as the mask kernels; rows past the last may
+    // wrap, but their outputs are never stored)
+    if (a.np.narrow) {
       const uint32_t qk = uint32_t(a.np.e_base >> 2) + uint32_t(k >> 2);
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
