@@ -20,7 +20,7 @@ Data layout (the same contract the library implements):
     bfloat16 type).
   * hard mask: flat bit array, uint32 words, bit b of word w = element 32*w + b.
 
-Readings of the paper taken here (each also listed in the design doc):
+Readings of the paper taken here:
   * Algorithm 1's candidate loop runs over the M members of a group and its
     output S has M entries; the number of relaxation steps is N (the paper's K).
   * lambda enters as kappa = phi / lambda + g (Sec. 4.2.3, Gumbel-top-K on the
