@@ -398,8 +398,10 @@ __device__ __forceinline__ void bwd_tail(const BwdArgs& a, const BwdOptArgs& o) 
 
 // ST: straight-through dW from the forward's hard bits; OPT: fused AdamW step on
 // the logits (separate instantiations, so the plain kernel's code is not touched)
-// NARROW_ONLY: launched only for calls whose counters are all below 2^32 (one tile
-// body, 32-bit counters; the 4:8 tau = 1 backward fused with AdamW)
+// NARROW_ONLY: launched only for calls whose counters are all below 2^32 (32-bit
+// counters): every M = 4 variant, and the 4:8 tau = 1 backward fused with AdamW (at
+// 4:8 the narrow plain backward spilled, 225 against 192 us per 18944 x 3584
+// tensor, while the fused one gained, 386 against 418 us)
 template <int N, int M, bool TAU1, bool ST, bool OPT, bool NARROW_ONLY = false>
 __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_kernel(BwdArgs a, BwdOptArgs o) {
   uint8_t* smem = roi_bwd_smem;
@@ -416,21 +418,7 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_
   const bool ok = run_tiles<C::kThreads, C::kTile, C::kStages, 3>(
       smem, src, a.full_tiles, a.status,
       [&](const uint8_t* const* stage, int64_t tile) {
-        // 32-bit counters in a second copy of the tile body for M = 4 (at M = 8 that
-        // copy spills; a narrow-only 4:8 kernel measured faster only when fused with
-        // AdamW: 386 against 418 us per 18944 x 3584 tensor, while the plain one
-        // spilled, 225 against 192 us)
-        if constexpr (NARROW_ONLY) {
-          bwd_tile<N, M, TAU1, ST, OPT, true>(stage, tile, a, o, smem);
-          return;
-        }
-        if constexpr (M == 4) {
-          if (a.np.narrow) {
-            bwd_tile<N, M, TAU1, ST, OPT, true>(stage, tile, a, o, smem);
-            return;
-          }
-        }
-        bwd_tile<N, M, TAU1, ST, OPT, false>(stage, tile, a, o, smem);
+        bwd_tile<N, M, TAU1, ST, OPT, NARROW_ONLY>(stage, tile, a, o, smem);
       });
   if (ok && blockIdx.x == gridDim.x - 1) bwd_tail<N, M, TAU1, ST, OPT>(a, o);
   // the launch completes only after the batch's previous one (stream order)
@@ -505,6 +493,18 @@ int launch_nm(const BwdArgs& a, const BwdOptArgs& o, cudaStream_t stream, bool p
   const bool t1 = a.tau == 1.0f;
   if constexpr (N == 4 && M == 8) {
     if (t1 && a.np.narrow && o.phi_out != nullptr) return launch_tiles<N, M, true, false, true, true>(a, o, stream, pdl);
+  }
+  if constexpr (M == 4) {
+    if (a.np.narrow) {
+      if (o.phi_out != nullptr)
+        return t1 ? launch_tiles<N, M, true, false, true, true>(a, o, stream, pdl)
+                  : launch_tiles<N, M, false, false, true, true>(a, o, stream, pdl);
+      if (a.hard_in != nullptr && a.dW != nullptr)
+        return t1 ? launch_tiles<N, M, true, true, false, true>(a, o, stream, pdl)
+                  : launch_tiles<N, M, false, true, false, true>(a, o, stream, pdl);
+      return t1 ? launch_tiles<N, M, true, false, false, true>(a, o, stream, pdl)
+                : launch_tiles<N, M, false, false, false, true>(a, o, stream, pdl);
+    }
   }
   if (o.phi_out != nullptr)
     return t1 ? launch_tiles<N, M, true, false, true>(a, o, stream, pdl)
