@@ -231,3 +231,52 @@ def test_straight_through_batch_equals_single_calls(roi):
         roi.roi_device_status()
         for a, b in zip(res, bat):
             assert_same(a, b)
+
+
+@pytest.mark.parametrize("N,M", [(2, 4), (4, 8)])
+def test_batch_mixes_counter_widths(roi, N, M):
+    """Items whose noise counters all fit 32 bits (the kernels form them in 32-bit
+    arithmetic) chained with items whose flat indices pass 2^34 (64-bit counters), in
+    one batch: each equals its single call bit for bit (plain and fused with AdamW,
+    tau = 1), and a wide item matches the oracle."""
+    import torch
+    shapes = [(37, 1024), (64, 3584), (29, 1536), (5, 2048)]
+    ts = make_set(shapes, 120 + M)
+    for k, t in enumerate(ts):
+        if k % 2:  # rows from flat index 2^34 on
+            seed, step, tid, lam, _ = t["st"]
+            t["st"] = (seed, step, tid, lam, 2 ** 34 // t["cols"] + k)
+    flags = [(True, True, True)] * len(ts)
+    single = run_single(roi, ts, N, M, 1.0, flags)
+    batch = run_batch(roi, ts, N, M, 1.0, flags)
+    for a, b in zip(single, batch):
+        assert_same(a, b)
+    t, o = ts[1], batch[1]
+    seed, step, tid, lam, roff = t["st"]
+    ph, Wb = t["phi"].cpu().numpy(), WL.bf16_bits(t["W"].cpu())
+    ref = O.mask_fwd(ph, Wb, N, M, 1.0, seed, step, tensor_id=tid, lam=lam, row_offset=roff)
+    ref32 = O.mask_fwd(ph, Wb, N, M, 1.0, seed, step, tensor_id=tid, lam=lam, row_offset=roff, dtype=np.float32)
+    outside, _ = C.hard_mismatches(o["hard"].cpu().numpy().view(np.uint32), ref["hard_bits"], ref["keys"], N, M,
+                                   t["rows"] * t["cols"])
+    assert outside == 0
+    n, _ = C.soft_violations(o["soft"].cpu().numpy(), ref["soft"], ref["keys"], N, M, 1.0,
+                             extra=4.0 * np.abs(ref32["soft"].astype(np.float64) - ref["soft"]))
+    assert n == 0
+    opt = roi.AdamW(1e-3, 0.9, 0.95, 1e-8, 0.05, 4)
+    def state():
+        return [{"phi": t["phi"].clone(), "m": torch.zeros_like(t["phi"]), "v": torch.full_like(t["phi"], 1e-8),
+                 "dphi": torch.empty_like(t["phi"])} for t in ts]
+    one, bat = state(), state()
+    for t, s_ in zip(ts, one):
+        roi.roi_mask_bwd_adamw(s_["phi"], t["W"], t["st"], N, M, t["dWm"], 1.0, s_["m"], s_["v"], opt, s_["dphi"])
+    roi.roi_mask_bwd_adamw_batch([(b["phi"], t["W"], t["st"], t["dWm"], b["m"], b["v"], b["dphi"], None)
+                                  for t, b in zip(ts, bat)], N, M, 1.0, opt)
+    roi.roi_device_status()
+    for a, b, r in zip(one, bat, single):
+        for k in ("phi", "m", "v", "dphi"):
+            assert torch.equal(a[k].view(torch.int32), b[k].view(torch.int32)), k
+        # the fused step's gradient is the plain backward's (up to the compilers'
+        # contraction of the two kernels)
+        g, gr = a["dphi"].cpu().numpy(), r["dphi"].cpu().numpy()
+        scale = np.abs(gr).reshape(-1, M).max(-1, keepdims=True).repeat(M, -1).reshape(gr.shape)
+        assert np.all(np.abs(g - gr) <= 1e-6 * scale + 1e-30)
