@@ -160,6 +160,9 @@ class ClockSampler:
 # --------------------------------------------------------------------------
 # roofline denominators and counters
 # --------------------------------------------------------------------------
+NOMINAL_HBM_GBS = 7900.0  # GB300 HBM3e, nominal (the measured copy bandwidth is the peak used)
+
+
 # Special-function-unit work per element of the general-tau path, in ex2 issue slots
 # (lg2 and rcp take two: 32 ex2 or 16 lg2 / rcp per clock per SM on this part).
 # Algorithmic counts: the Gumbel sample needs two logs; each of the N relaxation
@@ -465,7 +468,9 @@ def run_ours(args):
                 "fwd_gbs": round(fwd_gbs, 1), "bwd_gbs": round(bwd_gbs, 1),
                 "fwd_ms_per_step": round(1e3 * fwd_t / args.steps, 3),
                 "bwd_ms_per_step": round(1e3 * bwd_t / args.steps, 3),
-                "step_gbs": round(step_gbs / world, 1), "step_frac": round(step_gbs / world / peak, 4), "per_projection": per_projection}
+                "step_gbs": round(step_gbs / world, 1), "step_frac": round(step_gbs / world / peak, 4),
+                "nominal_hbm_gbs": NOMINAL_HBM_GBS, "frac_of_nominal": round(achieved / NOMINAL_HBM_GBS, 4),
+                "step_frac_of_nominal": round(step_gbs / world / NOMINAL_HBM_GBS, 4), "per_projection": per_projection}
     if M >= 16 and tau != 1.0:
         # the warp-slice configurations bind on the special-function units, not HBM:
         # the binding roofline is the SFU issue rate (the HBM figures stay beside it)
