@@ -405,24 +405,24 @@ def anneal(init: float, end: float, t, T_anneal: float):
 def adamw_step(phi, g, m, v, lr, beta1, beta2, eps, weight_decay, t, dtype=np.float64):
     """One AdamW step on the logits (decoupled weight decay; the optimizer and its
     hyper-parameters of Sec. 5.1 and the hyper-parameter table: beta1 = 0.9,
-    beta2 = 0.95, weight decay 0.05), written out from its definition in the
-    arrangement common to AdamW implementations:
-        phi  <- phi * (1 - lr * weight_decay)
-        m    <- beta1 m + (1 - beta1) g
-        v    <- beta2 v + (1 - beta2) g^2
-        step  = lr / (1 - beta1^t),   r = 1 / sqrt(1 - beta2^t)   (scalars, float64)
-        phi  <- phi - (step * m) / (sqrt(v) * r + eps)
-    t is the 1-based step count.  Returns (phi, m, v)."""
+    beta2 = 0.95, weight decay 0.05), written out from its definition, in the
+    order the definition states it:
+        phi   <- phi * (1 - lr * weight_decay)          (decoupled weight decay)
+        m     <- beta1 m + (1 - beta1) g
+        v     <- beta2 v + (1 - beta2) g^2
+        m_hat  = m / (1 - beta1^t),   v_hat = v / (1 - beta2^t)
+        phi   <- phi - lr * m_hat / (sqrt(v_hat) + eps)
+    t is the 1-based step count; the bias-correction denominators 1 - beta^t are
+    scalars formed in float64.  Returns (phi, m, v)."""
     ar = _Arith(dtype)
     phi, g, m, v = (ar.cast(np.asarray(x, dtype=np.float64)) for x in (phi, g, m, v))
     c = lambda x: ar.cast(np.float64(x))
     phi = phi * (c(1.0) - c(lr) * c(weight_decay))
     m = c(beta1) * m + (c(1.0) - c(beta1)) * g
     v = c(beta2) * v + (c(1.0) - c(beta2)) * (g * g)
-    step = c(lr / (1.0 - beta1 ** t))
-    r = c(1.0 / np.sqrt(1.0 - beta2 ** t))
-    den = ar.cast(np.sqrt(v)) * r + c(eps)
-    phi = phi - (step * m) / den
+    m_hat = m / c(1.0 - beta1 ** t)
+    v_hat = v / c(1.0 - beta2 ** t)
+    phi = phi - c(lr) * m_hat / (ar.cast(np.sqrt(v_hat)) + c(eps))
     return phi, m, v
 
 

@@ -51,16 +51,60 @@ def soft_violations(got, want, kappa64, N, M, tau, extra=None):
     return int(bad.sum()), float(np.max(np.abs(g - w) / np.maximum(tol, 1e-300)))
 
 
-def dlogit_violations(got, want, c, kappa64, N, M, tau, lam=1.0, extra=None):
-    g = np.asarray(got, dtype=np.float64).reshape(-1, M)
+def dlogit_tolerance(want, c, kappa64, N, M, tau, lam=1.0, extra=None):
+    """Allowed |got - want| of the logit gradients, per element ([groups, M])."""
     w = np.asarray(want, dtype=np.float64).reshape(-1, M)
     cs = np.abs(np.asarray(c, dtype=np.float64)).reshape(-1, M).max(axis=1, keepdims=True) / (tau * lam)
     scale = np.maximum(np.abs(w).max(axis=1, keepdims=True), cs)
     tol = (1e-5 + 8 * N * eps_z(kappa64, M, tau)) * scale
     if extra is not None:
         tol = tol + np.abs(np.asarray(extra, dtype=np.float64)).reshape(-1, M)
+    return np.broadcast_to(tol, w.shape)
+
+
+def dlogit_violations(got, want, c, kappa64, N, M, tau, lam=1.0, extra=None):
+    g = np.asarray(got, dtype=np.float64).reshape(-1, M)
+    w = np.asarray(want, dtype=np.float64).reshape(-1, M)
+    tol = dlogit_tolerance(want, c, kappa64, N, M, tau, lam, extra)
     bad = ~(np.abs(g - w) <= tol)
     return int(bad.sum()), float(np.max(np.abs(g - w) / np.maximum(tol, 1e-300)))
+
+
+def adamw_tolerance(phi0, g, m0, v0, tol_g, lr, beta1, beta2, eps, wd, t):
+    """Allowed |got - want| of (phi, m, v) after one AdamW step, for a float32
+    evaluation in any arrangement of the same definition (decoupled decay, moments,
+    bias corrections, lr * m_hat / (sqrt(v_hat) + eps)) whose gradient lies within
+    tol_g of the float64 gradient g, against the float64 step on g.
+
+    Gradient error, carried to first order (a factor 2 covers the curvature, since
+    tol_g / |g| is ~1e-5):
+        dm = (1 - b1) tol_g,   dv = (1 - b2) (2 |g| tol_g + tol_g^2),
+        A = m_hat / D, D = sqrt(v_hat) + eps,
+        dA = |dm_hat| / D + |m_hat| dsq / (D (D - dsq)),
+        dsq = min(sqrt(dv_hat), dv_hat / (2 sqrt(v_hat)))   (sqrt is 1/2-Hoelder),
+    and float32 rounding: each of the step's roughly ten operations rounds once
+    (relative 2^-24), so 16 u of the magnitudes involved (|phi|, lr |A|, |m|, |v|).
+    Returns (tol_phi, tol_m, tol_v)."""
+    u = 2.0 ** -24
+    phi0, g, m0, v0, tol_g = (np.asarray(x, dtype=np.float64) for x in (phi0, g, m0, v0, tol_g))
+    bc1, bc2 = 1.0 - beta1 ** t, 1.0 - beta2 ** t
+    m = beta1 * m0 + (1 - beta1) * g
+    v = beta2 * v0 + (1 - beta2) * g * g
+    dm = (1 - beta1) * tol_g + 16 * u * (np.abs(m) + beta1 * np.abs(m0) + (1 - beta1) * np.abs(g))
+    dv = (1 - beta2) * (2 * np.abs(g) * tol_g + tol_g ** 2) + 16 * u * (v + beta2 * v0 + (1 - beta2) * g * g)
+    m_hat, v_hat = m / bc1, v / bc2
+    sq = np.sqrt(v_hat)
+    D = sq + eps
+    dv_hat = dv / bc2
+    with np.errstate(divide="ignore", invalid="ignore"):
+        dsq = np.minimum(np.sqrt(dv_hat), np.where(sq > 0, dv_hat / (2 * sq), np.inf))
+        A = m_hat / D
+        dA = np.abs(dm / bc1) / D + np.abs(m_hat) * dsq / (D * (D - dsq))
+    # beyond half of D the first-order bound no longer holds: no allowance (such an
+    # input is too ill-conditioned for this comparison and fails it)
+    dA = np.where(dsq <= 0.5 * D, dA, 0.0)
+    tol_phi = 2 * lr * dA + 16 * u * (np.abs(phi0) + lr * np.abs(A))
+    return tol_phi, 2 * dm, 2 * dv
 
 
 def plain_relative(got, want, c=None, M=4, tau=1.0, lam=1.0):

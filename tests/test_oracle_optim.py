@@ -39,7 +39,7 @@ def test_adamw_float32_mode_rounds_like_float64_to_single_precision():
         assert np.allclose(x, y, rtol=1e-5, atol=1e-12)
 
 
-def test_anneal_schedule_eq9():
+def test_anneal_schedule_eq13():
     tau = O.anneal(1.0, 0.05, [0, 750, 1500, 2000], 1500)
     assert tau[0] == 1.0
     assert np.isclose(tau[1], np.sqrt(0.05), rtol=1e-14)    # geometric midpoint
