@@ -100,7 +100,7 @@ roi_status roi_mask_fwd_ex(const float* logits, const roi_bf16* W, int N, int M,
  * Each item is validated as the single call would be; in addition no output may
  * overlap any input or output of any item (ROI_ERR_ALIAS), so the items are
  * independent.  That lets the library chain their launches with programmatic
- * dependent launch (for (N, M) = (2, 4), (4, 8), (2, 8)): a tensor's kernel may start
+ * dependent launch (for (N, M) = (2, 4), (4, 8), (2, 8), (8, 16), (16, 32)): a tensor's kernel may start
  * on the SMs that the previous one frees as it drains, hiding the launch gap and
  * the ragged last wave of small tensors, while each launch still completes after
  * its predecessor, so the work queued after the call sees every item done.  Items
@@ -250,7 +250,9 @@ roi_status roi_export_compressed_2of4(const float* logits, const roi_bf16* W, in
  * tau, st), bit for bit, formed in the prologue of a tensor-core GEMM: Wm is
  * never written to memory and the logits and W are read once.  The sum runs in
  * float32 on the tensor cores (products of bf16 exact, accumulation order the
- * hardware's), Y is float32.
+ * hardware's), Y is float32.  If a kernel of the call gives up a wait
+ * (roi_device_status then returns ROI_ERR_TIMEOUT), out_Y is undefined: the
+ * split-K reduction still adds whatever partials the workspace holds.
  *  X             [T, cols] bf16, the layer's input tokens; 1 <= T <= 256
  *  out_Y         [T, rows] float32
  *  workspace     nullable caller-owned device memory for split-K partials
@@ -281,7 +283,12 @@ size_t roi_masked_linear_workspace_size(int64_t T, int64_t rows, int64_t cols);
  *    partials; calls that overlap in time (other streams, other threads) race on
  *    it and must be serialised by the caller;
  *  - the first call on a device looks the array up (cudaGetSymbolAddress); when
- *    calls are to be recorded by stream capture, make one call before it. */
+ *    calls are to be recorded by stream capture, make one call before it.
+ * Loading the library reserves the array on every device where its device code
+ * is loaded, whether or not this call is ever made: ROI_LINEAR_SCRATCH_BYTES of
+ * device memory per device until the process exits.  After a wait times out
+ * (ROI_ERR_TIMEOUT) out_Y is undefined, and here its partials may be stale ones
+ * of an earlier, unrelated call. */
 #define ROI_LINEAR_SCRATCH_BYTES (16u << 20)
 roi_status roi_masked_linear_fwd_noalloc(const roi_bf16* X, const float* logits, const roi_bf16* W, int N, int M,
                                          float tau, const roi_noise_state* st, int64_t T, int64_t rows, int64_t cols,
@@ -310,11 +317,25 @@ roi_status roi_noise_words(const roi_noise_state* st, int64_t rows, int64_t cols
 roi_status roi_gumbel_noise(const roi_noise_state* st, int64_t rows, int64_t cols, float* out_g, void* stream);
 
 /* Device-side status.  The kernels wait on their own asynchronous copies with
- * a time limit (about 2 s); a kernel that gives up records it in a per-device
- * status word and returns early (its outputs are then incomplete).  This call
+ * a time limit (2 s unless roi_set_ring_wait_limit_ns set another); a kernel
+ * that gives up records it in a status word and returns early, after its copies
+ * in flight have landed (the outputs of that call are then undefined).  This call
  * synchronises `stream`, returns ROI_ERR_TIMEOUT if the word is set (and
- * clears it), ROI_ERR_CUDA on a CUDA error, else ROI_OK. */
+ * clears it), ROI_ERR_CUDA on a CUDA error, else ROI_OK.
+ * The word is one per device, shared by every stream, thread and call on it:
+ * the return codes of the launching calls never see a timeout, and a timeout in
+ * one caller's work is reported to whichever thread calls roi_device_status
+ * first on that device (and cleared for the others). */
 roi_status roi_device_status(void* stream);
+
+/* Wall-time limit of a kernel's wait for a stage of its copy ring (the staged
+ * tiles of logits and weights) on the current device, in ns; default
+ * 2,000,000,000.  With 0 a wait that finds its stage not yet landed gives up at
+ * once; the tests use that to run the timeout path on valid copies.  The waits
+ * with which a kernel that gave up drains its own copies in flight keep the fixed
+ * 2 s limit.  Applies to kernels launched after the call returns (it is a
+ * synchronous copy to device memory); ROI_ERR_CUDA if that copy fails. */
+roi_status roi_set_ring_wait_limit_ns(uint64_t ns);
 
 /* Static description of a status code. */
 const char* roi_status_string(roi_status s);

@@ -17,7 +17,7 @@ __all__ = [
     "roi_hard_mask_export", "roi_device_status", "roi_status_string", "roi_launch_count",
     "library_path", "hard_words", "roi_noise_words", "roi_gumbel_noise",
     "roi_mask_fwd_st", "roi_mask_bwd_st", "roi_export_compressed_2of4", "AdamW", "roi_mask_bwd_adamw",
-    "roi_anneal",
+    "roi_anneal", "roi_set_ring_wait_limit_ns",
 ]
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
@@ -112,6 +112,7 @@ def lib() -> ctypes.CDLL:
     L.roi_anneal.restype = f32
     L.roi_hard_mask_export.argtypes = [_P, i32, i32, i64, i64, _P, _P, _P, _P]
     L.roi_device_status.argtypes = [_P]
+    L.roi_set_ring_wait_limit_ns.argtypes = [u64]
     L.roi_noise_words.argtypes = [ctypes.POINTER(NoiseState), i64, i64, _P, _P]
     L.roi_gumbel_noise.argtypes = [ctypes.POINTER(NoiseState), i64, i64, _P, _P]
     L.roi_status_string.argtypes = [i32]
@@ -122,7 +123,8 @@ def lib() -> ctypes.CDLL:
                  "roi_noise_words", "roi_gumbel_noise", "roi_mask_fwd_st", "roi_mask_bwd_st",
                  "roi_export_compressed_2of4", "roi_mask_bwd_adamw", "roi_masked_linear_fwd",
                  "roi_masked_linear_fwd_noalloc", "roi_mask_fwd_batch", "roi_mask_bwd_batch",
-                 "roi_mask_bwd_adamw_batch", "roi_mask_fwd_st_batch", "roi_mask_bwd_st_batch"):
+                 "roi_mask_bwd_adamw_batch", "roi_mask_fwd_st_batch", "roi_mask_bwd_st_batch",
+                 "roi_set_ring_wait_limit_ns"):
         getattr(L, name).restype = i32
     _LIB = L
     return L
@@ -470,3 +472,12 @@ def roi_gumbel_noise(state: NoiseState, rows, cols, out_g, stream=None):
 def roi_device_status(stream=None):
     """Synchronises the stream; raises RoiError if a kernel timed out or CUDA failed."""
     _raise(lib().roi_device_status(_stream(stream)), "roi_device_status")
+
+
+ROI_DEFAULT_RING_WAIT_NS = 2_000_000_000
+
+
+def roi_set_ring_wait_limit_ns(ns: int):
+    """Wall-time limit (ns) of the kernels' waits for their staged copies on the
+    current device; 0 gives up at once when a stage has not landed (tests)."""
+    _raise(lib().roi_set_ring_wait_limit_ns(int(ns)), "roi_set_ring_wait_limit_ns")

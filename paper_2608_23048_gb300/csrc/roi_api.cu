@@ -11,7 +11,9 @@
 
 namespace roi {
 
-__device__ unsigned int g_roi_device_status = 0;
+// The device status record: word 0 the status bits (kStatusTimeout), words 2-3
+// the ring-wait limit in ns (2 s).  One per device; the kernels get its address.
+__device__ __align__(16) unsigned int g_roi_device_status[4] = {0u, 0u, 2000000000u, 0u};
 
 namespace {
 
@@ -674,6 +676,13 @@ roi_status roi_noise_words(const roi_noise_state* st, int64_t rows, int64_t cols
 roi_status roi_gumbel_noise(const roi_noise_state* st, int64_t rows, int64_t cols, float* out_g, void* stream) {
   if (out_g == nullptr && rows > 0) return ROI_ERR_NULL;
   return noise_call(st, rows, cols, nullptr, out_g, stream);
+}
+
+roi_status roi_set_ring_wait_limit_ns(uint64_t ns) {
+  if (cudaMemcpyToSymbol(g_roi_device_status, &ns, sizeof(ns), kStatusLimitWord * sizeof(unsigned int)) !=
+      cudaSuccess)
+    return ROI_ERR_CUDA;
+  return ROI_OK;
 }
 
 roi_status roi_device_status(void* stream) {

@@ -27,9 +27,12 @@ constexpr float kLn2 = 0.6931471805599453f;
 // fast path's float range and the group is recomputed by the exact routine.
 constexpr float kTinyExcl = 7.888609052210118e-31f;  // 2^-100
 
-// Bit set in the device status word (defined in roi_api.cu, passed to the
-// kernels by address) when a kernel gave up waiting for its own bulk copies.
+// The device status record (defined in roi_api.cu, one per device, passed to the
+// kernels by address): word 0 holds the status bits, words 2-3 (a 64-bit value,
+// 8-byte aligned) the wall-time limit in ns of a wait for a stage of a copy ring.
+// kStatusTimeout is set in word 0 when a kernel gave up such a wait.
 constexpr unsigned int kStatusTimeout = 1u;
+constexpr int kStatusLimitWord = 2;
 
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;
@@ -791,13 +794,40 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Waits for phase `parity` of `bar` for at most ~2 s of wall time.
+// Non-blocking test of phase `parity` of `bar`.
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Waits for phase `parity` of `bar` for at most ~2 s of wall time (the fixed limit
+// of the waits that drain a CTA's own copies before it exits).
 __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (global_timer_ns() - t0 > 2000000000ull) return false;
+  }
+}
+// Waits for a stage of a copy ring, for at most the limit in the status record
+// (read only when the stage has not landed yet, through the read-only cache: the
+// host changes it only between launches; 2 s unless the caller set another one).
+// A limit of 0 gives up as soon as the stage is found incomplete.
+__device__ __forceinline__ bool mbar_wait_ring(uint64_t* bar, uint32_t parity, const unsigned int* status) {
+  if (mbar_test_wait(bar, parity)) return true;
+  const uint64_t lim = __ldg(reinterpret_cast<const unsigned long long*>(status + kStatusLimitWord));
+  if (lim == 0) return false;
+  const uint64_t t0 = global_timer_ns();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (global_timer_ns() - t0 > lim) return false;
   }
 }
 // Global -> shared bulk copy completing on `bar` (bytes % 16 == 0, both 16-B aligned).

@@ -256,15 +256,20 @@ __global__ void __launch_bounds__(LinCfg<M>::kThreads + 32, 1)
   const uint32_t tmem = misc[0];
 
   bool ok = true;
+  // producer lane: chunks whose TMA fill was issued, and whose MMAs were committed
+  int issued = 0, committed = 0;
   if (producer) {
     if (lane == 0) {
       const uint32_t idesc = tc_idesc_bf16_f32(kRows, a.T_pad);
       const uint32_t lbo_x = L.tile_x / 4, sbo_x = 128;
-      for (int c = 0; c < kStages && c < nc; ++c) issue_chunk(&tm_phi, &tm_w, &tm_x, smem, L, c, row0, c_begin + c);
+      for (int c = 0; c < kStages && c < nc; ++c) {
+        issue_chunk(&tm_phi, &tm_w, &tm_x, smem, L, c, row0, c_begin + c);
+        issued = c + 1;
+      }
       uint32_t phase = 0;  // parity of the current pass over the stages
       int s = 0;
       for (int c = 0; c < nc && ok; ++c) {
-        ok = mbar_wait_bounded(ready + s, phase);
+        ok = mbar_wait_ring(ready + s, phase, a.status);
         if (!ok) break;
         tc_fence_after();
         const uint32_t sa = smem_addr(smem + L.a + s * kTileA);
@@ -275,11 +280,15 @@ __global__ void __launch_bounds__(LinCfg<M>::kThreads + 32, 1)
                       tc_smem_desc(sx + j * 2 * lbo_x, lbo_x, sbo_x), idesc, c > 0 || j > 0);
         }
         tc_commit(mma + s);
+        committed = c + 1;
         if (c + kStages < nc) {
           // refill this stage once its MMAs are done (its staged logits and
           // weights were consumed before `ready` completed)
-          ok = mbar_wait_bounded(mma + s, phase);
-          if (ok) issue_chunk(&tm_phi, &tm_w, &tm_x, smem, L, s, row0, c_begin + c + kStages);
+          ok = mbar_wait_ring(mma + s, phase, a.status);
+          if (ok) {
+            issue_chunk(&tm_phi, &tm_w, &tm_x, smem, L, s, row0, c_begin + c + kStages);
+            issued = c + kStages + 1;
+          }
         }
         if (s == kStages - 1) {
           s = 0;
@@ -294,7 +303,7 @@ __global__ void __launch_bounds__(LinCfg<M>::kThreads + 32, 1)
     uint32_t phase = 0;
     int s = 0;
     for (int c = 0; c < nc; ++c) {
-      if (ok) ok = mbar_wait_bounded(full + s, phase);
+      if (ok) ok = mbar_wait_ring(full + s, phase, a.status);
       if (!ok) break;
       chunk_masked_weights<N, M, TAU1>(a, smem, L, s, row0, c_begin + c);
       fence_proxy_async_smem();
@@ -308,11 +317,21 @@ __global__ void __launch_bounds__(LinCfg<M>::kThreads + 32, 1)
     }
     // the last chunk's commit covers every MMA issued before it (the previous
     // completion of that stage preceded the refill this thread already saw)
-    if (nc > 0 && ok) ok = mbar_wait_bounded(mma + (nc - 1) % kStages, uint32_t((nc - 1) / kStages) & 1u);
+    if (nc > 0 && ok) ok = mbar_wait_ring(mma + (nc - 1) % kStages, uint32_t((nc - 1) / kStages) & 1u, a.status);
   }
   if (!ok) misc[2] = 0u;
   __syncthreads();
   ok = misc[2] != 0u;
+  if (!ok && producer && lane == 0) {
+    // a wait gave up: before this CTA releases its shared memory and TMEM, let the
+    // TMA fills it issued land (the last fill of each stage; fills of a stage
+    // complete in order) and the MMAs it committed finish (a commit tracks every
+    // earlier MMA of this thread), with the fixed bounded wait
+    for (int c = issued > kStages ? issued - kStages : 0; c < issued; ++c)
+      mbar_wait_bounded(full + c % kStages, uint32_t(c / kStages) & 1u);
+    if (committed > 0) mbar_wait_bounded(mma + (committed - 1) % kStages, uint32_t((committed - 1) / kStages) & 1u);
+  }
+  if (!ok) __syncthreads();
   tc_fence_after();
   if (!ok && tid == 0) atomicOr(a.status, kStatusTimeout);
 

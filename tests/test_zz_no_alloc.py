@@ -49,6 +49,32 @@ def test_noalloc_matches_workspace_call_two_in_a_row(roi):
         assert np.array_equal(g, w)
 
 
+def test_noalloc_back_to_back_on_one_stream(roi):
+    """Both no-alloc calls queued on one stream with no synchronisation between
+    them, so the second call's GEMM follows the first call's split-K reduction on
+    the shared array directly; one synchronisation after both.  Each result equals
+    the workspace call's, bit for bit."""
+    import torch
+    dev = torch.device("cuda")
+    shapes = [(384, 4096, 48, 2, 4, 1.0, 3), (128, 8192, 64, 4, 8, 0.5, 4)]
+    want = [_run(roi, *sh, noalloc=False) for sh in shapes]
+    stream = torch.cuda.Stream(device=dev)
+    outs = []
+    inputs = []
+    for rows, cols, T, N, M, tau, seed in shapes:
+        W, phi, _ = WL.make_inputs(rows, cols, "normal", seed, device=dev)
+        X = WL.make_tokens(T, cols, seed, device=dev)
+        inputs.append((X, phi, W))
+        outs.append(torch.full((T, rows), float("nan"), dtype=torch.float32, device=dev))
+    torch.cuda.synchronize()
+    for (rows, cols, T, N, M, tau, seed), (X, phi, W), Y in zip(shapes, inputs, outs):
+        roi.roi_masked_linear_fwd_noalloc(X, phi, W, N, M, tau, roi.NoiseState(seed, 2, 1, 1.0, 0), Y,
+                                          stream=stream)
+    roi.roi_device_status(stream)
+    for g, w in zip(outs, want):
+        assert np.array_equal(g.cpu().numpy(), w)
+
+
 def test_noalloc_rejects_scratch_beyond_the_limit(roi):
     import torch
     rows, cols, T = 3584, 18944, 256
