@@ -51,6 +51,8 @@ def parse_args():
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-configs", action="store_true",
+                   help="skip the timed records of the other configurations (default: after the headline)")
     p.add_argument("--layers", type=int, default=None, help="only the first L layers (profiling cases)")
     p.add_argument("--proj", default=None, help="comma-separated projections to keep, e.g. gate")
     p.add_argument("--op", choices=("mask", "st", "adamw", "export2of4", "linear"), default="mask",
@@ -321,6 +323,227 @@ def run_reference(args):
 # --------------------------------------------------------------------------
 # our arm
 # --------------------------------------------------------------------------
+def make_set_tensors(roi, set_name, sel, dev, rank=0):
+    """Device tensors of the selected layers of a layer set (inputs and outputs)."""
+    import torch
+    kind = WL.CONFIGS[set_name].logits
+    tensors = []
+    for layer, p, rows, cols in sel:
+        W, phi, dWm = WL.make_inputs(rows, cols, kind, WL.tensor_seed(layer, p) + 7919 * rank, device=dev)
+        tensors.append({
+            "id": layer * len(WL.PROJS) + p, "rows": rows, "cols": cols, "phi": phi, "W": W, "dWm": dWm,
+            "Wm": torch.empty_like(W), "dphi": torch.empty_like(phi),
+            "hard": torch.empty(roi.hard_words(rows, cols), dtype=torch.int32, device=dev)})
+    torch.cuda.synchronize()
+    return tensors
+
+
+class MaskStep:
+    """One step: roi_mask_fwd over every tensor (forward order), then roi_mask_bwd over
+    every tensor (reverse order), step-keyed noise, on one stream; batched calls (one
+    per direction) unless per_tensor.  step(s, ev) records events around each call
+    into ev = (fwd start, fwd end, bwd start, bwd end) lists when given."""
+
+    def __init__(self, roi, tensors, N, M, tau, stream, per_tensor=False):
+        self.roi, self.tensors, self.N, self.M, self.tau = roi, tensors, N, M, tau
+        self.stream, self.per_tensor = stream, per_tensor
+        self.states = {t["id"]: roi.NoiseState(0, 0, t["id"], 1.0, 0) for t in tensors}
+        self.fwd_items = roi.make_fwd_items([(t["phi"], t["W"], self.states[t["id"]], t["Wm"], None, t["hard"])
+                                             for t in tensors])
+        self.bwd_items = roi.make_bwd_items([(t["phi"], t["W"], self.states[t["id"]], t["dWm"], t["dphi"], None)
+                                             for t in reversed(tensors)])
+
+    def _mark(self, lst, ev):
+        import torch
+        if ev is not None:
+            lst.append(torch.cuda.Event(enable_timing=True))
+            lst[-1].record(self.stream)
+
+    def __call__(self, s, ev=None):
+        roi, N, M, tau, stream = self.roi, self.N, self.M, self.tau, self.stream
+        e = ev if ev is not None else (None,) * 4
+        if not self.per_tensor:
+            for arr in (self.fwd_items, self.bwd_items):
+                for k in range(len(arr)):
+                    arr[k].st.step = s
+            self._mark(e[0], ev)
+            roi.roi_mask_fwd_batch(self.fwd_items, N, M, tau, stream=stream)
+            self._mark(e[1], ev)
+            self._mark(e[2], ev)
+            roi.roi_mask_bwd_batch(self.bwd_items, N, M, tau, stream=stream)
+            self._mark(e[3], ev)
+            return
+        for t in self.tensors:
+            st = self.states[t["id"]]
+            st.step = s
+            self._mark(e[0], ev)
+            roi.roi_mask_fwd_ex(t["phi"], t["W"], N, M, tau, st, t["Wm"], None, t["hard"], stream=stream)
+            self._mark(e[1], ev)
+        for t in reversed(self.tensors):
+            st = self.states[t["id"]]
+            self._mark(e[2], ev)
+            roi.roi_mask_bwd(t["phi"], t["W"], st, N, M, t["dWm"], tau, t["dphi"], None, stream=stream)
+            self._mark(e[3], ev)
+
+
+def time_steps(roi, step, stream, steps, warmup, world, local):
+    """W untimed warm-up steps, then K timed steps bracketed by a barrier and a device
+    synchronisation, with per-call CUDA events on the launch stream and the clocks
+    sampled meanwhile.  Returns the timings (max over ranks for the whole region)."""
+    import torch
+    import torch.distributed as dist
+    with torch.cuda.stream(stream):
+        for w in range(warmup):
+            step(w)
+    torch.cuda.synchronize()
+    roi.roi_device_status(stream)
+    ev = ([], [], [], [])
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    launches0 = roi.roi_launch_count()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clocks:
+        start.record(stream)
+        for s in range(steps):
+            step(warmup + s, ev)
+        end.record(stream)
+        torch.cuda.synchronize()
+    launches = roi.roi_launch_count() - launches0
+    if world > 1:
+        dist.barrier()
+    roi.roi_device_status(stream)
+    elapsed = start.elapsed_time(end) / 1e3
+    if world > 1:
+        tt = torch.tensor([elapsed], device=torch.device("cuda", local))
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        elapsed = float(tt.item())
+    fwd_t = sum(a.elapsed_time(b) for a, b in zip(ev[0], ev[1])) / 1e3
+    bwd_t = sum(a.elapsed_time(b) for a, b in zip(ev[2], ev[3])) / 1e3
+    # per-step device time: first forward launch to last backward launch of each step
+    T = len(ev[0]) // steps  # events per step and direction: one per call
+    step_ms = sorted(ev[0][s * T].elapsed_time(ev[3][s * T + T - 1]) for s in range(steps))
+    pct = lambda q: round(step_ms[min(len(step_ms) - 1, int(q * (len(step_ms) - 1) + 0.5))], 3)
+    return {"elapsed": elapsed, "fwd_t": fwd_t, "bwd_t": bwd_t, "ev": ev, "launches": int(launches),
+            "clocks": clocks.summary(), "step_ms": {"p10": pct(0.1), "median": pct(0.5), "p90": pct(0.9)}}
+
+
+def mask_roofline(E, N, M, tau, tm, steps, world, dev, ntensors, per_tensor=False, per_projection=None):
+    """Roofline object of the dominant kernel of a mask step: HBM for the tile
+    kernels, the special-function units for the warp-slice configurations."""
+    fwd_t, bwd_t = tm["fwd_t"], tm["bwd_t"]
+    step_gbs = world * E * (FWD_BYTES + BWD_BYTES) * steps / tm["elapsed"] / 1e9
+    peak, peak_kind = hbm_peak()
+    fwd_gbs = E * FWD_BYTES * steps / fwd_t / 1e9
+    bwd_gbs = E * BWD_BYTES * steps / bwd_t / 1e9
+    dom = "bwd" if bwd_t >= fwd_t else "fwd"
+    tag = f"roi_{dom}_kernel<{N},{M},{'tau1' if tau == 1.0 else 'tau'}>"
+    traffic = recorded_traffic(tag)
+    per_elem = BWD_BYTES if dom == "bwd" else FWD_BYTES
+    achieved = bwd_gbs if dom == "bwd" else fwd_gbs
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4),
+                "traffic": (None if traffic is None else traffic * E / ntensors),
+                "kernel": tag, "peak_kind": peak_kind,
+                "algorithmic_bytes_per_element": per_elem,
+                "units_per_launch": (f"{E / ntensors:.0f} elements (mean over the {ntensors} tensors"
+                                     + ("" if per_tensor else
+                                        "; batched calls, one chained launch per tensor, achieved from the call's "
+                                        "time") + ")"),
+                "fwd_gbs": round(fwd_gbs, 1), "bwd_gbs": round(bwd_gbs, 1),
+                "fwd_frac": round(fwd_gbs / peak, 4), "bwd_frac": round(bwd_gbs / peak, 4),
+                "fwd_ms_per_step": round(1e3 * fwd_t / steps, 3),
+                "bwd_ms_per_step": round(1e3 * bwd_t / steps, 3),
+                "step_gbs": round(step_gbs / world, 1), "step_frac": round(step_gbs / world / peak, 4),
+                "nominal_hbm_gbs": NOMINAL_HBM_GBS, "frac_of_nominal": round(achieved / NOMINAL_HBM_GBS, 4),
+                "step_frac_of_nominal": round(step_gbs / world / NOMINAL_HBM_GBS, 4)}
+    if per_projection:
+        roofline["per_projection"] = per_projection
+    if M >= 16 and tau != 1.0:
+        # the warp-slice configurations bind on the special-function units, not HBM:
+        # the binding roofline is the SFU issue rate (the HBM figures stay beside it)
+        sf, sb = sfu_slots(N, M)
+        sp = sfu_peak(dev)
+        t_dom = bwd_t if dom == "bwd" else fwd_t
+        ach = E * (sb if dom == "bwd" else sf) * steps / t_dom / 1e9
+        step_ach = E * (sf + sb) * steps / (fwd_t + bwd_t) / 1e9
+        roofline = {"bound": "alu", "achieved": round(ach, 1), "peak": round(sp, 1), "unit": "G SFU slots/s",
+                    "frac": round(ach / sp, 4), "traffic": roofline["traffic"], "kernel": tag,
+                    "peak_kind": (f"derived: {SFU_SLOTS_PER_CLK_SM} ex2 slots per clock per SM x SMs x "
+                                  f"{SFU_CLOCK_MHZ} MHz (lg2 / rcp take two slots)"),
+                    "sfu_slots_per_element": {"fwd": sf, "bwd": sb},
+                    "units_per_launch": roofline["units_per_launch"],
+                    "fwd_ms_per_step": roofline["fwd_ms_per_step"], "bwd_ms_per_step": roofline["bwd_ms_per_step"],
+                    "fwd_sfu_frac": round(E * sf * steps / fwd_t / 1e9 / sp, 4),
+                    "bwd_sfu_frac": round(E * sb * steps / bwd_t / 1e9 / sp, 4),
+                    "step_sfu_frac": round(step_ach / sp, 4), "hbm": {k: roofline[k] for k in (
+                        "achieved", "peak", "unit", "frac", "algorithmic_bytes_per_element", "fwd_gbs", "bwd_gbs",
+                        "step_gbs", "step_frac")}}
+        if per_projection:
+            roofline["per_projection"] = per_projection
+    return roofline, step_gbs
+
+
+def near_ties(roi, t, N, M, step):
+    """Groups of tensor t whose N-th and (N+1)-th perturbed keys (lambda = 1) differ
+    by less than 1e-6 at `step`: the keys are the library's, phi + g in float32 with g
+    from roi_gumbel_noise (the noise the kernels regenerate)."""
+    import torch
+    rows, cols = t["rows"], t["cols"]
+    g = torch.empty(rows * cols, dtype=torch.float32, device=t["phi"].device)
+    roi.roi_gumbel_noise(roi.NoiseState(0, step, t["id"], 1.0, 0), rows, cols, g)
+    keys = (t["phi"].reshape(-1) + g).view(-1, M)
+    top = torch.topk(keys, N + 1, dim=1).values
+    n = int((top[:, N - 1] - top[:, N] < 1e-6).sum())
+    return {"tensor": f"{t['id']} ({rows}x{cols})", "step": step, "groups": rows * cols // M, "near_tie_groups": n}
+
+
+# The remaining configurations of the benchmark's configuration list, timed after the
+# headline (one GPU): (layer set, N, M, tau, timed steps).
+CONFIG_SWEEP = [
+    ("qwen2.5-7b", 4, 8, 1.0, 10),
+    ("qwen2.5-0.5b", 2, 4, 1.0, 50),
+    ("qwen2.5-0.5b", 2, 4, 0.1, 50),
+    ("qwen2.5-1.5b", 4, 8, 0.5, 20),
+    ("qwen2.5-3b", 8, 16, 0.2, 5),
+    ("qwen2.5-3b", 16, 32, 0.2, 5),
+]
+
+
+def config_sweep(roi, stream, dev, local, cache, warmup=3):
+    """One record per configuration of CONFIG_SWEEP: the full layer set, batched calls,
+    ms/step, groups/s, roofline, clocks and near ties of the set's first gate tensor.
+    `cache` maps a layer set to its tensors (the headline's, to reuse); the sweep
+    empties it when it moves to another set, so only one set is resident at a time."""
+    import torch
+    out = []
+    for set_name, N, M, tau, steps in CONFIG_SWEEP:
+        if set_name not in cache:
+            cache.clear()
+            torch.cuda.synchronize()
+            torch.cuda.empty_cache()
+            cache[set_name] = make_set_tensors(roi, set_name, WL.LAYER_SETS[set_name].tensors(), dev)
+        tensors = cache[set_name]
+        E = sum(t["rows"] * t["cols"] for t in tensors)
+        step = MaskStep(roi, tensors, N, M, tau, stream)
+        tm = time_steps(roi, step, stream, steps, warmup, 1, local)
+        roofline, step_gbs = mask_roofline(E, N, M, tau, tm, steps, 1, dev, len(tensors))
+        gate = next(t for t in tensors if t["id"] % len(WL.PROJS) == WL.PROJS.index("gate"))
+        lset = WL.LAYER_SETS[set_name]
+        h, kv, i = lset.hidden, lset.kv, lset.inter
+        out.append({
+            "workload": (f"{set_name}-shaped layer set, {N}:{M}, tau={tau}, {lset.layers} layers x "
+                         f"{{q,o {h}x{h}; k,v {kv}x{h}; gate,up {i}x{h}; down {h}x{i}}}, "
+                         f"logits {WL.CONFIGS[set_name].logits}, step-keyed noise"),
+            "N": N, "M": M, "tau": tau, "elements": E, "groups": E // M, "steps": steps, "warmup": warmup,
+            "ms_per_step": round(1e3 * tm["elapsed"] / steps, 3), "groups_per_s": (E // M) * steps / tm["elapsed"],
+            "hbm_gbs": round(step_gbs, 1), "step_ms": tm["step_ms"], "gpu_launches": tm["launches"],
+            "roofline": roofline, "clocks": tm["clocks"],
+            "near_ties": near_ties(roi, gate, N, M, warmup + steps - 1)})
+    cache.clear()
+    return out
+
+
 def run_ours(args):
     import torch
     import torch.distributed as dist
@@ -350,78 +573,13 @@ def run_ours(args):
     roi.lib()
 
     lset = WL.LAYER_SETS[args.set]
-    kind = WL.CONFIGS[args.set].logits
-    tensors = []
-    for layer, p, rows, cols in selected_tensors(args):
-        W, phi, dWm = WL.make_inputs(rows, cols, kind, WL.tensor_seed(layer, p) + 7919 * rank, device=dev)
-        tensors.append({
-            "id": layer * len(WL.PROJS) + p, "rows": rows, "cols": cols, "phi": phi, "W": W, "dWm": dWm,
-            "Wm": torch.empty_like(W), "dphi": torch.empty_like(phi),
-            "hard": torch.empty(roi.hard_words(rows, cols), dtype=torch.int32, device=dev)})
-    torch.cuda.synchronize()
+    tensors = make_set_tensors(roi, args.set, selected_tensors(args), dev, rank)
     stream = torch.cuda.Stream(device=dev)
-    states = {t["id"]: roi.NoiseState(0, 0, t["id"], 1.0, 0) for t in tensors}
+    step = MaskStep(roi, tensors, N, M, tau, stream, per_tensor=args.per_tensor)
 
-    # batched (default): every tensor's forward in one call, every backward in one
-    fwd_items = roi.make_fwd_items([(t["phi"], t["W"], states[t["id"]], t["Wm"], None, t["hard"]) for t in tensors])
-    bwd_items = roi.make_bwd_items([(t["phi"], t["W"], states[t["id"]], t["dWm"], t["dphi"], None)
-                                    for t in reversed(tensors)])
-
-    def mark(lst, ev):
-        if ev is not None:
-            lst.append(torch.cuda.Event(enable_timing=True))
-            lst[-1].record(stream)
-
-    def step(s, ev=None):
-        if not args.per_tensor:
-            for arr in (fwd_items, bwd_items):
-                for k in range(len(arr)):
-                    arr[k].st.step = s
-            mark(ev[0] if ev else None, ev)
-            roi.roi_mask_fwd_batch(fwd_items, N, M, tau, stream=stream)
-            mark(ev[1] if ev else None, ev)
-            mark(ev[2] if ev else None, ev)
-            roi.roi_mask_bwd_batch(bwd_items, N, M, tau, stream=stream)
-            mark(ev[3] if ev else None, ev)
-            return
-        for t in tensors:
-            st = states[t["id"]]
-            st.step = s
-            mark(ev[0] if ev else None, ev)
-            roi.roi_mask_fwd_ex(t["phi"], t["W"], N, M, tau, st, t["Wm"], None, t["hard"], stream=stream)
-            mark(ev[1] if ev else None, ev)
-        for t in reversed(tensors):
-            st = states[t["id"]]
-            mark(ev[2] if ev else None, ev)
-            roi.roi_mask_bwd(t["phi"], t["W"], st, N, M, t["dWm"], tau, t["dphi"], None, stream=stream)
-            mark(ev[3] if ev else None, ev)
-
-    with torch.cuda.stream(stream):
-        for w in range(args.warmup):
-            step(w)
-    torch.cuda.synchronize()
-    roi.roi_device_status(stream)
-
-    # timed region: K steps, per-launch events for the per-kernel roofline
-    ev = ([], [], [], [])
-    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    launches0 = roi.roi_launch_count()
-    if world > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
-    with ClockSampler(local) as clocks:
-        start.record(stream)
-        for s in range(args.steps):
-            step(args.warmup + s, ev)
-        end.record(stream)
-        torch.cuda.synchronize()
-    launches = roi.roi_launch_count() - launches0
-    if world > 1:
-        dist.barrier()
-    roi.roi_device_status(stream)
-    elapsed = start.elapsed_time(end) / 1e3
-    fwd_t = sum(a.elapsed_time(b) for a, b in zip(ev[0], ev[1])) / 1e3
-    bwd_t = sum(a.elapsed_time(b) for a, b in zip(ev[2], ev[3])) / 1e3
+    # timed region: K steps, per-call events for the per-kernel roofline
+    tm = time_steps(roi, step, stream, args.steps, args.warmup, world, local)
+    elapsed, ev = tm["elapsed"], tm["ev"]
     # per projection, summed over layers, per step: fwd ms, bwd ms, fraction of the roofline
     # (per-tensor calls only)
     per_proj = {}
@@ -434,67 +592,17 @@ def run_ours(args):
         per_proj[WL.PROJS[t["id"] % len(WL.PROJS)]][1] += a.elapsed_time(b) / args.steps
     for t in tensors if args.per_tensor else ():
         per_proj[WL.PROJS[t["id"] % len(WL.PROJS)]][2] += t["rows"] * t["cols"]
-    if world > 1:
-        tt = torch.tensor([elapsed], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        elapsed = float(tt.item())
-
-    E = cfg["elements"]
-    groups_all = world * (E // M) * args.steps
-    value = groups_all / elapsed
-    step_gbs = world * E * (FWD_BYTES + BWD_BYTES) * args.steps / elapsed / 1e9
-    peak, peak_kind = hbm_peak()
-    fwd_gbs = E * FWD_BYTES * args.steps / fwd_t / 1e9
-    bwd_gbs = E * BWD_BYTES * args.steps / bwd_t / 1e9
-    dom = "bwd" if bwd_t >= fwd_t else "fwd"
-    tag = f"roi_{dom}_kernel<{N},{M},{'tau1' if tau == 1.0 else 'tau'}>"
-    traffic = recorded_traffic(tag)
-    per_elem = BWD_BYTES if dom == "bwd" else FWD_BYTES
-    achieved = bwd_gbs if dom == "bwd" else fwd_gbs
-    launches_per_kernel = len(tensors)  # one launch per tensor, batched (chained) or not
     pk = hbm_peak()[0]
     per_projection = {k: {"fwd_ms": round(f, 3), "bwd_ms": round(b, 3),
                           "frac": round(n * (FWD_BYTES + BWD_BYTES) / ((f + b) * 1e-3) / 1e9 / pk, 3)}
                       for k, (f, b, n) in per_proj.items()}
-    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
-                "frac": round(achieved / peak, 4),
-                "traffic": (None if traffic is None else traffic * E / launches_per_kernel),
-                "kernel": tag, "peak_kind": peak_kind,
-                "algorithmic_bytes_per_element": per_elem,
-                "units_per_launch": (f"{E / launches_per_kernel:.0f} elements (mean over the {launches_per_kernel} tensors"
-                                     + ("" if args.per_tensor else
-                                        "; batched calls, one chained launch per tensor, achieved from the call's "
-                                        "time") + ")"),
-                "fwd_gbs": round(fwd_gbs, 1), "bwd_gbs": round(bwd_gbs, 1),
-                "fwd_ms_per_step": round(1e3 * fwd_t / args.steps, 3),
-                "bwd_ms_per_step": round(1e3 * bwd_t / args.steps, 3),
-                "step_gbs": round(step_gbs / world, 1), "step_frac": round(step_gbs / world / peak, 4),
-                "nominal_hbm_gbs": NOMINAL_HBM_GBS, "frac_of_nominal": round(achieved / NOMINAL_HBM_GBS, 4),
-                "step_frac_of_nominal": round(step_gbs / world / NOMINAL_HBM_GBS, 4), "per_projection": per_projection}
-    if M >= 16 and tau != 1.0:
-        # the warp-slice configurations bind on the special-function units, not HBM:
-        # the binding roofline is the SFU issue rate (the HBM figures stay beside it)
-        sf, sb = sfu_slots(N, M)
-        sp = sfu_peak(dev)
-        t_dom = bwd_t if dom == "bwd" else fwd_t
-        ach = E * (sb if dom == "bwd" else sf) * args.steps / t_dom / 1e9
-        step_ach = E * (sf + sb) * args.steps / (fwd_t + bwd_t) / 1e9
-        roofline = {"bound": "alu", "achieved": round(ach, 1), "peak": round(sp, 1), "unit": "G SFU slots/s",
-                    "frac": round(ach / sp, 4), "traffic": roofline["traffic"], "kernel": tag,
-                    "peak_kind": (f"derived: {SFU_SLOTS_PER_CLK_SM} ex2 slots per clock per SM x SMs x "
-                                  f"{SFU_CLOCK_MHZ} MHz (lg2 / rcp take two slots)"),
-                    "sfu_slots_per_element": {"fwd": sf, "bwd": sb},
-                    "units_per_launch": roofline["units_per_launch"],
-                    "fwd_ms_per_step": roofline["fwd_ms_per_step"], "bwd_ms_per_step": roofline["bwd_ms_per_step"],
-                    "step_sfu_frac": round(step_ach / sp, 4), "hbm": {k: roofline[k] for k in (
-                        "achieved", "peak", "unit", "frac", "algorithmic_bytes_per_element", "fwd_gbs", "bwd_gbs",
-                        "step_gbs", "step_frac")}, "per_projection": per_projection}
 
-    # per-step device time: first forward launch to last backward launch of each step
-    T = len(ev[0]) // args.steps  # events per step and direction: one per call
-    step_ms = sorted(ev[0][s * T].elapsed_time(ev[3][s * T + T - 1]) for s in range(args.steps))
-    pct = lambda q: round(step_ms[min(len(step_ms) - 1, int(q * (len(step_ms) - 1) + 0.5))], 3)
-    step_stats = {"p10": pct(0.1), "median": pct(0.5), "p90": pct(0.9)}
+    E = cfg["elements"]
+    groups_all = world * (E // M) * args.steps
+    value = groups_all / elapsed
+    roofline, step_gbs = mask_roofline(E, N, M, tau, tm, args.steps, world, dev, len(tensors),
+                                       args.per_tensor, per_projection)
+    peak = hbm_peak()[0]
 
     # the hard masks change with the step and each step reproduces (outside the timed region)
     t0 = tensors[0]
@@ -508,13 +616,24 @@ def run_ours(args):
         st = roi.NoiseState(0, s_, t0["id"], 1.0, 0)
         roi.roi_mask_fwd_ex(t0["phi"], t0["W"], N, M, tau, st, scratch_Wm, None, out_h, stream=stream)
     torch.cuda.synchronize()
+    gate = [t for t in tensors if t["id"] % len(WL.PROJS) == WL.PROJS.index("gate")]
     checks = {"step_reproducible": bool(torch.equal(h_again, h_last)),
               "masks_differ_across_steps": bool(not torch.equal(h_prev, h_last)),
-              "checked_on": f"tensor {t0['id']} ({t0['rows']}x{t0['cols']}), steps {other} and {last}"}
+              "checked_on": f"tensor {t0['id']} ({t0['rows']}x{t0['cols']}), steps {other} and {last}",
+              "near_ties": [near_ties(roi, t, N, M, last) for t in [t0] + gate[:1]],
+              "near_ties_rule": ("groups whose N-th and (N+1)-th perturbed keys (the library's float32 keys) "
+                                 "differ by less than 1e-6, at the last timed step")}
 
     e2e = None
     if not args.no_e2e:
         e2e = run_e2e(args, roi, tensors, lset, N, M, tau, dev, world)
+
+    configs = None
+    if (world == 1 and not args.no_configs and args.set == "qwen2.5-7b" and args.layers is None
+            and args.proj is None and not args.per_tensor):
+        holder = {args.set: tensors}
+        del step, tensors, t0, gate
+        configs = config_sweep(roi, stream, dev, local, holder)
 
     if rank == 0:
         out = {"metric": METRIC, "value": value, "unit": "groups/s", "n_gpus": world, "steps": args.steps,
@@ -522,8 +641,11 @@ def run_ours(args):
                "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": cfg,
                "hbm_gbs": round(step_gbs, 1), "hbm_frac": round(step_gbs / world / peak, 4),
                "roofline": roofline, "cpu_baseline": base, "e2e": e2e,
-               "gpu_launches": int(launches), "step_ms": step_stats, "checks": checks, "clocks": clocks.summary(),
-               "clocks_note": "sampled with nvidia-smi every 100 ms during the timed region"}
+               "gpu_launches": tm["launches"], "step_ms": tm["step_ms"], "checks": checks, "clocks": tm["clocks"],
+               "clocks_note": "sampled with nvidia-smi every 100 ms during the timed region",
+               "configs": configs,
+               "configs_note": ("the other configurations of the benchmark list, each its full layer set with "
+                                "batched calls, timed after the headline on the same GPU (one GPU runs only)")}
         print(json.dumps(out), flush=True)
     if world > 1:
         dist.destroy_process_group()
