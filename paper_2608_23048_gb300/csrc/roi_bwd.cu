@@ -280,9 +280,11 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
   }
   if constexpr (HIST) bwd_upstream<M, V>(W_g, dWm_g, c);
   fg.backward(c, a.inv_tau, dkv);
-  // dL/dphi = dL/dkappa / lambda
+  // dL/dphi = dL/dkappa / lambda (lambda = 1: nothing to scale, the same bits)
+  if (a.np.inv_lam != 1.0f) {
 #pragma unroll
-  for (int l = 0; l < M; ++l) dkv[l] = vmul(dkv[l], vconst<V>(a.np.inv_lam));
+    for (int l = 0; l < M; ++l) dkv[l] = vmul(dkv[l], vconst<V>(a.np.inv_lam));
+  }
   if constexpr (kStageMoments) cp_async_wait_all();
 #pragma unroll
   for (int h = 0; h < L; ++h) {

@@ -577,11 +577,10 @@ struct SmemSteps {
 template <int N, int M, bool TAU1, bool KEEP, class V = float,
           class Steps = RegSteps<KEEP ? N : 1, KEEP ? M : 1, V>>
 struct FastGroup {
-  // KEEP: store mu of every step for a backward sweep.  With the history in
-  // registers S is re-summed from it on demand (in the order forward()
-  // accumulates it) instead of being kept live; with a shared-memory history S
-  // is accumulated as without KEEP.
-  static constexpr bool kSumS = !KEEP || Steps::kSmem;
+  // KEEP: store mu of every step for a backward sweep.  S is then not
+  // accumulated: soft() re-sums it from the history on demand (in the order
+  // forward() accumulates it), which only the backward's optional dW asks for.
+  static constexpr bool kSumS = !KEEP;
   Steps st;
   V S[kSumS ? M : 1];
   V rt_last;  // tau = 1, KEEP: 1 / sum(mu om) of step N-2 (mu(N-1) = mu(N-2) om rt_last)

@@ -305,7 +305,74 @@ __device__ __forceinline__ uint32_t slice_topn_bits(const float (&kap)[4], int N
   return bits;
 }
 
-// Hard bits of L slots (one per lane of V): comparison ranking per slot.
+// Compare-exchange keeping x[a] >= x[b].
+__device__ __forceinline__ void ce_desc(float (&x)[4], int a, int b) {
+  const float u = x[a], v = x[b];
+  x[a] = fmaxf(u, v);
+  x[b] = fminf(u, v);
+}
+// Sorts a bitonic run of four descending.
+__device__ __forceinline__ void bitonic4_desc(float (&x)[4]) {
+  ce_desc(x, 0, 2), ce_desc(x, 1, 3), ce_desc(x, 0, 1), ce_desc(x, 2, 3);
+}
+// One bitonic merge step across lanes: with this lane's four keys sorted
+// descending and the partner lane's (lane ^ o) too, the lane keeps the larger
+// (upper = false) or smaller (upper = true) element of each pair (i, partner's
+// 3 - i); the result is a bitonic run, sorted again in the lane.
+__device__ __forceinline__ void merge_across(float (&x)[4], int o, bool upper) {
+  float p[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) p[i] = __shfl_xor_sync(0xffffffffu, x[3 - i], o);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) x[i] = upper ? fminf(x[i], p[i]) : fmaxf(x[i], p[i]);
+  bitonic4_desc(x);
+}
+
+// Hard bits of a slot for N = M / 2 (the two patterns of these kernels) from the
+// group's N-th largest key.  Each lane sorts its four keys; bitonic merges across
+// lanes sort each half of the slice (M / 2 keys over SL / 2 lanes); the top M / 2
+// of the group are then the larger elements of the pairs (i-th of the first half,
+// i-th from the end of the second half), so their minimum is the threshold.  A
+// member is kept iff its key is at least the threshold.  Returns false (bits
+// unusable) if the slice's keys are not all finite or the threshold is tied, so
+// that more than N members pass: the caller ranks such groups by comparison.
+template <int N, int M>
+__device__ __forceinline__ bool slice_topn_threshold(const float (&kap)[4], int q, uint32_t& bits) {
+  static_assert(2 * N == M, "threshold selection needs N = M / 2");
+  constexpr int SL = M / 4;
+  float x[4] = {kap[0], kap[1], kap[2], kap[3]};
+  ce_desc(x, 0, 1), ce_desc(x, 2, 3), ce_desc(x, 0, 2), ce_desc(x, 1, 3), ce_desc(x, 1, 2);
+  // sorted runs of 8 over lane pairs
+  merge_across(x, 1, (q & 1) != 0);
+  if constexpr (SL == 8) {
+    // sorted runs of 16 over lane quads: the larger / smaller 8 of the two runs of
+    // 8 go to the quad's lower / upper lane pair (each lane's four sorted), and a
+    // merge within each pair orders them
+    merge_across(x, 3, (q & 2) != 0);
+    merge_across(x, 1, (q & 1) != 0);
+  }
+  // pairs (i, M/2 - 1 - i) across the two halves: lane q pairs with lane SL - 1 - q
+  float m = INFINITY;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) m = fminf(m, fmaxf(x[i], __shfl_xor_sync(0xffffffffu, x[3 - i], SL - 1)));
+#pragma unroll
+  for (int o = 1; o < SL / 2; o <<= 1) m = fminf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  bits = 0;
+  float fin = 0.0f;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    bits |= uint32_t(kap[j] >= m) << j;
+    fin += kap[j] - kap[j];  // 0 for finite keys, NaN otherwise
+  }
+  int cnt = __popc(bits) + (fin == 0.0f ? 0 : 64);
+#pragma unroll
+  for (int o = 1; o < SL; o <<= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+  return cnt == N;
+}
+
+// Hard bits of L slots (one per lane of V): the threshold selection, and for a
+// group it cannot settle (a tie at the threshold, a non-finite key) comparison
+// ranking, run by the whole warp when any of its slots needs it.
 template <int N, int M, class V>
 __device__ __forceinline__ void slot_topn(const V (&kap)[4], int base_lane, int q, uint32_t (&bits)[vlanes<V>()]) {
 #pragma unroll
@@ -313,7 +380,11 @@ __device__ __forceinline__ void slot_topn(const V (&kap)[4], int base_lane, int 
     float k[4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) k[j] = lane_of(kap[j], h);
-    bits[h] = slice_topn_bits<M>(k, N, base_lane, q);
+    const bool ok = slice_topn_threshold<N, M>(k, q, bits[h]);
+    if (__any_sync(0xffffffffu, !ok)) {
+      const uint32_t b = slice_topn_bits<M>(k, N, base_lane, q);
+      if (!ok) bits[h] = b;
+    }
   }
 }
 
@@ -448,8 +519,10 @@ __device__ __forceinline__ void bwd_slots(const float* const* p, const uint16_t*
   V dk[4];
   rx.backward(c, a.inv_tau, dk);
   if (!active) return;
+  if (a.np.inv_lam != 1.0f) {  // lambda = 1: nothing to scale, the same bits
 #pragma unroll
-  for (int j = 0; j < 4; ++j) dk[j] = vmul(dk[j], vconst<V>(a.np.inv_lam));
+    for (int j = 0; j < 4; ++j) dk[j] = vmul(dk[j], vconst<V>(a.np.inv_lam));
+  }
 #pragma unroll
   for (int h = 0; h < L; ++h) {
     if (!((flag >> h) & 1u)) {
