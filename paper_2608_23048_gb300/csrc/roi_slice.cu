@@ -18,14 +18,25 @@ constexpr int kThreads = 256;
 constexpr int kTile = 2048;  // 512 four-member slots: slots t and t + 256 per thread
 constexpr int kStagesFwd = 4;
 constexpr int kStagesBwd = 3;
-
-// Pairing doubles the per-thread state: the forward pairs M = 16; the backward,
-// which keeps the N steps of the relaxation in registers, runs one group at a time.
+// Both directions relax the two slots of a thread in lockstep on packed FP32; the
+// backward keeps its step history in shared memory behind the tile ring.  CTAs per
+// SM the registers are sized for (measured on the 3B-shaped set, tau = 0.2):
+// forward two; backward two at 8:16 (128 registers) and one at 16:32, whose paired
+// sixteen steps take 255 registers (at two CTAs it spills: 86.4 against 65.3 ms).
 template <int M>
-constexpr bool kPairedFwd = M <= 16;
+constexpr bool kPairedFwd = true;
+template <int M>
+constexpr bool kPairedBwd = true;
 constexpr int kMinBlocksFwd = 2;
 template <int M>
 constexpr int kMinBlocksBwd = M == 32 ? 1 : 2;
+// The backward's step history: steps 0 .. N-2 of one slot, or of the two slots of
+// a pair (four floats or F2 a step), per thread, thread-strided so a warp touches
+// consecutive words; the last step stays in registers.
+template <int M>
+constexpr size_t kSliceHistOffset = (tile_smem_bytes<kTile, kStagesBwd>(8) + 15) & ~size_t(15);
+template <int N, int M>
+constexpr size_t kSliceHistBytes = size_t(N - 1) * 4 * (kPairedBwd<M> ? 8 : 4) * kThreads;
 
 __device__ __forceinline__ float shfl_xor(float v, int o) { return __shfl_xor_sync(0xffffffffu, v, o); }
 __device__ __forceinline__ F2 shfl_xor(F2 v, int o) {
@@ -120,6 +131,9 @@ struct SliceArgs {
   unsigned int* status;
 };
 
+// Dynamic shared memory of the backward kernel (tile ring, then the step history).
+extern __shared__ __align__(128) uint8_t roi_slice_smem[];
+
 // Keys (log2 units, t = kappa log2 e) of L four-member slots (one per lane of V)
 // whose first elements have call-flat indices e0[h].
 template <class V>
@@ -156,9 +170,36 @@ __device__ __forceinline__ void slot_keys(const float* const* p4, const int64_t*
 template <int N, int M, bool TAU1, bool KEEP, class V>
 struct SliceRelax {
   static constexpr int SL = M / 4;
-  V mu[KEEP ? N : 1][4];
+  // KEEP: mu of the last step in registers, of steps 0 .. N-2 in shared memory
+  // at hist[(4 k + j) kThreads] (V = float)
+  V mu_last[4];
+  V* hist;
   V S[4];
   V rt_last;
+  __device__ __forceinline__ void put(int k, int j, V v) {
+    if (k == N - 1) {
+      mu_last[j] = v;
+    } else {
+      hist[(4 * k + j) * kThreads] = v;
+    }
+  }
+  __device__ __forceinline__ V get(int k, int j) const { return k == N - 1 ? mu_last[j] : hist[(4 * k + j) * kThreads]; }
+  __device__ __forceinline__ void get4(int k, V (&m)[4]) const {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) m[j] = get(k, j);
+  }
+  // S_j: accumulated by forward() without KEEP; with KEEP summed from the history
+  // on demand (in forward()'s order), which only the backward's optional dW asks for.
+  __device__ __forceinline__ V soft(int j) const {
+    if constexpr (!KEEP) {
+      return S[j];
+    } else {
+      V t = get(0, j);
+#pragma unroll
+      for (int k = 1; k < N; ++k) t = vadd(t, get(k, j));
+      return t;
+    }
+  }
 
   __device__ __forceinline__ uint32_t forward(const V (&kap)[4], float inv_tau, int base_lane) {
     uint32_t flag = 0;
@@ -180,8 +221,8 @@ struct SliceRelax {
       for (int k = 0; k < N; ++k) {
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          if constexpr (KEEP) mu[k][j] = cur[j];
-          S[j] = k == 0 ? cur[j] : vadd(S[j], cur[j]);
+          if constexpr (KEEP) put(k, j, cur[j]);
+          if constexpr (!KEEP) S[j] = k == 0 ? cur[j] : vadd(S[j], cur[j]);
         }
         if (k + 1 < N) {
           V totc, o[4], v[4];
@@ -213,8 +254,8 @@ struct SliceRelax {
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           cur[j] = vmul(e[j], r);
-          if constexpr (KEEP) mu[k][j] = cur[j];
-          S[j] = k == 0 ? cur[j] : vadd(S[j], cur[j]);
+          if constexpr (KEEP) put(k, j, cur[j]);
+          if constexpr (!KEEP) S[j] = k == 0 ? cur[j] : vadd(S[j], cur[j]);
         }
         if (k + 1 < N) {
           V ex[4];
@@ -239,37 +280,38 @@ struct SliceRelax {
     {
       V cm[4];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) cm[j] = vmul(c[j], mu[N - 1][j]);
+      for (int j = 0; j < 4; ++j) cm[j] = vmul(c[j], mu_last[j]);
       const V cmu = Slice<SL, V>::total(sum4(cm));
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         V t = vsub(c[j], cmu);
         if constexpr (!TAU1) t = vmul(itau, t);
-        b[j] = vmul(mu[N - 1][j], t);
-        if constexpr (TAU1) hl[j] = vmul(vmul(mu[N - 2][j], rt_last), t);
+        b[j] = vmul(mu_last[j], t);
+        if constexpr (TAU1) hl[j] = vmul(vmul(get(N - 2, j), rt_last), t);
       }
     }
 #pragma unroll
     for (int k = N - 2; k >= 0; --k) {
-      V cm[4], h[4], H[4];
+      V cm[4], h[4], H[4], mk[4];
+      get4(k, mk);
       if (TAU1 && k == N - 2) {
 #pragma unroll
         for (int j = 0; j < 4; ++j) h[j] = hl[j];
       } else {
         V om[4], tmp;
-        excl4(mu[k], Slice<SL, V>::others(sum4(mu[k]), tmp), om);
+        excl4(mk, Slice<SL, V>::others(sum4(mk), tmp), om);
 #pragma unroll
         for (int j = 0; j < 4; ++j) h[j] = vmul(b[j], vmap(om[j], rcp_approx));
       }
       // c_l - <c, mu> + H_l - B as (c_l + H_l) - K, K = <c, mu> + B = sum of (c mu + b)
 #pragma unroll
-      for (int j = 0; j < 4; ++j) cm[j] = vfma(c[j], mu[k][j], b[j]);
+      for (int j = 0; j < 4; ++j) cm[j] = vfma(c[j], mk[j], b[j]);
       const V K = Slice<SL, V>::total(sum4(cm));
       V tmp;
       excl4(h, Slice<SL, V>::others(sum4(h), tmp), H);
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
-        const V mu_j = TAU1 ? mu[k][j] : vmul(mu[k][j], itau);
+        const V mu_j = TAU1 ? mk[j] : vmul(mk[j], itau);
         b[j] = vfma(mu_j, vsub(vadd(c[j], H[j]), K), b[j]);
       }
     }
@@ -500,6 +542,7 @@ __device__ __forceinline__ void bwd_slots(const float* const* p, const uint16_t*
     for (int j = 0; j < 4; ++j) kap[j] = c[j] = vconst<V>(0.0f);
   }
   SliceRelax<N, M, TAU1, true, V> rx;
+  rx.hist = reinterpret_cast<V*>(roi_slice_smem + kSliceHistOffset<M>) + threadIdx.x;
   const uint32_t flag = rx.forward(kap, a.inv_tau, base_lane);
   if (active && a.dW != nullptr) {
 #pragma unroll
@@ -511,7 +554,7 @@ __device__ __forceinline__ void bwd_slots(const float* const* p, const uint16_t*
         float dv[4], sv[4];
         unpack_bf16x4(*reinterpret_cast<const uint2*>(dw[h]), dv);
 #pragma unroll
-        for (int j = 0; j < 4; ++j) sv[j] = lane_of(rx.S[j], h);
+        for (int j = 0; j < 4; ++j) sv[j] = lane_of(rx.soft(j), h);
         *reinterpret_cast<uint2*>(a.dW + e0[h]) = pack4(dv, sv);
       }
     }
@@ -643,7 +686,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksFwd) roi_slice_fwd_kernel(
 
 template <int N, int M, bool TAU1>
 __global__ void __launch_bounds__(kThreads, kMinBlocksBwd<M>) roi_slice_bwd_kernel(SliceArgs a) {
-  extern __shared__ __align__(128) uint8_t smem[];
+  uint8_t* smem = roi_slice_smem;
   TileSrc<3> src;
   src.ptr[0] = reinterpret_cast<const uint8_t*>(a.phi);
   src.esize[0] = 4;
@@ -663,8 +706,12 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksBwd<M>) roi_slice_bwd_kern
         const uint16_t* pw[2] = {sW + 4 * s0, sW + 4 * s1};
         const uint16_t* pd[2] = {sdW + 4 * s0, sdW + 4 * s1};
         const int64_t e0[2] = {base + 4 * s0, base + 4 * s1};
+        if constexpr (kPairedBwd<M>) {
+          bwd_slots<N, M, TAU1, F2>(pp, pw, pd, e0, true, a);
+        } else {
 #pragma unroll 1
-        for (int j = 0; j < 2; ++j) bwd_slots<N, M, TAU1, float>(pp + j, pw + j, pd + j, e0 + j, true, a);
+          for (int j = 0; j < 2; ++j) bwd_slots<N, M, TAU1, float>(pp + j, pw + j, pd + j, e0 + j, true, a);
+        }
       });
   if (ok && blockIdx.x == gridDim.x - 1) {
     const int64_t t0 = a.full_tiles * kTile;
@@ -713,8 +760,9 @@ int slice_fwd(const SliceArgs& a, cudaStream_t stream, bool pdl) {
 template <int N, int M, bool TAU1>
 int slice_bwd(const SliceArgs& a, cudaStream_t stream, bool pdl) {
   static LaunchCache cache;
-  return launch_persistent(roi_slice_bwd_kernel<N, M, TAU1>, cache, tile_smem_bytes<kTile, kStagesBwd>(8), a, stream,
-                           pdl);
+  constexpr size_t smem = kSliceHistOffset<M> + kSliceHistBytes<N, M>;
+  static_assert(smem <= 232448, "shared memory per CTA");
+  return launch_persistent(roi_slice_bwd_kernel<N, M, TAU1>, cache, smem, a, stream, pdl);
 }
 
 template <int N, int M>
