@@ -292,9 +292,9 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
 #pragma unroll
     for (int l = 0; l < M; ++l) dk[l] = lane_of(dkv[l], h);
     if ((fg.flag >> h) & 1u) {
-      // rare: the exact routine (with HIST from re-formed keys of this group; the
-      // opaque copy of the parameters keeps the compiler from holding the first
-      // keys live)
+      // rare: the log2-domain or (non-finite keys) the exact routine, with HIST
+      // from re-formed keys of this group (the opaque copy of the parameters keeps
+      // the compiler from holding the first keys live)
       float k[M], cc[M], S[M];
       if constexpr (HIST) {
         NoiseParams np = a.np;
@@ -305,13 +305,18 @@ __device__ __forceinline__ void bwd_groups(const float* const* phi_g, const uint
         for (int l = 0; l < M; ++l) k[l] = lane_of(kap[l], h);
       }
 #pragma unroll
-      for (int l = 0; l < M; ++l) {
-        k[l] *= kLn2;  // natural-log keys
-        cc[l] = lane_of(c[l], h);
+      for (int l = 0; l < M; ++l) cc[l] = lane_of(c[l], h);
+      if (!TAU1 && all_finite(k)) {
+        RobustGroup<N, M> rg;  // finite keys spread beyond the fast path's float range (as roi_fwd.cu)
+        rg.forward(k, a.inv_tau, S);
+        rg.backward(cc, a.inv_tau, dk);
+      } else {
+#pragma unroll
+        for (int l = 0; l < M; ++l) k[l] *= kLn2;  // natural-log keys
+        ExactGroup<N, M> ex;
+        ex.forward(k, N, M, a.tau, S);
+        ex.backward(cc, N, M, a.tau, dk);
       }
-      ExactGroup<N, M> ex;
-      ex.forward(k, N, M, a.tau, S);
-      ex.backward(cc, N, M, a.tau, dk);
 #pragma unroll
       for (int l = 0; l < M; ++l) dk[l] = __fmul_rn(dk[l], a.np.inv_lam);
       if (!ST && a.dW != nullptr) {

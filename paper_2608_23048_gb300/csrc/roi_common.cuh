@@ -474,6 +474,133 @@ struct ExactGroup {
 };
 
 // ---------------------------------------------------------------------------
+// Log2-domain relaxation of one group whose keys are finite but spread beyond
+// the fast path's float range (compile-time N, M; the fast kernels' fallback).
+// The same recursion as ExactGroup, in log2 units z = t / tau (t: keys in log2
+// units), with the hardware exp2 / log2: every log-sum-exp, and every exclusive
+// one (over all members but l), is formed against its own maximum, so no sum
+// underflows whatever the spread; O(M^2) exponentials per step.  mu and the
+// softmax-without-i weights nu do not depend on the base, so the backward below
+// is ExactGroup's (the oracle's bounded form) and returns dL/dkappa as it does.
+// ---------------------------------------------------------------------------
+template <int M>
+__device__ __forceinline__ void lse2_excluding_each(const float (&x)[M], float (&out)[M]) {
+  float pre[M], suf[M];  // maxima of the members before / after l
+  pre[0] = -INFINITY;
+#pragma unroll
+  for (int l = 1; l < M; ++l) pre[l] = fmaxf(pre[l - 1], x[l - 1]);
+  suf[M - 1] = -INFINITY;
+#pragma unroll
+  for (int l = M - 2; l >= 0; --l) suf[l] = fmaxf(suf[l + 1], x[l + 1]);
+#pragma unroll
+  for (int l = 0; l < M; ++l) {
+    const float m = fmaxf(pre[l], suf[l]);
+    float s = 0.0f;
+#pragma unroll
+    for (int i = 0; i < M; ++i)
+      if (i != l) s = __fadd_rn(s, ex2_approx(__fsub_rn(x[i], m)));
+    out[l] = __fadd_rn(m, lg2_approx(s));
+  }
+}
+
+template <int N, int M>
+struct RobustGroup {
+  float zh[N][M];  // z entering each step, shifted so its maximum is 0
+
+  // mu = softmax of z (log2 units); returns log2 of the normaliser against max 0
+  static __device__ __forceinline__ float softmax2(const float (&z)[M], float (&mu)[M]) {
+    float s = 0.0f;
+#pragma unroll
+    for (int l = 0; l < M; ++l) {
+      mu[l] = ex2_approx(z[l]);
+      s = __fadd_rn(s, mu[l]);
+    }
+    const float r = rcp_approx(s);
+#pragma unroll
+    for (int l = 0; l < M; ++l) mu[l] = __fmul_rn(mu[l], r);
+    return lg2_approx(s);
+  }
+
+  // t: the keys in log2 units (t = kappa log2 e), all finite.  Fills S.
+  __device__ __forceinline__ void forward(const float (&t)[M], float inv_tau, float (&S)[M]) {
+    float z[M], zmax = -INFINITY;
+#pragma unroll
+    for (int l = 0; l < M; ++l) {
+      z[l] = __fmul_rn(t[l], inv_tau);
+      zmax = fmaxf(zmax, z[l]);
+      S[l] = 0.0f;
+    }
+#pragma unroll
+    for (int k = 0; k < N; ++k) {
+#pragma unroll
+      for (int l = 0; l < M; ++l) {
+        z[l] = __fsub_rn(z[l], zmax);
+        zh[k][l] = z[l];
+      }
+      float mu[M];
+      const float lz = softmax2(z, mu);
+#pragma unroll
+      for (int l = 0; l < M; ++l) S[l] = __fadd_rn(S[l], mu[l]);
+      if (k + 1 < N) {
+        // z_l += log2(1 - mu_l) / tau, log2(1 - mu_l) = LSE2 over the others - LSE2 of all
+        float lx[M];
+        lse2_excluding_each(z, lx);
+        zmax = -INFINITY;
+#pragma unroll
+        for (int l = 0; l < M; ++l) {
+          z[l] = __fmaf_rn(__fsub_rn(lx[l], lz), inv_tau, z[l]);
+          zmax = fmaxf(zmax, z[l]);
+        }
+      }
+    }
+  }
+
+  // After forward(): dk = dL/dkappa for c = dL/dS.
+  __device__ __forceinline__ void backward(const float (&c)[M], float inv_tau, float (&dk)[M]) const {
+    float b[M];
+#pragma unroll
+    for (int l = 0; l < M; ++l) b[l] = 0.0f;
+#pragma unroll
+    for (int k = N - 1; k >= 0; --k) {
+      const float(&z)[M] = zh[k];
+      float mu[M], gz[M];
+      softmax2(z, mu);
+      float cmu = 0.0f, B = 0.0f;
+#pragma unroll
+      for (int l = 0; l < M; ++l) {
+        cmu = __fmaf_rn(c[l], mu[l], cmu);
+        B = __fadd_rn(B, b[l]);
+      }
+#pragma unroll
+      for (int l = 0; l < M; ++l) gz[l] = __fmul_rn(mu[l], __fsub_rn(__fsub_rn(c[l], cmu), B));
+      if (k + 1 < N) {
+        // (J^T b)_l adds sum over i != l of b_i nu(-i)_l, nu(-i)_l = 2^(z_l - LSE2 over j != i)
+        float lx[M];
+        lse2_excluding_each(z, lx);
+#pragma unroll
+        for (int i = 0; i < M; ++i)
+#pragma unroll
+          for (int l = 0; l < M; ++l)
+            if (l != i) gz[l] = __fmaf_rn(b[i], ex2_approx(__fsub_rn(z[l], lx[i])), gz[l]);
+      }
+#pragma unroll
+      for (int l = 0; l < M; ++l) b[l] = __fmaf_rn(gz[l], inv_tau, b[l]);
+    }
+#pragma unroll
+    for (int l = 0; l < M; ++l) dk[l] = b[l];
+  }
+};
+
+// True if every key of a group is finite.
+template <int M>
+__device__ __forceinline__ bool all_finite(const float (&k)[M]) {
+  float s = 0.0f;
+#pragma unroll
+  for (int l = 0; l < M; ++l) s += k[l] - k[l];  // 0 for finite keys, NaN otherwise
+  return s == 0.0f;
+}
+
+// ---------------------------------------------------------------------------
 // Fast register-resident relaxation of one group (V = float) or of two groups in
 // lockstep (V = F2, one per half), M <= 8, held by one thread.
 //

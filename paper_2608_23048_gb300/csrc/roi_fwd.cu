@@ -182,8 +182,16 @@ __device__ __forceinline__ void fwd_finish(const V (&kap)[M], const uint16_t* co
             bits[h] = topn_bits<M>(k, N);
           }
         }
-        ExactGroup<N, M> ex;
-        ex.forward(kn, N, M, a.tau, S[h]);
+        // finite keys spread beyond the fast path's float range (tau != 1: at tau = 1
+        // that takes a key gap of ~69 natural-log units, and the tau = 1 kernels keep
+        // their code to the exact routine)
+        if (!TAU1 && all_finite(k)) {
+          RobustGroup<N, M> rg;
+          rg.forward(k, a.inv_tau, S[h]);
+        } else {
+          ExactGroup<N, M> ex;
+          ex.forward(kn, N, M, a.tau, S[h]);
+        }
       }
     }
   }

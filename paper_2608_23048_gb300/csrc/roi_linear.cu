@@ -185,11 +185,20 @@ __device__ __forceinline__ void chunk_masked_weights(const LinArgs& a, uint8_t* 
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
       if ((fg.flag >> h) & 1u) {
-        float kn[M];
+        // the mask forward's fallback, so Wm stays its bit for bit
+        float k[M], kn[M];
 #pragma unroll
-        for (int l = 0; l < M; ++l) kn[l] = lane_of(kap[l], h) * kLn2;  // natural-log keys
-        ExactGroup<N, M> ex;
-        ex.forward(kn, N, M, a.tau, S[h]);
+        for (int l = 0; l < M; ++l) {
+          k[l] = lane_of(kap[l], h);
+          kn[l] = k[l] * kLn2;  // natural-log keys
+        }
+        if (!TAU1 && all_finite(k)) {
+          RobustGroup<N, M> rg;
+          rg.forward(k, a.inv_tau, S[h]);
+        } else {
+          ExactGroup<N, M> ex;
+          ex.forward(kn, N, M, a.tau, S[h]);
+        }
       }
     }
   }
