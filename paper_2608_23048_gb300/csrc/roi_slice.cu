@@ -167,6 +167,8 @@ __device__ __forceinline__ void slot_keys(const float* const* p4, const int64_t*
 // Forward relaxation of the group(s) held by this slice; mu of every step kept
 // if KEEP.  forward() returns the fallback flags (bit h: lane h of V), uniform
 // over the slice.
+constexpr float kTinyTotal = 7.52316384526264e-37f;  // 2^-120
+
 template <int N, int M, bool TAU1, bool KEEP, class V>
 struct SliceRelax {
   static constexpr int SL = M / 4;
@@ -258,14 +260,21 @@ struct SliceRelax {
           if constexpr (!KEEP) S[j] = k == 0 ? cur[j] : vadd(S[j], cur[j]);
         }
         if (k + 1 < N) {
-          V ex[4];
+          // d_l += log2(1 - mu_l) / tau, the offsets first renormalised by log2 of the
+          // total (so sum 2^d = 1, every offset <= 0 and the largest >= -log2 M): the
+          // total comes from the butterfly above, so no maximum over the slice is
+          // needed on the step's critical path.  A group whose exclusive sums drop
+          // below 2^-100 of the total, or whose total drops below 2^-120 (offsets that
+          // fell too far in one step, possible only for tau well below 0.05), goes
+          // to the exact routine.
+          V ex[4], om[4];
           excl4(e, oth, ex);
-          flag |= vbelow(min4(ex), kTinyExcl);
 #pragma unroll
-          for (int j = 0; j < 4; ++j) d[j] = vfma(vmap(vmul(ex[j], r), lg2_approx), sc, d[j]);
-          const V dm = Slice<SL, V>::max(max4(d));
+          for (int j = 0; j < 4; ++j) om[j] = vmul(ex[j], r);
+          flag |= vbelow(min4(om), kTinyExcl) | vbelow(tot, kTinyTotal);
+          const V lz = vmap(tot, lg2_approx);
 #pragma unroll
-          for (int j = 0; j < 4; ++j) d[j] = vsub(d[j], dm);
+          for (int j = 0; j < 4; ++j) d[j] = vfma(vmap(om[j], lg2_approx), sc, vsub(d[j], lz));
         }
       }
     }
