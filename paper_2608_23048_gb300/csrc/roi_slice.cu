@@ -17,7 +17,10 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kTile = 2048;  // 512 four-member slots: slots t and t + 256 per thread
 constexpr int kStagesFwd = 4;
-constexpr int kStagesBwd = 3;
+// backward ring stages: two at 8:16, whose two CTAs per SM also hold their step
+// histories in shared memory, three at 16:32 (one CTA per SM)
+template <int M>
+constexpr int kStagesBwd = M == 16 ? 2 : 3;
 // Both directions relax the two slots of a thread in lockstep on packed FP32; the
 // backward keeps its step history in shared memory behind the tile ring.  CTAs per
 // SM the registers are sized for (measured on the 3B-shaped set, tau = 0.2):
@@ -32,11 +35,12 @@ template <int M>
 constexpr int kMinBlocksBwd = M == 32 ? 1 : 2;
 // The backward's step history: steps 0 .. N-2 of one slot, or of the two slots of
 // a pair (four floats or F2 a step), per thread, thread-strided so a warp touches
-// consecutive words; the last step stays in registers.
+// consecutive words; the last step stays in registers.  Behind it, per step, the
+// sum of mu over the slice's other lanes, which the sweep needs for 1 - mu.
 template <int M>
-constexpr size_t kSliceHistOffset = (tile_smem_bytes<kTile, kStagesBwd>(8) + 15) & ~size_t(15);
+constexpr size_t kSliceHistOffset = (tile_smem_bytes<kTile, kStagesBwd<M>>(8) + 15) & ~size_t(15);
 template <int N, int M>
-constexpr size_t kSliceHistBytes = size_t(N - 1) * 4 * (kPairedBwd<M> ? 8 : 4) * kThreads;
+constexpr size_t kSliceHistBytes = size_t(N - 1) * 5 * (kPairedBwd<M> ? 8 : 4) * kThreads;
 
 __device__ __forceinline__ float shfl_xor(float v, int o) { return __shfl_xor_sync(0xffffffffu, v, o); }
 __device__ __forceinline__ F2 shfl_xor(F2 v, int o) {
@@ -186,6 +190,9 @@ struct SliceRelax {
     }
   }
   __device__ __forceinline__ V get(int k, int j) const { return k == N - 1 ? mu_last[j] : hist[(4 * k + j) * kThreads]; }
+  // the other lanes' sum of mu of step k < N - 1, kept by forward() for the sweep
+  __device__ __forceinline__ void put_oth(int k, V v) { hist[(4 * (N - 1) + k) * kThreads] = v; }
+  __device__ __forceinline__ V get_oth(int k) const { return hist[(4 * (N - 1) + k) * kThreads]; }
   __device__ __forceinline__ void get4(int k, V (&m)[4]) const {
 #pragma unroll
     for (int j = 0; j < 4; ++j) m[j] = get(k, j);
@@ -229,6 +236,7 @@ struct SliceRelax {
         if (k + 1 < N) {
           V totc, o[4], v[4];
           const V oth = Slice<SL, V>::others(sum4(cur), totc);
+          if constexpr (KEEP) put_oth(k, oth);
           excl4(cur, oth, o);
 #pragma unroll
           for (int j = 0; j < 4; ++j) v[j] = vmul(cur[j], o[j]);
@@ -253,6 +261,9 @@ struct SliceRelax {
         V tot;
         const V oth = Slice<SL, V>::others(sum4(e), tot);
         const V r = vmap(tot, rcp_approx);
+        if constexpr (KEEP) {
+          if (k + 1 < N) put_oth(k, vmul(oth, r));
+        }
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           cur[j] = vmul(e[j], r);
@@ -307,8 +318,8 @@ struct SliceRelax {
 #pragma unroll
         for (int j = 0; j < 4; ++j) h[j] = hl[j];
       } else {
-        V om[4], tmp;
-        excl4(mk, Slice<SL, V>::others(sum4(mk), tmp), om);
+        V om[4];
+        excl4(mk, get_oth(k), om);
 #pragma unroll
         for (int j = 0; j < 4; ++j) h[j] = vmul(b[j], vmap(om[j], rcp_approx));
       }
@@ -704,7 +715,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksBwd<M>) roi_slice_bwd_kern
   src.ptr[2] = reinterpret_cast<const uint8_t*>(a.dWm);
   src.esize[2] = 2;
   pdl_launch_dependents();
-  const bool ok = run_tiles<kThreads, kTile, kStagesBwd, 3>(
+  const bool ok = run_tiles<kThreads, kTile, kStagesBwd<M>, 3>(
       smem, src, a.full_tiles, a.status, [&](const uint8_t* const* stage, int64_t tile) {
         const float* sphi = reinterpret_cast<const float*>(stage[0]);
         const uint16_t* sW = reinterpret_cast<const uint16_t*>(stage[1]);

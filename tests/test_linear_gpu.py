@@ -144,7 +144,13 @@ def test_prologue_wm_is_the_mask_forward(roi):
     rows, cols, T = 256, 1024, 32
     W, phi, _ = WL.make_inputs(rows, cols, "logw", 21)
     X = WL.make_tokens(T, cols, 21)
-    for N, M, tau in ((2, 4, 1.0), (4, 8, 1.0), (2, 8, 0.7)):
+    # outlier logits (about one in eight shifted by +-100): groups for both fallbacks
+    g = torch.Generator().manual_seed(21)
+    shift = torch.randint(0, 16, phi.shape, generator=g)
+    wide = (phi + 100.0 * (shift == 0).float() - 100.0 * (shift == 1).float()).contiguous()
+    for N, M, tau, ph in ((2, 4, 1.0, phi), (4, 8, 1.0, phi), (2, 8, 0.7, phi), (2, 4, 0.3, wide),
+                          (4, 8, 0.5, wide), (2, 4, 1.0, wide)):
+        phi = ph
         st = roi.NoiseState(5, 9, 1, 1.0, 0)
         Y = gpu_linear(roi, X, phi, W, N, M, tau, st)
         Wm = torch.empty(rows, cols, dtype=torch.bfloat16, device="cuda")
