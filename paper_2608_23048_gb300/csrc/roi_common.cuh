@@ -601,6 +601,51 @@ __device__ __forceinline__ bool all_finite(const float (&k)[M]) {
 }
 
 // ---------------------------------------------------------------------------
+// Groups the fast path leaves to an exact routine, deferred: each warp queues their
+// first element indices in its own CAP entries of shared memory and, once 32 are
+// queued (checked between tiles) or at the end of its work, handles them one per
+// lane.  The exact routines then run on every lane of the warp, and their code sits
+// outside the fast path's loop body instead of inside it.  All 32 lanes call
+// push() and drain() together; `n` is the same on every lane.
+// ---------------------------------------------------------------------------
+template <int CAP>
+struct DeferredGroups {
+  uint32_t base;  // shared-memory address of this warp's entries
+  int n;
+
+  __device__ __forceinline__ void init(const void* entries) {
+    base = static_cast<uint32_t>(__cvta_generic_to_shared(entries)) + (threadIdx.x >> 5) * CAP * 8;
+    n = 0;
+  }
+  // Queues g for the lanes with `want` (at most CAP - n of them in all).
+  __device__ __forceinline__ void push(bool want, int64_t g) {
+    const uint32_t m = __ballot_sync(0xffffffffu, want);
+    if (want) {
+      const uint32_t at = base + 8u * uint32_t(n + __popc(m & ((1u << (threadIdx.x & 31)) - 1u)));
+      asm volatile("st.shared.u64 [%0], %1;" ::"r"(at), "l"(g) : "memory");
+    }
+    n += __popc(m);
+  }
+  // Handles queued groups 32 at a time (all of them if `all`), fn(g) on one lane each.
+  template <class Fn>
+  __device__ __forceinline__ void drain(bool all, Fn&& fn) {
+    if (n < 32 && !(all && n > 0)) return;
+    __syncwarp();
+    const int lane = threadIdx.x & 31;
+    do {
+      const int k = n < 32 ? n : 32;
+      if (lane < k) {
+        int64_t g;
+        asm volatile("ld.shared.u64 %0, [%1];" : "=l"(g) : "r"(base + 8u * uint32_t(n - k + lane)) : "memory");
+        fn(g);
+      }
+      n -= k;
+      __syncwarp();
+    } while (n >= 32 || (all && n > 0));
+  }
+};
+
+// ---------------------------------------------------------------------------
 // Fast register-resident relaxation of one group (V = float) or of two groups in
 // lockstep (V = F2, one per half), M <= 8, held by one thread.
 //

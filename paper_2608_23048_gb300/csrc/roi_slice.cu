@@ -6,8 +6,8 @@
 // subtracts.  A thread holds the slots t and t + 256 of a tile; where registers
 // allow, the two groups of those slots are relaxed in lockstep on packed FP32
 // (V = F2, one group per half), otherwise one after the other (V = float).
-// Groups whose keys leave the fast path's range go to ExactGroup, run by the
-// slice's first lane.
+// Groups whose keys leave the fast path's range are queued by the slice's first
+// lane (DeferredGroups) and handled 32 at a time, one per lane, by ExactGroup.
 #include "roi_launch.h"
 #include "roi_tiles.cuh"
 
@@ -39,8 +39,25 @@ constexpr int kMinBlocksBwd = M == 32 ? 1 : 2;
 // sum of mu over the slice's other lanes, which the sweep needs for 1 - mu.
 template <int M>
 constexpr size_t kSliceHistOffset = (tile_smem_bytes<kTile, kStagesBwd<M>>(8) + 15) & ~size_t(15);
+template <int M>
+constexpr bool kReloadHist = M == 16;
+// Deferred exact-routine groups (DeferredGroups): a warp queues at most 64 / SL
+// groups per tile (or per round of the ragged tail) and drains once 32 are queued.
+constexpr int kDeferCap = 48;
+// DEFER: the kernels queue flagged groups (DeferredGroups) instead of running the
+// exact routine in place.  8:16 always defers.  16:32 defers only for tau < 0.15:
+// there (the paper anneals tau to 0.05) a few per cent of the groups leave the fast
+// path's range (key gaps beyond ~69 tau natural-log units) and the queued routine
+// runs 15x faster per step than in place; above it no group does, and the 16:32
+// kernels, at 255 registers and one CTA per SM, measured 10 % slower with the
+// queue's code than with the exact routine in place.
+constexpr float kDeferBelowTau = 0.15f;
+constexpr size_t kDeferBytes = size_t(kDeferCap) * 8 * (kThreads / 32);
+constexpr size_t kFwdDeferOffset = (tile_smem_bytes<kTile, kStagesFwd>(6) + 15) & ~size_t(15);
 template <int N, int M>
 constexpr size_t kSliceHistBytes = size_t(N - 1) * 5 * (kPairedBwd<M> ? 8 : 4) * kThreads;
+template <int N, int M>
+constexpr size_t kSliceDeferOffset = (kSliceHistOffset<M> + kSliceHistBytes<N, M> + 15) & ~size_t(15);
 
 __device__ __forceinline__ float shfl_xor(float v, int o) { return __shfl_xor_sync(0xffffffffu, v, o); }
 __device__ __forceinline__ F2 shfl_xor(F2 v, int o) {
@@ -450,8 +467,8 @@ __device__ __forceinline__ void slot_topn(const V (&kap)[4], int base_lane, int 
   }
 }
 
-// Exact fallback for one whole group, run by one lane: natural-log keys of all
-// M elements from logits at phi_g (call-flat index g0).
+// The keys of all M elements of one group, in natural-log units, from logits at
+// phi_g (call-flat index g0), by one lane.
 template <int N, int M>
 __device__ __forceinline__ void group_keys_all(const float* phi_g, int64_t g0, const NoiseParams& np, float (&k)[M]) {
 #pragma unroll 1
@@ -478,13 +495,68 @@ __device__ __forceinline__ void unpack_bf16x4(uint2 q, float (&out)[4]) {
   out[3] = bf16_bits_to_float(q.y >> 16);
 }
 
+// The exact routine for one group (first element g0, call-flat), from global
+// memory: the forward's outputs (Wm unless straight-through, soft).
+template <int N, int M>
+__device__ __forceinline__ void exact_group_fwd(int64_t g0, const SliceArgs& a) {
+  if (a.soft == nullptr && a.st) return;
+  float k[M], S[M];
+  group_keys_all<N, M>(a.phi + g0, g0, a.np, k);
+  ExactGroup<N, M> ex;
+  ex.forward(k, N, M, a.tau, S);
+#pragma unroll 1
+  for (int s = 0; s < M / 4; ++s) {
+    float wv[4], sv[4];
+    unpack_bf16x4(*reinterpret_cast<const uint2*>(a.W + g0 + 4 * s), wv);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) sv[j] = S[4 * s + j];
+    if (!a.st) *reinterpret_cast<uint2*>(a.Wm + g0 + 4 * s) = pack4(wv, sv);
+    if (a.soft != nullptr) *reinterpret_cast<float4*>(a.soft + g0 + 4 * s) = make_float4(sv[0], sv[1], sv[2], sv[3]);
+  }
+}
+// The backward's outputs of one group: dphi, the fused AdamW step, dW unless the
+// straight-through variant (which wrote it with the fast path).  The group's logits
+// are untouched until here (the fast path skips its AdamW step).
+template <int N, int M>
+__device__ __forceinline__ void exact_group_bwd(int64_t g0, const SliceArgs& a) {
+  float k[M], cc[M], S[M], dkk[M];
+  group_keys_all<N, M>(a.phi + g0, g0, a.np, k);
+#pragma unroll 1
+  for (int s = 0; s < M / 4; ++s) {
+    float wv[4], dv[4];
+    unpack_bf16x4(*reinterpret_cast<const uint2*>(a.W + g0 + 4 * s), wv);
+    unpack_bf16x4(*reinterpret_cast<const uint2*>(a.dWm + g0 + 4 * s), dv);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) cc[4 * s + j] = __fmul_rn(dv[j], wv[j]);
+  }
+  ExactGroup<N, M> ex;
+  ex.forward(k, N, M, a.tau, S);
+  ex.backward(cc, N, M, a.tau, dkk);
+#pragma unroll 1
+  for (int s = 0; s < M / 4; ++s) {
+    const int64_t e = g0 + 4 * s;
+    const float g4[4] = {__fmul_rn(dkk[4 * s], a.np.inv_lam), __fmul_rn(dkk[4 * s + 1], a.np.inv_lam),
+                         __fmul_rn(dkk[4 * s + 2], a.np.inv_lam), __fmul_rn(dkk[4 * s + 3], a.np.inv_lam)};
+    if (a.dphi != nullptr) *reinterpret_cast<float4*>(a.dphi + e) = make_float4(g4[0], g4[1], g4[2], g4[3]);
+    if (a.phi_out != nullptr) adamw4(a.phi_out, a.m, a.v, e, *reinterpret_cast<const float4*>(a.phi + e), g4, a.opt);
+    if (a.dW != nullptr && a.hard_in == nullptr) {
+      float dv[4], sv[4];
+      unpack_bf16x4(*reinterpret_cast<const uint2*>(a.dWm + e), dv);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) sv[j] = S[4 * s + j];
+      *reinterpret_cast<uint2*>(a.dW + e) = pack4(dv, sv);
+    }
+  }
+}
+
 // Forward of L slots (one per lane of V; p/w: each slot's logits and weights in
 // shared or global memory, e0: call-flat index of its first element).  All 32
 // lanes of the warp call this together; inactive slots (ragged tail, V = float
 // only) take part in the shuffles with zero keys.  Returns each slot's hard bits.
-template <int N, int M, bool TAU1, class V>
+template <int N, int M, bool TAU1, bool DEFER, class V>
 __device__ __forceinline__ void fwd_slots(const float* const* p, const uint16_t* const* w, const int64_t* e0,
-                                          bool active, const SliceArgs& a, uint32_t (&bits)[vlanes<V>()]) {
+                                          bool active, const SliceArgs& a, uint32_t (&bits)[vlanes<V>()],
+                                          uint32_t& defer) {
   constexpr int SL = M / 4;
   constexpr int L = vlanes<V>();
   const int lane = threadIdx.x & 31;
@@ -500,6 +572,9 @@ __device__ __forceinline__ void fwd_slots(const float* const* p, const uint16_t*
   slot_topn<N, M, V>(kap, base_lane, q, bits);
   SliceRelax<N, M, TAU1, false, V> rx;
   const uint32_t flag = rx.forward(kap, a.inv_tau, base_lane);
+  // groups out of the fast path's range: queued by their first lane for the exact
+  // routine, which writes their outputs
+  defer = DEFER && active && q == 0 ? flag : 0u;
   if (!active) return;
 #pragma unroll
   for (int h = 0; h < L; ++h) {
@@ -512,29 +587,16 @@ __device__ __forceinline__ void fwd_slots(const float* const* p, const uint16_t*
       for (int j = 0; j < 4; ++j) sv[j] = lane_of(rx.S[j], h);
       if (!a.st) *reinterpret_cast<uint2*>(a.Wm + e0[h]) = pack4(wv, sv);
       if (a.soft != nullptr) *reinterpret_cast<float4*>(a.soft + e0[h]) = make_float4(sv[0], sv[1], sv[2], sv[3]);
-    } else if (q == 0 && (a.soft != nullptr || !a.st)) {
-      float k[M], S[M];
-      group_keys_all<N, M>(p[h], e0[h], a.np, k);
-      ExactGroup<N, M> ex;
-      ex.forward(k, N, M, a.tau, S);
-#pragma unroll 1
-      for (int s = 0; s < SL; ++s) {
-        float wv[4], sv[4];
-        unpack_bf16x4(*reinterpret_cast<const uint2*>(w[h] + 4 * s), wv);
-#pragma unroll
-        for (int j = 0; j < 4; ++j) sv[j] = S[4 * s + j];
-        if (!a.st) *reinterpret_cast<uint2*>(a.Wm + e0[h] + 4 * s) = pack4(wv, sv);
-        if (a.soft != nullptr)
-          *reinterpret_cast<float4*>(a.soft + e0[h] + 4 * s) = make_float4(sv[0], sv[1], sv[2], sv[3]);
-      }
+    } else if constexpr (!DEFER) {
+      if (q == 0) exact_group_fwd<N, M>(e0[h], a);
     }
   }
 }
 
 // Backward of L slots (as fwd_slots).
-template <int N, int M, bool TAU1, class V>
+template <int N, int M, bool TAU1, bool DEFER, class V>
 __device__ __forceinline__ void bwd_slots(const float* const* p, const uint16_t* const* w, const uint16_t* const* dw,
-                                          const int64_t* e0, bool active, const SliceArgs& a) {
+                                          const int64_t* e0, bool active, const SliceArgs& a, uint32_t& defer) {
   constexpr int SL = M / 4;
   constexpr int L = vlanes<V>();
   const int lane = threadIdx.x & 31;
@@ -564,6 +626,7 @@ __device__ __forceinline__ void bwd_slots(const float* const* p, const uint16_t*
   SliceRelax<N, M, TAU1, true, V> rx;
   rx.hist = reinterpret_cast<V*>(roi_slice_smem + kSliceHistOffset<M>) + threadIdx.x;
   const uint32_t flag = rx.forward(kap, a.inv_tau, base_lane);
+  defer = DEFER && active && q == 0 ? flag : 0u;
   if (active && a.dW != nullptr) {
 #pragma unroll
     for (int h = 0; h < L; ++h) {
@@ -580,6 +643,10 @@ __device__ __forceinline__ void bwd_slots(const float* const* p, const uint16_t*
     }
   }
   V dk[4];
+  // 8:16: the sweep re-reads the step history from shared memory (a compiler memory
+  // barrier here keeps the forward's values from being carried in registers, which
+  // spills at two CTAs per SM); 16:32 runs one CTA per SM and keeps them in registers.
+  if constexpr (kReloadHist<M>) asm volatile("" ::: "memory");
   rx.backward(c, a.inv_tau, dk);
   if (!active) return;
   if (a.np.inv_lam != 1.0f) {  // lambda = 1: nothing to scale, the same bits
@@ -592,36 +659,8 @@ __device__ __forceinline__ void bwd_slots(const float* const* p, const uint16_t*
       const float g4[4] = {lane_of(dk[0], h), lane_of(dk[1], h), lane_of(dk[2], h), lane_of(dk[3], h)};
       if (a.dphi != nullptr) *reinterpret_cast<float4*>(a.dphi + e0[h]) = make_float4(g4[0], g4[1], g4[2], g4[3]);
       if (a.phi_out != nullptr) adamw4(a.phi_out, a.m, a.v, e0[h], *reinterpret_cast<const float4*>(p[h]), g4, a.opt);
-    } else if (q == 0) {
-      float k[M], cc[M], S[M], dkk[M];
-      group_keys_all<N, M>(p[h], e0[h], a.np, k);
-#pragma unroll 1
-      for (int s = 0; s < SL; ++s) {
-        float wv[4], dv[4];
-        unpack_bf16x4(*reinterpret_cast<const uint2*>(w[h] + 4 * s), wv);
-        unpack_bf16x4(*reinterpret_cast<const uint2*>(dw[h] + 4 * s), dv);
-#pragma unroll
-        for (int j = 0; j < 4; ++j) cc[4 * s + j] = __fmul_rn(dv[j], wv[j]);
-      }
-      ExactGroup<N, M> ex;
-      ex.forward(k, N, M, a.tau, S);
-      ex.backward(cc, N, M, a.tau, dkk);
-#pragma unroll 1
-      for (int s = 0; s < SL; ++s) {
-        const float g4[4] = {__fmul_rn(dkk[4 * s], a.np.inv_lam), __fmul_rn(dkk[4 * s + 1], a.np.inv_lam),
-                             __fmul_rn(dkk[4 * s + 2], a.np.inv_lam), __fmul_rn(dkk[4 * s + 3], a.np.inv_lam)};
-        if (a.dphi != nullptr)
-          *reinterpret_cast<float4*>(a.dphi + e0[h] + 4 * s) = make_float4(g4[0], g4[1], g4[2], g4[3]);
-        if (a.phi_out != nullptr)
-          adamw4(a.phi_out, a.m, a.v, e0[h] + 4 * s, reinterpret_cast<const float4*>(p[h])[s], g4, a.opt);
-        if (a.dW != nullptr && a.hard_in == nullptr) {
-          float dv[4], sv[4];
-          unpack_bf16x4(*reinterpret_cast<const uint2*>(dw[h] + 4 * s), dv);
-#pragma unroll
-          for (int j = 0; j < 4; ++j) sv[j] = S[4 * s + j];
-          *reinterpret_cast<uint2*>(a.dW + e0[h] + 4 * s) = pack4(dv, sv);
-        }
-      }
+    } else if constexpr (!DEFER) {
+      if (q == 0) exact_group_bwd<N, M>(e0[h], a);
     }
   }
 }
@@ -653,7 +692,7 @@ __device__ __forceinline__ void store_hard_slot_pair(uint32_t* hard, int64_t e0a
   if ((lane & 3) == 0) hard[(upper ? e0b : e0a) >> 5] = word;
 }
 
-template <int N, int M, bool TAU1>
+template <int N, int M, bool TAU1, bool DEFER>
 __global__ void __launch_bounds__(kThreads, kMinBlocksFwd) roi_slice_fwd_kernel(SliceArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   TileSrc<2> src;
@@ -661,6 +700,9 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksFwd) roi_slice_fwd_kernel(
   src.esize[0] = 4;
   src.ptr[1] = reinterpret_cast<const uint8_t*>(a.W);
   src.esize[1] = 2;
+  DeferredGroups<kDeferCap> dg;
+  dg.init(reinterpret_cast<int64_t*>(smem + kFwdDeferOffset));
+  const auto exact = [&](int64_t g0) { exact_group_fwd<N, M>(g0, a); };
   // a batch's next tensor may start on the SMs this launch frees (no-op otherwise)
   pdl_launch_dependents();
   const bool ok = run_tiles<kThreads, kTile, kStagesFwd, 2>(
@@ -672,18 +714,25 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksFwd) roi_slice_fwd_kernel(
         const float* pp[2] = {sphi + 4 * s0, sphi + 4 * s1};
         const uint16_t* pw[2] = {sW + 4 * s0, sW + 4 * s1};
         const int64_t e0[2] = {base + 4 * s0, base + 4 * s1};
-        uint32_t bits[2];
+        uint32_t bits[2], defer[2];
         if constexpr (kPairedFwd<M>) {
-          fwd_slots<N, M, TAU1, F2>(pp, pw, e0, true, a, bits);
+          uint32_t d2;
+          fwd_slots<N, M, TAU1, DEFER, F2>(pp, pw, e0, true, a, bits, d2);
+          defer[0] = d2 & 1u, defer[1] = d2 >> 1;
         } else {
 #pragma unroll 1
           for (int j = 0; j < 2; ++j) {
             uint32_t b1[1];
-            fwd_slots<N, M, TAU1, float>(pp + j, pw + j, e0 + j, true, a, b1);
+            fwd_slots<N, M, TAU1, DEFER, float>(pp + j, pw + j, e0 + j, true, a, b1, defer[j]);
             bits[j] = b1[0];
           }
         }
         if (a.hard != nullptr) store_hard_slot_pair(a.hard, e0[0], e0[1], bits[0], bits[1]);
+        if constexpr (DEFER) {
+          dg.push(defer[0] != 0u, e0[0]);
+          dg.push(defer[1] != 0u, e0[1]);
+          dg.drain(false, exact);
+        }
       });
   if (ok && blockIdx.x == gridDim.x - 1) {
     const int64_t t0 = a.full_tiles * kTile;
@@ -695,16 +744,23 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksFwd) roi_slice_fwd_kernel(
       const float* pp[1] = {a.phi + off};
       const uint16_t* pw[1] = {a.W + off};
       const int64_t e0[1] = {t0 + 4 * si};
-      uint32_t bits[1];
-      fwd_slots<N, M, TAU1, float>(pp, pw, e0, active, a, bits);
+      uint32_t bits[1], defer;
+      fwd_slots<N, M, TAU1, DEFER, float>(pp, pw, e0, active, a, bits, defer);
       if (a.hard != nullptr) store_hard_slot(a.hard, e0[0], bits[0], active);
+      if constexpr (DEFER) {
+        dg.push(defer != 0u, e0[0]);
+        dg.drain(false, exact);
+      }
     }
+  }
+  if constexpr (DEFER) {
+    if (ok) dg.drain(true, exact);
   }
   // the launch completes only after the batch's previous one (stream order)
   if (blockIdx.x == 0) pdl_wait();
 }
 
-template <int N, int M, bool TAU1>
+template <int N, int M, bool TAU1, bool DEFER>
 __global__ void __launch_bounds__(kThreads, kMinBlocksBwd<M>) roi_slice_bwd_kernel(SliceArgs a) {
   uint8_t* smem = roi_slice_smem;
   TileSrc<3> src;
@@ -714,6 +770,9 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksBwd<M>) roi_slice_bwd_kern
   src.esize[1] = 2;
   src.ptr[2] = reinterpret_cast<const uint8_t*>(a.dWm);
   src.esize[2] = 2;
+  DeferredGroups<kDeferCap> dg;
+  dg.init(reinterpret_cast<int64_t*>(smem + kSliceDeferOffset<N, M>));
+  const auto exact = [&](int64_t g0) { exact_group_bwd<N, M>(g0, a); };
   pdl_launch_dependents();
   const bool ok = run_tiles<kThreads, kTile, kStagesBwd<M>, 3>(
       smem, src, a.full_tiles, a.status, [&](const uint8_t* const* stage, int64_t tile) {
@@ -726,11 +785,20 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksBwd<M>) roi_slice_bwd_kern
         const uint16_t* pw[2] = {sW + 4 * s0, sW + 4 * s1};
         const uint16_t* pd[2] = {sdW + 4 * s0, sdW + 4 * s1};
         const int64_t e0[2] = {base + 4 * s0, base + 4 * s1};
+        uint32_t defer[2];
         if constexpr (kPairedBwd<M>) {
-          bwd_slots<N, M, TAU1, F2>(pp, pw, pd, e0, true, a);
+          uint32_t d2;
+          bwd_slots<N, M, TAU1, DEFER, F2>(pp, pw, pd, e0, true, a, d2);
+          defer[0] = d2 & 1u, defer[1] = d2 >> 1;
         } else {
 #pragma unroll 1
-          for (int j = 0; j < 2; ++j) bwd_slots<N, M, TAU1, float>(pp + j, pw + j, pd + j, e0 + j, true, a);
+          for (int j = 0; j < 2; ++j)
+            bwd_slots<N, M, TAU1, DEFER, float>(pp + j, pw + j, pd + j, e0 + j, true, a, defer[j]);
+        }
+        if constexpr (DEFER) {
+          dg.push(defer[0] != 0u, e0[0]);
+          dg.push(defer[1] != 0u, e0[1]);
+          dg.drain(false, exact);
         }
       });
   if (ok && blockIdx.x == gridDim.x - 1) {
@@ -744,8 +812,16 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksBwd<M>) roi_slice_bwd_kern
       const uint16_t* pw[1] = {a.W + off};
       const uint16_t* pd[1] = {a.dWm + off};
       const int64_t e0[1] = {t0 + 4 * si};
-      bwd_slots<N, M, TAU1, float>(pp, pw, pd, e0, active, a);
+      uint32_t defer;
+      bwd_slots<N, M, TAU1, DEFER, float>(pp, pw, pd, e0, active, a, defer);
+      if constexpr (DEFER) {
+        dg.push(defer != 0u, e0[0]);
+        dg.drain(false, exact);
+      }
     }
+  }
+  if constexpr (DEFER) {
+    if (ok) dg.drain(true, exact);
   }
   if (blockIdx.x == 0) pdl_wait();
 }
@@ -771,27 +847,39 @@ int launch_persistent(Kern kern, LaunchCache& cache, size_t smem, const SliceArg
   return launch_maybe_pdl(kern, grid, kThreads, smem, stream, pdl, a);
 }
 
-template <int N, int M, bool TAU1>
+template <int N, int M, bool TAU1, bool DEFER>
 int slice_fwd(const SliceArgs& a, cudaStream_t stream, bool pdl) {
   static LaunchCache cache;
-  return launch_persistent(roi_slice_fwd_kernel<N, M, TAU1>, cache, tile_smem_bytes<kTile, kStagesFwd>(6), a, stream,
+  return launch_persistent(roi_slice_fwd_kernel<N, M, TAU1, DEFER>, cache, kFwdDeferOffset + kDeferBytes, a, stream,
                            pdl);
 }
-template <int N, int M, bool TAU1>
+template <int N, int M, bool TAU1, bool DEFER>
 int slice_bwd(const SliceArgs& a, cudaStream_t stream, bool pdl) {
   static LaunchCache cache;
-  constexpr size_t smem = kSliceHistOffset<M> + kSliceHistBytes<N, M>;
+  constexpr size_t smem = kSliceDeferOffset<N, M> + kDeferBytes;
   static_assert(smem <= 232448, "shared memory per CTA");
-  return launch_persistent(roi_slice_bwd_kernel<N, M, TAU1>, cache, smem, a, stream, pdl);
+  return launch_persistent(roi_slice_bwd_kernel<N, M, TAU1, DEFER>, cache, smem, a, stream, pdl);
 }
 
 template <int N, int M>
 int slice_fwd_nm(const SliceArgs& a, cudaStream_t stream, bool pdl) {
-  return a.tau == 1.0f ? slice_fwd<N, M, true>(a, stream, pdl) : slice_fwd<N, M, false>(a, stream, pdl);
+  if (a.tau == 1.0f) return slice_fwd<N, M, true, M == 16>(a, stream, pdl);
+  if constexpr (M == 16) {
+    return slice_fwd<N, M, false, true>(a, stream, pdl);
+  } else {
+    return a.tau < kDeferBelowTau ? slice_fwd<N, M, false, true>(a, stream, pdl)
+                                  : slice_fwd<N, M, false, false>(a, stream, pdl);
+  }
 }
 template <int N, int M>
 int slice_bwd_nm(const SliceArgs& a, cudaStream_t stream, bool pdl) {
-  return a.tau == 1.0f ? slice_bwd<N, M, true>(a, stream, pdl) : slice_bwd<N, M, false>(a, stream, pdl);
+  if (a.tau == 1.0f) return slice_bwd<N, M, true, M == 16>(a, stream, pdl);
+  if constexpr (M == 16) {
+    return slice_bwd<N, M, false, true>(a, stream, pdl);
+  } else {
+    return a.tau < kDeferBelowTau ? slice_bwd<N, M, false, true>(a, stream, pdl)
+                                  : slice_bwd<N, M, false, false>(a, stream, pdl);
+  }
 }
 
 }  // namespace
