@@ -21,6 +21,11 @@ struct Cfg {
   static constexpr int kStages = 2;  // 144 KB (M = 4) or 96 KB (M = 8)
   static constexpr int kMinBlocks = 1;
   static constexpr int kTile = 2 * kPairs * kThreads * M;  // elements
+  // groups out of the fast path's range, queued per warp (DeferredGroups): at most
+  // 64 kPairs a tile on top of fewer than 32 left from earlier tiles
+  static constexpr int kDeferCap = 32 + 64 * kPairs;
+  static constexpr size_t kDeferOffset = (tile_smem_bytes<kTile, kStages>(6) + 15) & ~size_t(15);
+  static constexpr size_t kSmem = kDeferOffset + size_t(kDeferCap) * 8 * (kThreads / 32);
 };
 
 struct FwdArgs {
@@ -119,9 +124,9 @@ __device__ __forceinline__ void fwd_keys(const float* const* phi_g, const int64_
 }
 
 // Relaxation, hard bits and outputs of L groups whose keys are `kap`.
-template <int N, int M, bool TAU1, class V, bool ST = false>
-__device__ __forceinline__ void fwd_finish(const V (&kap)[M], const uint16_t* const* W_g, const int64_t* e0,
-                                           const FwdArgs& a, uint32_t* bits) {
+template <int N, int M, bool TAU1, class V, bool ST = false, bool DEFER = false>
+__device__ __forceinline__ uint32_t fwd_finish(const V (&kap)[M], const uint16_t* const* W_g, const int64_t* e0,
+                                               const FwdArgs& a, uint32_t* bits) {
   constexpr int L = vlanes<V>();
   FastGroup<N, M, TAU1, false, V> fg;
   fg.forward(kap, a.inv_tau);
@@ -165,32 +170,52 @@ __device__ __forceinline__ void fwd_finish(const V (&kap)[M], const uint16_t* co
       }
     }
   }
-  if (fg.flag != 0u) {
+  // groups out of the fast path's range: ranked by comparison, and either relaxed
+  // here by the exact routine (DEFER off) or (DEFER) left to fwd_exact_group, which
+  // the caller runs for them from the deferred queue and which writes their soft
+  // mask and Wm again
+  if constexpr (!DEFER) {
+    if (fg.flag != 0u) {
+#pragma unroll
+      for (int h = 0; h < L; ++h) {
+        if ((fg.flag >> h) & 1u) {
+          float k[M], kn[M];
+#pragma unroll
+          for (int l = 0; l < M; ++l) {
+            k[l] = lane_of(kap[l], h);
+            kn[l] = k[l] * kLn2;  // natural-log keys
+          }
+          if constexpr (kFastTopn) {
+            if constexpr (M == 4) {
+              bits[h] = topn_bits4(k, N);
+            } else {
+              bits[h] = topn_bits<M>(k, N);
+            }
+          }
+          // finite keys spread beyond the fast path's float range (tau != 1: at tau = 1
+          // that takes a key gap of ~69 natural-log units, and the tau = 1 kernels keep
+          // their code to the exact routine)
+          if (!TAU1 && all_finite(k)) {
+            RobustGroup<N, M> rg;
+            rg.forward(k, a.inv_tau, S[h]);
+          } else {
+            ExactGroup<N, M> ex;
+            ex.forward(kn, N, M, a.tau, S[h]);
+          }
+        }
+      }
+    }
+  } else if (kFastTopn && fg.flag != 0u) {
 #pragma unroll
     for (int h = 0; h < L; ++h) {
       if ((fg.flag >> h) & 1u) {
-        float k[M], kn[M];
+        float k[M];
 #pragma unroll
-        for (int l = 0; l < M; ++l) {
-          k[l] = lane_of(kap[l], h);
-          kn[l] = k[l] * kLn2;  // natural-log keys
-        }
-        if constexpr (kFastTopn) {
-          if constexpr (M == 4) {
-            bits[h] = topn_bits4(k, N);
-          } else {
-            bits[h] = topn_bits<M>(k, N);
-          }
-        }
-        // finite keys spread beyond the fast path's float range (tau != 1: at tau = 1
-        // that takes a key gap of ~69 natural-log units, and the tau = 1 kernels keep
-        // their code to the exact routine)
-        if (!TAU1 && all_finite(k)) {
-          RobustGroup<N, M> rg;
-          rg.forward(k, a.inv_tau, S[h]);
+        for (int l = 0; l < M; ++l) k[l] = lane_of(kap[l], h);
+        if constexpr (M == 4) {
+          bits[h] = topn_bits4(k, N);
         } else {
-          ExactGroup<N, M> ex;
-          ex.forward(kn, N, M, a.tau, S[h]);
+          bits[h] = topn_bits<M>(k, N);
         }
       }
     }
@@ -234,14 +259,58 @@ __device__ __forceinline__ void fwd_finish(const V (&kap)[M], const uint16_t* co
       }
     }
   }
+  return DEFER ? fg.flag : 0u;
 }
 
-template <int N, int M, bool TAU1, class V, bool ST = false>
+// The exact routine for one group out of the fast path's range (first element g0,
+// call-flat), from global memory: the log2-domain routine for finite keys spread
+// beyond the float range (tau != 1; at tau = 1 that takes a key gap of ~69
+// natural-log units and the tau = 1 kernels keep only the general routine), the
+// exact one otherwise.  Writes soft and (unless straight-through) Wm.
+template <int N, int M, bool TAU1, bool ST>
+__device__ __forceinline__ void fwd_exact_group(int64_t g0, const FwdArgs& a) {
+  if (ST && a.soft == nullptr) return;
+  // the keys as the tiles' packed code forms them (the group in both halves), so they
+  // equal, bit for bit, those the fast path and the masked linear's prologue see
+  const float* pp[2] = {a.phi + g0, a.phi + g0};
+  const int64_t e0[2] = {g0, g0};
+  F2 k2[M];
+  fwd_keys<M, F2>(pp, e0, nullptr, a, k2);
+  float k[M], S[M];
+#pragma unroll
+  for (int l = 0; l < M; ++l) k[l] = lo(k2[l]);
+  if (!TAU1 && all_finite(k)) {
+    RobustGroup<N, M> rg;
+    rg.forward(k, a.inv_tau, S);
+  } else {
+#pragma unroll
+    for (int l = 0; l < M; ++l) k[l] *= kLn2;  // natural-log keys
+    ExactGroup<N, M> ex;
+    ex.forward(k, N, M, a.tau, S);
+  }
+#pragma unroll
+  for (int s = 0; s < M / 4; ++s) {
+    if constexpr (!ST) {
+      const uint2 q = reinterpret_cast<const uint2*>(a.W + g0)[s];
+      uint2 o;
+      o.x = pack_bf16x2(__fmul_rn(bf16_bits_to_float(q.x & 0xffffu), S[4 * s]),
+                        __fmul_rn(bf16_bits_to_float(q.x >> 16), S[4 * s + 1]));
+      o.y = pack_bf16x2(__fmul_rn(bf16_bits_to_float(q.y & 0xffffu), S[4 * s + 2]),
+                        __fmul_rn(bf16_bits_to_float(q.y >> 16), S[4 * s + 3]));
+      reinterpret_cast<uint2*>(a.Wm + g0)[s] = o;
+    }
+    if (a.soft != nullptr)
+      reinterpret_cast<float4*>(a.soft + g0)[s] = make_float4(S[4 * s], S[4 * s + 1], S[4 * s + 2], S[4 * s + 3]);
+  }
+}
+
+// One group straight from global memory (the ragged tail; the exact routine in place).
+template <int N, int M, bool TAU1, bool ST = false>
 __device__ __forceinline__ void fwd_groups(const float* const* phi_g, const uint16_t* const* W_g, const int64_t* e0,
                                            const FwdArgs& a, uint32_t* bits) {
-  V kap[M];
-  fwd_keys<M, V>(phi_g, e0, nullptr, a, kap);
-  fwd_finish<N, M, TAU1, V, ST>(kap, W_g, e0, a, bits);
+  float kap[M];
+  fwd_keys<M, float>(phi_g, e0, nullptr, a, kap);
+  fwd_finish<N, M, TAU1, float, ST>(kap, W_g, e0, a, bits);
 }
 
 // Combine the M-bit masks of 32 / M consecutive lanes into words and store.
@@ -280,8 +349,8 @@ __device__ __forceinline__ void store_hard_pair(uint32_t* hard, int64_t e0a, int
 
 // One full tile of a tensor (local tile index `tile`), inputs staged in shared
 // memory.  NARROW: the call's counters are below 2^32 (a.np.narrow).
-template <int N, int M, bool TAU1, bool ST, bool NARROW>
-__device__ __forceinline__ void fwd_tile(const uint8_t* const* stage, int64_t tile, const FwdArgs& a) {
+template <int N, int M, bool TAU1, bool ST, bool NARROW, bool DEFER, class Defer>
+__device__ __forceinline__ void fwd_tile(const uint8_t* const* stage, int64_t tile, const FwdArgs& a, Defer& dg) {
   using C = Cfg<M>;
   constexpr int kT = C::kTile;
   const float* sphi = reinterpret_cast<const float*>(stage[0]);
@@ -314,9 +383,14 @@ __device__ __forceinline__ void fwd_tile(const uint8_t* const* stage, int64_t ti
     const uint16_t* pw[2] = {sW + g0 * M, sW + g1 * M};
     const int64_t e0[2] = {base + g0 * M, base + g1 * M};
     uint32_t bits[2];
-    fwd_finish<N, M, TAU1, F2, ST>(kap[p & 1], pw, e0, a, bits);
+    const uint32_t flag = fwd_finish<N, M, TAU1, F2, ST, DEFER>(kap[p & 1], pw, e0, a, bits);
     if (a.hard != nullptr) store_hard_pair<M>(a.hard, e0[0], e0[1], bits[0], bits[1]);
+    if constexpr (DEFER) {
+      dg.push((flag & 1u) != 0u, e0[0]);
+      dg.push((flag & 2u) != 0u, e0[1]);
+    }
   }
+  if constexpr (DEFER) dg.drain(false, [&](int64_t g0) { fwd_exact_group<N, M, TAU1, ST>(g0, a); });
 }
 
 // The ragged tail of a tensor (fewer than one tile after its full tiles), by one
@@ -335,14 +409,14 @@ __device__ __forceinline__ void fwd_tail(const FwdArgs& a) {
       const float* pp[1] = {a.phi + t0 + gi * M};
       const uint16_t* pw[1] = {a.W + t0 + gi * M};
       const int64_t e0[1] = {t0 + gi * M};
-      fwd_groups<N, M, TAU1, float, ST>(pp, pw, e0, a, &bits);
+      fwd_groups<N, M, TAU1, ST>(pp, pw, e0, a, &bits);
     }
     if (a.hard != nullptr) store_hard<M>(a.hard, t0 + gi * M, bits, active);
   }
 }
 
 // ST: straight-through Wm (a separate instantiation)
-template <int N, int M, bool TAU1, bool ST>
+template <int N, int M, bool TAU1, bool ST, bool DEFER>
 __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_fwd_kernel(FwdArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   using C = Cfg<M>;
@@ -351,6 +425,8 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_fwd_
   src.esize[0] = 4;
   src.ptr[1] = reinterpret_cast<const uint8_t*>(a.W);
   src.esize[1] = 2;
+  DeferredGroups<C::kDeferCap> dg;
+  dg.init(smem + C::kDeferOffset);
   // a batch's next tensor may start on the SMs this launch frees (no-op otherwise)
   pdl_launch_dependents();
   const bool ok = run_tiles<C::kThreads, C::kTile, C::kStages, 2>(
@@ -360,12 +436,15 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_fwd_
         // body measured slower (register allocation), so those keep one
         if constexpr (M == 4) {
           if (a.np.narrow) {
-            fwd_tile<N, M, TAU1, ST, true>(stage, tile, a);
+            fwd_tile<N, M, TAU1, ST, true, DEFER>(stage, tile, a, dg);
             return;
           }
         }
-        fwd_tile<N, M, TAU1, ST, false>(stage, tile, a);
+        fwd_tile<N, M, TAU1, ST, false, DEFER>(stage, tile, a, dg);
       });
+  if constexpr (DEFER) {
+    if (ok) dg.drain(true, [&](int64_t g0) { fwd_exact_group<N, M, TAU1, ST>(g0, a); });
+  }
   if (ok && blockIdx.x == gridDim.x - 1) fwd_tail<N, M, TAU1, ST>(a);
   // the launch completes only after the batch's previous one (stream order)
   if (blockIdx.x == 0) pdl_wait();
@@ -406,11 +485,12 @@ struct LaunchCache {
   int per_sm[64] = {0};
 };
 
-template <int N, int M, bool TAU1, bool ST>
+template <int N, int M, bool TAU1, bool ST, bool DEFER>
 int launch_tiles(const FwdArgs& a, cudaStream_t stream, bool pdl) {
   using C = Cfg<M>;
-  auto kern = roi_fwd_kernel<N, M, TAU1, ST>;
-  const size_t smem = tile_smem_bytes<C::kTile, C::kStages>(6);
+  auto kern = roi_fwd_kernel<N, M, TAU1, ST, DEFER>;
+  const size_t smem = C::kSmem;
+  static_assert(C::kSmem <= 232448, "shared memory per CTA");
   static LaunchCache cache;  // per instantiation and device; racing writers store the same value
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return -1;
@@ -426,12 +506,23 @@ int launch_tiles(const FwdArgs& a, cudaStream_t stream, bool pdl) {
   return launch_maybe_pdl(kern, grid, C::kThreads, smem, stream, pdl, a);
 }
 
+// Groups out of the fast path's range go to the exact routine in place (one thread,
+// the rest of its warp waiting) or, below tau = 0.075, through the deferred queue
+// (32 at a time).  At tau = 0.05 (the end of the paper's schedule) some 4-5 % of
+// the groups leave the range and the queue makes the 7B-shaped 4:8 forward 2.1x
+// faster; at tau >= 0.1 (under 0.2 % of them) the queue's code measured 2-9 % slower.
+constexpr float kDeferBelowTau = 0.075f;
+
+template <int N, int M, bool ST>
+int launch_st(const FwdArgs& a, cudaStream_t stream, bool pdl) {
+  if (a.tau == 1.0f) return launch_tiles<N, M, true, ST, false>(a, stream, pdl);
+  return a.tau < kDeferBelowTau ? launch_tiles<N, M, false, ST, true>(a, stream, pdl)
+                                : launch_tiles<N, M, false, ST, false>(a, stream, pdl);
+}
+
 template <int N, int M>
 int launch_nm(const FwdArgs& a, cudaStream_t stream, bool pdl = false) {
-  if (a.st)
-    return a.tau == 1.0f ? launch_tiles<N, M, true, true>(a, stream, pdl) : launch_tiles<N, M, false, true>(a, stream, pdl);
-  return a.tau == 1.0f ? launch_tiles<N, M, true, false>(a, stream, pdl)
-                       : launch_tiles<N, M, false, false>(a, stream, pdl);
+  return a.st ? launch_st<N, M, true>(a, stream, pdl) : launch_st<N, M, false>(a, stream, pdl);
 }
 
 }  // namespace
