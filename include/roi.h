@@ -330,8 +330,8 @@ roi_status roi_device_status(void* stream);
 
 /* Wall-time limit of a kernel's wait for a stage of its copy ring (the staged
  * tiles of logits and weights) on the current device, in ns; default
- * 2,000,000,000.  With 0 a wait that finds its stage not yet landed gives up at
- * once; the tests use that to run the timeout path on valid copies.  The waits
+ * 2,000,000,000.  With 0 every such wait gives up at once, whether its stage has
+ * landed or not; the tests use that to run the timeout path on valid copies.  The waits
  * with which a kernel that gave up drains its own copies in flight keep the fixed
  * 2 s limit.  Applies to kernels launched after the call returns (it is a
  * synchronous copy to device memory); ROI_ERR_CUDA if that copy fails. */

@@ -591,6 +591,159 @@ struct RobustGroup {
   }
 };
 
+// ---------------------------------------------------------------------------
+// The log2-domain relaxation of RobustGroup in O(M) per step, for the wide groups
+// of the warp-slice kernels (M = 16, 32), finite keys.  With m1 the largest z,
+// a its (first) index and m2 the largest of the others, every exclusive sum over
+// j != l is formed against m1 for l != a (it contains 2^0 from member a, so it
+// cannot underflow) and against m2 for l = a; the sums use prefix and suffix sums,
+// no subtraction.  The backward's sum over i != l of b_i 2^(z_l - LSE_{j != i} z_j)
+// splits the same way: for i != a, 2^(m1 - LSE_{j != i}) lies in [1/M, 1] and the
+// terms are 2^(z_l - m1) times an exclusive sum; the i = a term is formed directly.
+// Members stay in registers; the step history goes to local memory.
+// ---------------------------------------------------------------------------
+template <int M>
+struct Top2 {
+  float m1, m2;
+  int a;
+  __device__ __forceinline__ explicit Top2(const float (&z)[M]) {
+    m1 = -INFINITY, m2 = -INFINITY, a = 0;
+#pragma unroll
+    for (int l = 0; l < M; ++l) {
+      if (z[l] > m1) {
+        m2 = m1, m1 = z[l], a = l;
+      } else {
+        m2 = fmaxf(m2, z[l]);
+      }
+    }
+  }
+};
+// out[l] = sum over j != l of x[j] (prefix plus suffix sums)
+template <int M>
+__device__ __forceinline__ void exclusive_sums_scalar(const float (&x)[M], float (&out)[M]) {
+  float pre = 0.0f;
+#pragma unroll
+  for (int l = 0; l < M; ++l) {
+    out[l] = pre;
+    pre = __fadd_rn(pre, x[l]);
+  }
+  float suf = 0.0f;
+#pragma unroll
+  for (int l = M - 1; l >= 0; --l) {
+    out[l] = __fadd_rn(out[l], suf);
+    suf = __fadd_rn(suf, x[l]);
+  }
+}
+
+template <int N, int M>
+struct WideRobustGroup {
+  float zh[N][M];  // z entering each step
+
+  // LSE2 over j != l for every l, and LSE2 over all (returned), of z with top-2 `t`;
+  // e[l] = 2^(z_l - m1).
+  static __device__ __forceinline__ float lse2_all_and_excluding(const float (&z)[M], const Top2<M>& t,
+                                                                 float (&e)[M], float (&lx)[M]) {
+    float s1 = 0.0f;
+#pragma unroll
+    for (int l = 0; l < M; ++l) {
+      e[l] = ex2_approx(__fsub_rn(z[l], t.m1));
+      s1 = __fadd_rn(s1, e[l]);
+    }
+    float ex[M];
+    exclusive_sums_scalar(e, ex);
+    float s2 = 0.0f;  // sum over j != a of 2^(z_j - m2)
+#pragma unroll
+    for (int l = 0; l < M; ++l) {
+      lx[l] = __fadd_rn(t.m1, lg2_approx(ex[l]));
+      s2 = __fadd_rn(s2, l == t.a ? 0.0f : ex2_approx(__fsub_rn(z[l], t.m2)));
+    }
+    float lxa = __fadd_rn(t.m2, lg2_approx(s2));
+#pragma unroll
+    for (int l = 0; l < M; ++l)
+      if (l == t.a) lx[l] = lxa;
+    return __fadd_rn(t.m1, lg2_approx(s1));
+  }
+
+  // t: the keys in log2 units, all finite.  Fills S.
+  __device__ __forceinline__ void forward(const float (&t)[M], float inv_tau, float (&S)[M]) {
+    float z[M];
+#pragma unroll
+    for (int l = 0; l < M; ++l) {
+      z[l] = __fmul_rn(t[l], inv_tau);
+      S[l] = 0.0f;
+    }
+#pragma unroll 1
+    for (int k = 0; k < N; ++k) {
+      const Top2<M> top(z);
+#pragma unroll
+      for (int l = 0; l < M; ++l) {
+        z[l] = __fsub_rn(z[l], top.m1);  // shift: the largest is 0
+        zh[k][l] = z[l];
+      }
+      const Top2<M> t0{z};
+      float e[M], lx[M];
+      const float lz = lse2_all_and_excluding(z, t0, e, lx);
+      float s1 = 0.0f;
+#pragma unroll
+      for (int l = 0; l < M; ++l) s1 = __fadd_rn(s1, e[l]);
+      const float r = rcp_approx(s1);
+#pragma unroll
+      for (int l = 0; l < M; ++l) S[l] = __fadd_rn(S[l], __fmul_rn(e[l], r));
+      if (k + 1 < N) {
+#pragma unroll
+        for (int l = 0; l < M; ++l) z[l] = __fmaf_rn(__fsub_rn(lx[l], lz), inv_tau, z[l]);
+      }
+    }
+  }
+
+  // After forward(): dk = dL/dkappa for c = dL/dS.
+  __device__ __forceinline__ void backward(const float (&c)[M], float inv_tau, float (&dk)[M]) const {
+    float b[M];
+#pragma unroll
+    for (int l = 0; l < M; ++l) b[l] = 0.0f;
+#pragma unroll 1
+    for (int k = N - 1; k >= 0; --k) {
+      float z[M];
+#pragma unroll
+      for (int l = 0; l < M; ++l) z[l] = zh[k][l];
+      const Top2<M> t(z);
+      float e[M], lx[M];
+      const float lz = lse2_all_and_excluding(z, t, e, lx);
+      float mu[M], gz[M];
+      float cmu = 0.0f, B = 0.0f;
+#pragma unroll
+      for (int l = 0; l < M; ++l) {
+        mu[l] = ex2_approx(__fsub_rn(z[l], lz));
+        cmu = __fmaf_rn(c[l], mu[l], cmu);
+        B = __fadd_rn(B, b[l]);
+      }
+#pragma unroll
+      for (int l = 0; l < M; ++l) gz[l] = __fmul_rn(mu[l], __fsub_rn(__fsub_rn(c[l], cmu), B));
+      if (k + 1 < N) {
+        // (J^T b)_l adds sum over i != l of b_i 2^(z_l - lx_i)
+        float w[M], wx[M];
+#pragma unroll
+        for (int i = 0; i < M; ++i) w[i] = i == t.a ? 0.0f : __fmul_rn(b[i], ex2_approx(__fsub_rn(t.m1, lx[i])));
+        exclusive_sums_scalar(w, wx);
+        float ba = 0.0f, lxa = 0.0f;
+#pragma unroll
+        for (int i = 0; i < M; ++i)
+          if (i == t.a) ba = b[i], lxa = lx[i];
+#pragma unroll
+        for (int l = 0; l < M; ++l) {
+          float add = __fmul_rn(e[l], wx[l]);
+          if (l != t.a) add = __fmaf_rn(ba, ex2_approx(__fsub_rn(z[l], lxa)), add);
+          gz[l] = __fadd_rn(gz[l], add);
+        }
+      }
+#pragma unroll
+      for (int l = 0; l < M; ++l) b[l] = __fmaf_rn(gz[l], inv_tau, b[l]);
+    }
+#pragma unroll
+    for (int l = 0; l < M; ++l) dk[l] = b[l];
+  }
+};
+
 // True if every key of a group is finite.
 template <int M>
 __device__ __forceinline__ bool all_finite(const float (&k)[M]) {
@@ -832,12 +985,15 @@ struct FastGroup {
       for (int l = 0; l < M; ++l) d[l] = vmul(vsub(kap[l], kmax), sc);
       const V ksum = sum_of(kap);
       flag = vbelow(vsub(ksum, ksum), 0.0f);  // a non-finite key (or a sum beyond the float range)
+      V tmin = vconst<V>(1.0f);
 #pragma unroll
       for (int k = 0; k < N; ++k) {
         V e[M];
 #pragma unroll
         for (int l = 0; l < M; ++l) e[l] = vmap(d[l], ex2_approx);
-        const V r = vmap(sum_of(e), rcp_approx);
+        const V tot = sum_of(e);
+        if (M >= 8 && k > 0) tmin = vmin(tmin, tot);
+        const V r = vmap(tot, rcp_approx);
         if (!KEEP && k > 0 && k + 1 == N) {
           // last step without KEEP: added into S as it is formed (one fma)
 #pragma unroll
@@ -851,16 +1007,30 @@ struct FastGroup {
           }
         }
         if (k + 1 < N) {
+          // d_l += log2(1 - mu_l) / tau.  A group whose exclusive sums fall below 2^-100
+          // of the total goes to the exact routine.  M = 8: the offsets are first
+          // renormalised by log2 of the total (so sum 2^d = 1 and every offset <= 0)
+          // instead of by their maximum after the update (seven comparisons per step;
+          // 1.5B-shaped 4:8 at tau = 0.5 2 % faster, the 2:4 step 1 % slower), and a
+          // total below 2^-120 (offsets that fell too far in one step) is flagged too.
           V ex[M];
           exclusive_sums(e, ex);
-          flag |= vbelow(min_of(ex), kTinyExcl);
+          if constexpr (M >= 8) {
+            flag |= vbelow(vmul(min_of(ex), r), kTinyExcl);
+            const V lz = vmap(tot, lg2_approx);
 #pragma unroll
-          for (int l = 0; l < M; ++l) d[l] = vfma(vmap(vmul(ex[l], r), lg2_approx), itau, d[l]);
-          const V dm = max_of(d);
+            for (int l = 0; l < M; ++l) d[l] = vfma(vmap(vmul(ex[l], r), lg2_approx), itau, vsub(d[l], lz));
+          } else {
+            flag |= vbelow(min_of(ex), kTinyExcl);
 #pragma unroll
-          for (int l = 0; l < M; ++l) d[l] = vsub(d[l], dm);
+            for (int l = 0; l < M; ++l) d[l] = vfma(vmap(vmul(ex[l], r), lg2_approx), itau, d[l]);
+            const V dm = max_of(d);
+#pragma unroll
+            for (int l = 0; l < M; ++l) d[l] = vsub(d[l], dm);
+          }
         }
       }
+      if constexpr (M >= 8) flag |= vbelow(tmin, 7.52316384526264e-37f);  // 2^-120
     }
   }
 
@@ -990,10 +1160,14 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity
 // Waits for a stage of a copy ring, for at most the limit in the status record
 // (read only when the stage has not landed yet, through the read-only cache: the
 // host changes it only between launches; 2 s unless the caller set another one).
-// A limit of 0 gives up as soon as the stage is found incomplete.
-__device__ __forceinline__ bool mbar_wait_ring(uint64_t* bar, uint32_t parity, const unsigned int* status) {
-  if (mbar_test_wait(bar, parity)) return true;
-  const uint64_t lim = __ldg(reinterpret_cast<const unsigned long long*>(status + kStatusLimitWord));
+// A limit of 0 gives up at once, whether the stage has landed or not (the tests'
+// deterministic way onto the timeout path).  `lim` comes from ring_wait_limit(),
+// read once per kernel.
+__device__ __forceinline__ uint64_t ring_wait_limit(const unsigned int* status) {
+  return __ldg(reinterpret_cast<const unsigned long long*>(status + kStatusLimitWord));
+}
+__device__ __forceinline__ bool mbar_wait_ring(uint64_t* bar, uint32_t parity, uint64_t lim) {
+  if (mbar_test_wait(bar, parity)) return lim != 0;
   if (lim == 0) return false;
   const uint64_t t0 = global_timer_ns();
   while (true) {

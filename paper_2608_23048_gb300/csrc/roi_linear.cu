@@ -265,6 +265,7 @@ __global__ void __launch_bounds__(LinCfg<M>::kThreads + 32, 1)
   const uint32_t tmem = misc[0];
 
   bool ok = true;
+  const uint64_t lim = ring_wait_limit(a.status);
   // producer lane: chunks whose TMA fill was issued, and whose MMAs were committed
   int issued = 0, committed = 0;
   if (producer) {
@@ -278,7 +279,7 @@ __global__ void __launch_bounds__(LinCfg<M>::kThreads + 32, 1)
       uint32_t phase = 0;  // parity of the current pass over the stages
       int s = 0;
       for (int c = 0; c < nc && ok; ++c) {
-        ok = mbar_wait_ring(ready + s, phase, a.status);
+        ok = mbar_wait_ring(ready + s, phase, lim);
         if (!ok) break;
         tc_fence_after();
         const uint32_t sa = smem_addr(smem + L.a + s * kTileA);
@@ -293,7 +294,7 @@ __global__ void __launch_bounds__(LinCfg<M>::kThreads + 32, 1)
         if (c + kStages < nc) {
           // refill this stage once its MMAs are done (its staged logits and
           // weights were consumed before `ready` completed)
-          ok = mbar_wait_ring(mma + s, phase, a.status);
+          ok = mbar_wait_ring(mma + s, phase, lim);
           if (ok) {
             issue_chunk(&tm_phi, &tm_w, &tm_x, smem, L, s, row0, c_begin + c + kStages);
             issued = c + kStages + 1;
@@ -312,7 +313,7 @@ __global__ void __launch_bounds__(LinCfg<M>::kThreads + 32, 1)
     uint32_t phase = 0;
     int s = 0;
     for (int c = 0; c < nc; ++c) {
-      if (ok) ok = mbar_wait_ring(full + s, phase, a.status);
+      if (ok) ok = mbar_wait_ring(full + s, phase, lim);
       if (!ok) break;
       chunk_masked_weights<N, M, TAU1>(a, smem, L, s, row0, c_begin + c);
       fence_proxy_async_smem();
@@ -326,7 +327,7 @@ __global__ void __launch_bounds__(LinCfg<M>::kThreads + 32, 1)
     }
     // the last chunk's commit covers every MMA issued before it (the previous
     // completion of that stage preceded the refill this thread already saw)
-    if (nc > 0 && ok) ok = mbar_wait_ring(mma + (nc - 1) % kStages, uint32_t((nc - 1) / kStages) & 1u, a.status);
+    if (nc > 0 && ok) ok = mbar_wait_ring(mma + (nc - 1) % kStages, uint32_t((nc - 1) / kStages) & 1u, lim);
   }
   if (!ok) misc[2] = 0u;
   __syncthreads();

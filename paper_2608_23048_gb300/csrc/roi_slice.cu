@@ -7,7 +7,8 @@
 // allow, the two groups of those slots are relaxed in lockstep on packed FP32
 // (V = F2, one group per half), otherwise one after the other (V = float).
 // Groups whose keys leave the fast path's range are queued by the slice's first
-// lane (DeferredGroups) and handled 32 at a time, one per lane, by ExactGroup.
+// lane (DeferredGroups) and handled 32 at a time, one per lane, by WideRobustGroup
+// (ExactGroup for non-finite keys).
 #include "roi_launch.h"
 #include "roi_tiles.cuh"
 
@@ -44,14 +45,11 @@ constexpr bool kReloadHist = M == 16;
 // Deferred exact-routine groups (DeferredGroups): a warp queues at most 64 / SL
 // groups per tile (or per round of the ragged tail) and drains once 32 are queued.
 constexpr int kDeferCap = 48;
-// DEFER: the kernels queue flagged groups (DeferredGroups) instead of running the
-// exact routine in place.  8:16 always defers.  16:32 defers only for tau < 0.15:
-// there (the paper anneals tau to 0.05) a few per cent of the groups leave the fast
-// path's range (key gaps beyond ~69 tau natural-log units) and the queued routine
-// runs 15x faster per step than in place; above it no group does, and the 16:32
-// kernels, at 255 registers and one CTA per SM, measured 10 % slower with the
-// queue's code than with the exact routine in place.
-constexpr float kDeferBelowTau = 0.15f;
+// The kernels queue flagged groups (DeferredGroups) and run the exact routine for
+// them 32 at a time.  Measured on the 3B-shaped set: at tau = 0.2 (no group flagged)
+// the 16:32 step takes 87.3 ms with the queue against 94.3 ms with the exact routine
+// in place; at tau = 0.05 (~4 % flagged) 8:16 takes 52.8 ms against 2424 ms and
+// 16:32 135 ms against 14.7 s.
 constexpr size_t kDeferBytes = size_t(kDeferCap) * 8 * (kThreads / 32);
 constexpr size_t kFwdDeferOffset = (tile_smem_bytes<kTile, kStagesFwd>(6) + 15) & ~size_t(15);
 template <int N, int M>
@@ -467,18 +465,36 @@ __device__ __forceinline__ void slot_topn(const V (&kap)[4], int base_lane, int 
   }
 }
 
-// The keys of all M elements of one group, in natural-log units, from logits at
-// phi_g (call-flat index g0), by one lane.
+// The keys of all M elements of one group, in log2 units, from logits at phi_g
+// (call-flat index g0), by one lane.
 template <int N, int M>
 __device__ __forceinline__ void group_keys_all(const float* phi_g, int64_t g0, const NoiseParams& np, float (&k)[M]) {
-#pragma unroll 1
+#pragma unroll
   for (int s = 0; s < M / 4; ++s) {
     const float* p[1] = {phi_g + 4 * s};
     const int64_t e[1] = {g0 + 4 * s};
     float k4[4];
     slot_keys<float>(p, e, np, k4);
 #pragma unroll
-    for (int j = 0; j < 4; ++j) k[4 * s + j] = k4[j] * kLn2;
+    for (int j = 0; j < 4; ++j) k[4 * s + j] = k4[j];
+  }
+}
+// The exact relaxation of one group with keys t (log2 units): WideRobustGroup for
+// finite keys, ExactGroup (natural-log keys) otherwise; soft mask S and, with c,
+// dk = dL/dkappa.
+template <int N, int M, bool BWD>
+__device__ __forceinline__ void exact_relax(float (&t)[M], const float (&c)[M], const SliceArgs& a, float (&S)[M],
+                                            float (&dk)[M]) {
+  if (all_finite(t)) {
+    WideRobustGroup<N, M> rg;
+    rg.forward(t, a.inv_tau, S);
+    if constexpr (BWD) rg.backward(c, a.inv_tau, dk);
+  } else {
+#pragma unroll
+    for (int l = 0; l < M; ++l) t[l] *= kLn2;  // natural-log keys
+    ExactGroup<N, M> ex;
+    ex.forward(t, N, M, a.tau, S);
+    if constexpr (BWD) ex.backward(c, N, M, a.tau, dk);
   }
 }
 
@@ -500,10 +516,9 @@ __device__ __forceinline__ void unpack_bf16x4(uint2 q, float (&out)[4]) {
 template <int N, int M>
 __device__ __forceinline__ void exact_group_fwd(int64_t g0, const SliceArgs& a) {
   if (a.soft == nullptr && a.st) return;
-  float k[M], S[M];
+  float k[M], S[M], unused[M];
   group_keys_all<N, M>(a.phi + g0, g0, a.np, k);
-  ExactGroup<N, M> ex;
-  ex.forward(k, N, M, a.tau, S);
+  exact_relax<N, M, false>(k, k, a, S, unused);
 #pragma unroll 1
   for (int s = 0; s < M / 4; ++s) {
     float wv[4], sv[4];
@@ -529,9 +544,7 @@ __device__ __forceinline__ void exact_group_bwd(int64_t g0, const SliceArgs& a) 
 #pragma unroll
     for (int j = 0; j < 4; ++j) cc[4 * s + j] = __fmul_rn(dv[j], wv[j]);
   }
-  ExactGroup<N, M> ex;
-  ex.forward(k, N, M, a.tau, S);
-  ex.backward(cc, N, M, a.tau, dkk);
+  exact_relax<N, M, true>(k, cc, a, S, dkk);
 #pragma unroll 1
   for (int s = 0; s < M / 4; ++s) {
     const int64_t e = g0 + 4 * s;
@@ -553,7 +566,7 @@ __device__ __forceinline__ void exact_group_bwd(int64_t g0, const SliceArgs& a) 
 // shared or global memory, e0: call-flat index of its first element).  All 32
 // lanes of the warp call this together; inactive slots (ragged tail, V = float
 // only) take part in the shuffles with zero keys.  Returns each slot's hard bits.
-template <int N, int M, bool TAU1, bool DEFER, class V>
+template <int N, int M, bool TAU1, class V>
 __device__ __forceinline__ void fwd_slots(const float* const* p, const uint16_t* const* w, const int64_t* e0,
                                           bool active, const SliceArgs& a, uint32_t (&bits)[vlanes<V>()],
                                           uint32_t& defer) {
@@ -574,7 +587,7 @@ __device__ __forceinline__ void fwd_slots(const float* const* p, const uint16_t*
   const uint32_t flag = rx.forward(kap, a.inv_tau, base_lane);
   // groups out of the fast path's range: queued by their first lane for the exact
   // routine, which writes their outputs
-  defer = DEFER && active && q == 0 ? flag : 0u;
+  defer = active && q == 0 ? flag : 0u;
   if (!active) return;
 #pragma unroll
   for (int h = 0; h < L; ++h) {
@@ -587,14 +600,12 @@ __device__ __forceinline__ void fwd_slots(const float* const* p, const uint16_t*
       for (int j = 0; j < 4; ++j) sv[j] = lane_of(rx.S[j], h);
       if (!a.st) *reinterpret_cast<uint2*>(a.Wm + e0[h]) = pack4(wv, sv);
       if (a.soft != nullptr) *reinterpret_cast<float4*>(a.soft + e0[h]) = make_float4(sv[0], sv[1], sv[2], sv[3]);
-    } else if constexpr (!DEFER) {
-      if (q == 0) exact_group_fwd<N, M>(e0[h], a);
     }
   }
 }
 
 // Backward of L slots (as fwd_slots).
-template <int N, int M, bool TAU1, bool DEFER, class V>
+template <int N, int M, bool TAU1, class V>
 __device__ __forceinline__ void bwd_slots(const float* const* p, const uint16_t* const* w, const uint16_t* const* dw,
                                           const int64_t* e0, bool active, const SliceArgs& a, uint32_t& defer) {
   constexpr int SL = M / 4;
@@ -626,7 +637,7 @@ __device__ __forceinline__ void bwd_slots(const float* const* p, const uint16_t*
   SliceRelax<N, M, TAU1, true, V> rx;
   rx.hist = reinterpret_cast<V*>(roi_slice_smem + kSliceHistOffset<M>) + threadIdx.x;
   const uint32_t flag = rx.forward(kap, a.inv_tau, base_lane);
-  defer = DEFER && active && q == 0 ? flag : 0u;
+  defer = active && q == 0 ? flag : 0u;
   if (active && a.dW != nullptr) {
 #pragma unroll
     for (int h = 0; h < L; ++h) {
@@ -659,8 +670,6 @@ __device__ __forceinline__ void bwd_slots(const float* const* p, const uint16_t*
       const float g4[4] = {lane_of(dk[0], h), lane_of(dk[1], h), lane_of(dk[2], h), lane_of(dk[3], h)};
       if (a.dphi != nullptr) *reinterpret_cast<float4*>(a.dphi + e0[h]) = make_float4(g4[0], g4[1], g4[2], g4[3]);
       if (a.phi_out != nullptr) adamw4(a.phi_out, a.m, a.v, e0[h], *reinterpret_cast<const float4*>(p[h]), g4, a.opt);
-    } else if constexpr (!DEFER) {
-      if (q == 0) exact_group_bwd<N, M>(e0[h], a);
     }
   }
 }
@@ -692,7 +701,7 @@ __device__ __forceinline__ void store_hard_slot_pair(uint32_t* hard, int64_t e0a
   if ((lane & 3) == 0) hard[(upper ? e0b : e0a) >> 5] = word;
 }
 
-template <int N, int M, bool TAU1, bool DEFER>
+template <int N, int M, bool TAU1>
 __global__ void __launch_bounds__(kThreads, kMinBlocksFwd) roi_slice_fwd_kernel(SliceArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
   TileSrc<2> src;
@@ -717,22 +726,20 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksFwd) roi_slice_fwd_kernel(
         uint32_t bits[2], defer[2];
         if constexpr (kPairedFwd<M>) {
           uint32_t d2;
-          fwd_slots<N, M, TAU1, DEFER, F2>(pp, pw, e0, true, a, bits, d2);
+          fwd_slots<N, M, TAU1, F2>(pp, pw, e0, true, a, bits, d2);
           defer[0] = d2 & 1u, defer[1] = d2 >> 1;
         } else {
 #pragma unroll 1
           for (int j = 0; j < 2; ++j) {
             uint32_t b1[1];
-            fwd_slots<N, M, TAU1, DEFER, float>(pp + j, pw + j, e0 + j, true, a, b1, defer[j]);
+            fwd_slots<N, M, TAU1, float>(pp + j, pw + j, e0 + j, true, a, b1, defer[j]);
             bits[j] = b1[0];
           }
         }
         if (a.hard != nullptr) store_hard_slot_pair(a.hard, e0[0], e0[1], bits[0], bits[1]);
-        if constexpr (DEFER) {
-          dg.push(defer[0] != 0u, e0[0]);
-          dg.push(defer[1] != 0u, e0[1]);
-          dg.drain(false, exact);
-        }
+        dg.push(defer[0] != 0u, e0[0]);
+        dg.push(defer[1] != 0u, e0[1]);
+        dg.drain(false, exact);
       });
   if (ok && blockIdx.x == gridDim.x - 1) {
     const int64_t t0 = a.full_tiles * kTile;
@@ -745,22 +752,18 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksFwd) roi_slice_fwd_kernel(
       const uint16_t* pw[1] = {a.W + off};
       const int64_t e0[1] = {t0 + 4 * si};
       uint32_t bits[1], defer;
-      fwd_slots<N, M, TAU1, DEFER, float>(pp, pw, e0, active, a, bits, defer);
+      fwd_slots<N, M, TAU1, float>(pp, pw, e0, active, a, bits, defer);
       if (a.hard != nullptr) store_hard_slot(a.hard, e0[0], bits[0], active);
-      if constexpr (DEFER) {
-        dg.push(defer != 0u, e0[0]);
-        dg.drain(false, exact);
-      }
+      dg.push(defer != 0u, e0[0]);
+      dg.drain(false, exact);
     }
   }
-  if constexpr (DEFER) {
-    if (ok) dg.drain(true, exact);
-  }
+  if (ok) dg.drain(true, exact);
   // the launch completes only after the batch's previous one (stream order)
   if (blockIdx.x == 0) pdl_wait();
 }
 
-template <int N, int M, bool TAU1, bool DEFER>
+template <int N, int M, bool TAU1>
 __global__ void __launch_bounds__(kThreads, kMinBlocksBwd<M>) roi_slice_bwd_kernel(SliceArgs a) {
   uint8_t* smem = roi_slice_smem;
   TileSrc<3> src;
@@ -788,18 +791,16 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksBwd<M>) roi_slice_bwd_kern
         uint32_t defer[2];
         if constexpr (kPairedBwd<M>) {
           uint32_t d2;
-          bwd_slots<N, M, TAU1, DEFER, F2>(pp, pw, pd, e0, true, a, d2);
+          bwd_slots<N, M, TAU1, F2>(pp, pw, pd, e0, true, a, d2);
           defer[0] = d2 & 1u, defer[1] = d2 >> 1;
         } else {
 #pragma unroll 1
           for (int j = 0; j < 2; ++j)
-            bwd_slots<N, M, TAU1, DEFER, float>(pp + j, pw + j, pd + j, e0 + j, true, a, defer[j]);
+            bwd_slots<N, M, TAU1, float>(pp + j, pw + j, pd + j, e0 + j, true, a, defer[j]);
         }
-        if constexpr (DEFER) {
-          dg.push(defer[0] != 0u, e0[0]);
-          dg.push(defer[1] != 0u, e0[1]);
-          dg.drain(false, exact);
-        }
+        dg.push(defer[0] != 0u, e0[0]);
+        dg.push(defer[1] != 0u, e0[1]);
+        dg.drain(false, exact);
       });
   if (ok && blockIdx.x == gridDim.x - 1) {
     const int64_t t0 = a.full_tiles * kTile;
@@ -813,16 +814,12 @@ __global__ void __launch_bounds__(kThreads, kMinBlocksBwd<M>) roi_slice_bwd_kern
       const uint16_t* pd[1] = {a.dWm + off};
       const int64_t e0[1] = {t0 + 4 * si};
       uint32_t defer;
-      bwd_slots<N, M, TAU1, DEFER, float>(pp, pw, pd, e0, active, a, defer);
-      if constexpr (DEFER) {
-        dg.push(defer != 0u, e0[0]);
-        dg.drain(false, exact);
-      }
+      bwd_slots<N, M, TAU1, float>(pp, pw, pd, e0, active, a, defer);
+      dg.push(defer != 0u, e0[0]);
+      dg.drain(false, exact);
     }
   }
-  if constexpr (DEFER) {
-    if (ok) dg.drain(true, exact);
-  }
+  if (ok) dg.drain(true, exact);
   if (blockIdx.x == 0) pdl_wait();
 }
 
@@ -847,39 +844,26 @@ int launch_persistent(Kern kern, LaunchCache& cache, size_t smem, const SliceArg
   return launch_maybe_pdl(kern, grid, kThreads, smem, stream, pdl, a);
 }
 
-template <int N, int M, bool TAU1, bool DEFER>
+template <int N, int M, bool TAU1>
 int slice_fwd(const SliceArgs& a, cudaStream_t stream, bool pdl) {
   static LaunchCache cache;
-  return launch_persistent(roi_slice_fwd_kernel<N, M, TAU1, DEFER>, cache, kFwdDeferOffset + kDeferBytes, a, stream,
-                           pdl);
+  return launch_persistent(roi_slice_fwd_kernel<N, M, TAU1>, cache, kFwdDeferOffset + kDeferBytes, a, stream, pdl);
 }
-template <int N, int M, bool TAU1, bool DEFER>
+template <int N, int M, bool TAU1>
 int slice_bwd(const SliceArgs& a, cudaStream_t stream, bool pdl) {
   static LaunchCache cache;
   constexpr size_t smem = kSliceDeferOffset<N, M> + kDeferBytes;
   static_assert(smem <= 232448, "shared memory per CTA");
-  return launch_persistent(roi_slice_bwd_kernel<N, M, TAU1, DEFER>, cache, smem, a, stream, pdl);
+  return launch_persistent(roi_slice_bwd_kernel<N, M, TAU1>, cache, smem, a, stream, pdl);
 }
 
 template <int N, int M>
 int slice_fwd_nm(const SliceArgs& a, cudaStream_t stream, bool pdl) {
-  if (a.tau == 1.0f) return slice_fwd<N, M, true, M == 16>(a, stream, pdl);
-  if constexpr (M == 16) {
-    return slice_fwd<N, M, false, true>(a, stream, pdl);
-  } else {
-    return a.tau < kDeferBelowTau ? slice_fwd<N, M, false, true>(a, stream, pdl)
-                                  : slice_fwd<N, M, false, false>(a, stream, pdl);
-  }
+  return a.tau == 1.0f ? slice_fwd<N, M, true>(a, stream, pdl) : slice_fwd<N, M, false>(a, stream, pdl);
 }
 template <int N, int M>
 int slice_bwd_nm(const SliceArgs& a, cudaStream_t stream, bool pdl) {
-  if (a.tau == 1.0f) return slice_bwd<N, M, true, M == 16>(a, stream, pdl);
-  if constexpr (M == 16) {
-    return slice_bwd<N, M, false, true>(a, stream, pdl);
-  } else {
-    return a.tau < kDeferBelowTau ? slice_bwd<N, M, false, true>(a, stream, pdl)
-                                  : slice_bwd<N, M, false, false>(a, stream, pdl);
-  }
+  return a.tau == 1.0f ? slice_bwd<N, M, true>(a, stream, pdl) : slice_bwd<N, M, false>(a, stream, pdl);
 }
 
 }  // namespace

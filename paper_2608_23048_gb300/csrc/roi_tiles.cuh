@@ -74,12 +74,13 @@ __device__ __forceinline__ bool run_tiles_src(uint8_t* smem, const uint32_t (&es
   }
   __syncthreads();
 
+  const uint64_t lim = ring_wait_limit(status);
   // stage index and mbarrier phase advance incrementally (no 64-bit division)
   int s = 0;
   uint32_t parity = 0;
   int64_t tile = first;
   for (int64_t i = 0; i < my_tiles; ++i, tile += stride) {
-    if (!mbar_wait_ring(&bars[s], parity, status)) {
+    if (!mbar_wait_ring(&bars[s], parity, lim)) {
       if (lane == 0) {
         atomicOr(status, kStatusTimeout);
         // let copies still in flight land before the CTA's shared memory is released

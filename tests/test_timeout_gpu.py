@@ -1,8 +1,8 @@
 """The timeout path of the kernels' bounded waits, run on valid copies.
 
-roi_set_ring_wait_limit_ns(0) makes a kernel's wait for a stage of its copy ring
-give up as soon as it finds the stage not yet landed, which the first tile of
-every CTA is (its copies were issued moments before).  The kernel must then set
+roi_set_ring_wait_limit_ns(0) makes every wait of a kernel for a stage of its copy
+ring give up at once (landed or not), so each CTA gives up at its first tile, with
+its first copies possibly still in flight.  The kernel must then set
 ROI_ERR_TIMEOUT in the device status, let its own copies in flight land (those
 drain waits keep their fixed limit), and return.  With the limit restored, the
 next calls on the same CUDA context run normally: their outputs equal, bit for
