@@ -278,6 +278,26 @@ def test_wide_key_gaps_take_exact_path(roi, N, M, tau):
     check_against_oracle(got, phi.numpy(), WL.bf16_bits(W), WL.bf16_bits(dWm), N, M, tau, 3, 0, 0, 1.0, 0)
 
 
+@pytest.mark.parametrize("N,M", [(2, 4), (4, 8), (8, 16), (16, 32)])
+def test_every_group_out_of_range(roi, N, M):
+    """Every group leaves the fast paths' range at tau = 0.05: the logits of a group
+    are 20 natural-log units apart (a random permutation of 0, 20, 40, ... per group),
+    so each step's top key leads the next by far more than the ~3.5 units the fast
+    path's float range allows, and each step takes one member cleanly (a well-
+    conditioned input, unlike spreads where consumed members come back).  The
+    per-warp queues of the exact routine then fill tile after tile (32 drained at a
+    time) over several tiles and a ragged tail; results match the oracle."""
+    import torch
+    rows, cols = 40, 4160
+    W, _, dWm, *_ = make(rows, cols, "normal", data_seed=17)
+    g = torch.Generator().manual_seed(18)
+    perm = torch.argsort(torch.rand(rows * cols // M, M, generator=g), dim=1).float()
+    phi = (20.0 * perm).reshape(rows, cols).contiguous()
+    st = roi.NoiseState(9, 4, 3, 1.0, 0)
+    got = gpu_run(roi, phi, W, dWm, N, M, 0.05, st)
+    check_against_oracle(got, phi.numpy(), WL.bf16_bits(W), WL.bf16_bits(dWm), N, M, 0.05, 9, 4, 3, 1.0, 0)
+
+
 @pytest.mark.parametrize("rows,cols", [(4, 64), (8, 2112)])
 def test_non_finite_logits_propagate(roi, rows, cols):
     """NaN / +inf logits make their group's outputs NaN (for N = 1 a +inf member
