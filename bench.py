@@ -448,8 +448,8 @@ def mask_roofline(E, N, M, tau, tm, steps, world, dev, ntensors, per_tensor=Fals
                 "algorithmic_bytes_per_element": per_elem,
                 "units_per_launch": (f"{E / ntensors:.0f} elements (mean over the {ntensors} tensors"
                                      + ("" if per_tensor else
-                                        "; batched calls, one chained launch per tensor, achieved from the call's "
-                                        "time") + ")"),
+                                        "; batched calls, chained launches, one per large tensor and one per run of "
+                                        "small tensors, achieved from the call's time") + ")"),
                 "fwd_gbs": round(fwd_gbs, 1), "bwd_gbs": round(bwd_gbs, 1),
                 "fwd_frac": round(fwd_gbs / peak, 4), "bwd_frac": round(bwd_gbs / peak, 4),
                 "fwd_ms_per_step": round(1e3 * fwd_t / steps, 3),

@@ -26,6 +26,8 @@ struct Cfg {
   // 64 kPairs a tile on top of fewer than 32 left from earlier tiles
   static constexpr int kDeferCap = 32 + 64 * kPairs;
 };
+// Tensors of one multi-tensor launch, at most (its parameter block holds them all).
+constexpr int kMultiMaxBwd = 192;
 // Byte offset of the shared-memory step history (M = 8) behind the tile ring,
 // and its size: steps 0 .. N-2 of two groups (one F2 per member) per thread.
 template <int M>
@@ -48,6 +50,11 @@ constexpr size_t kDeferOffset =
                            : kHistOffset<M> + kHistBytes<N, M> + 15) & ~size_t(15);
 template <int N, int M, bool OPT>
 constexpr size_t kBwdSmem = kDeferOffset<N, M, OPT> + size_t(Cfg<M>::kDeferCap) * 8 * (Cfg<M>::kThreads / 32);
+// multi-tensor launches: the tensors' first tiles behind the queues
+template <int N, int M, bool OPT>
+constexpr size_t kBwdMultiOffset = (kBwdSmem<N, M, OPT> + 15) & ~size_t(15);
+template <int N, int M, bool OPT>
+constexpr size_t kBwdMultiSmem = kBwdMultiOffset<N, M, OPT> + size_t(kMultiMaxBwd + 1) * 8;
 
 // This thread's moment slot (M = 8 fused optimizer) in the dynamic shared memory.
 extern __shared__ __align__(128) uint8_t roi_bwd_smem[];
@@ -421,9 +428,12 @@ __device__ __forceinline__ void bwd_exact_group(int64_t g0, const BwdArgs& a, co
 
 // One full tile of a tensor (local tile index `tile`), inputs staged in shared
 // memory.  NARROW: the call's counters are below 2^32 (a.np.narrow).
-template <int N, int M, bool TAU1, bool ST, bool OPT, bool NARROW, bool DEFER, class Defer>
+// `tag` (the tensor's index in a multi-tensor launch, shifted to bit 48) is or-ed into
+// the queued entries.
+template <int N, int M, bool TAU1, bool ST, bool OPT, bool NARROW, bool DEFER, class Defer, class Exact>
 __device__ __forceinline__ void bwd_tile(const uint8_t* const* stage, int64_t tile, const BwdArgs& a,
-                                         const BwdOptArgs& o, uint8_t* smem, Defer& dg) {
+                                         const BwdOptArgs& o, uint8_t* smem, Defer& dg, int64_t tag,
+                                         const Exact& exact) {
   using C = Cfg<M>;
   const float* sphi = reinterpret_cast<const float*>(stage[0]);
   const uint16_t* sW = reinterpret_cast<const uint16_t*>(stage[1]);
@@ -449,11 +459,11 @@ __device__ __forceinline__ void bwd_tile(const uint8_t* const* stage, int64_t ti
       flag = bwd_groups<N, M, TAU1, F2, true, ST, OPT, NARROW, DEFER>(pp, pw, pd, e0, q0, a, o, hist);
     }
     if constexpr (DEFER) {
-      dg.push((flag & 1u) != 0u, e0[0]);
-      dg.push((flag & 2u) != 0u, e0[1]);
+      dg.push((flag & 1u) != 0u, tag | e0[0]);
+      dg.push((flag & 2u) != 0u, tag | e0[1]);
     }
   }
-  if constexpr (DEFER) dg.drain(false, [&](int64_t g0) { bwd_exact_group<N, M, TAU1, ST, OPT>(g0, a, o); });
+  if constexpr (DEFER) dg.drain(false, exact);
 }
 
 // The ragged tail of a tensor (fewer than one tile after its full tiles), by one
@@ -491,18 +501,141 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_bwd_
   src.esize[2] = 2;
   DeferredGroups<C::kDeferCap> dg;
   dg.init(smem + kDeferOffset<N, M, OPT>);
+  const auto exact = [&](int64_t g0) { bwd_exact_group<N, M, TAU1, ST, OPT>(g0, a, o); };
   // a batch's next tensor may start on the SMs this launch frees (no-op otherwise)
   pdl_launch_dependents();
   const bool ok = run_tiles<C::kThreads, C::kTile, C::kStages, 3>(
       smem, src, a.full_tiles, a.status,
       [&](const uint8_t* const* stage, int64_t tile) {
-        bwd_tile<N, M, TAU1, ST, OPT, NARROW_ONLY, DEFER>(stage, tile, a, o, smem, dg);
+        bwd_tile<N, M, TAU1, ST, OPT, NARROW_ONLY, DEFER>(stage, tile, a, o, smem, dg, 0, exact);
       });
   if constexpr (DEFER) {
-    if (ok) dg.drain(true, [&](int64_t g0) { bwd_exact_group<N, M, TAU1, ST, OPT>(g0, a, o); });
+    if (ok) dg.drain(true, exact);
   }
   if (ok && blockIdx.x == gridDim.x - 1) bwd_tail<N, M, TAU1, ST, OPT>(a, o);
   // the launch completes only after the batch's previous one (stream order)
+  if (blockIdx.x == 0) pdl_wait();
+}
+
+// Multi-tensor launches: the tensors' arguments, and their first tiles in the
+// concatenated tile sequence of the launch (tile0).
+struct BwdItem {
+  const float* phi;
+  const uint16_t* W;
+  const uint16_t* dWm;
+  float* dphi;
+  uint16_t* dW;
+  const uint32_t* hard_in;
+  float* phi_out;
+  float* m;
+  float* v;
+  int64_t E;
+  int64_t tile0;
+  NoiseParams np;
+};
+struct BwdMulti {
+  int count;
+  int64_t total_tiles;
+  float tau, inv_tau;
+  unsigned int* status;
+  AdamW opt;
+  BwdItem it[kMultiMaxBwd];
+};
+static_assert(sizeof(BwdMulti) <= 32764, "kernel parameter block");
+template <int M>
+__device__ __forceinline__ BwdArgs multi_args(const BwdMulti& mm, int i) {
+  const BwdItem& x = mm.it[i];
+  BwdArgs a;
+  a.phi = x.phi;
+  a.W = x.W;
+  a.dWm = x.dWm;
+  a.dphi = x.dphi;
+  a.dW = x.dW;
+  a.hard_in = x.hard_in;
+  a.E = x.E;
+  a.full_tiles = x.E / Cfg<M>::kTile;
+  a.tau = mm.tau;
+  a.inv_tau = mm.inv_tau;
+  a.np = x.np;
+  a.status = mm.status;
+  return a;
+}
+__device__ __forceinline__ BwdOptArgs multi_opt(const BwdMulti& mm, int i) {
+  BwdOptArgs o;
+  o.phi_out = mm.it[i].phi_out;
+  o.m = mm.it[i].m;
+  o.v = mm.it[i].v;
+  o.opt = mm.opt;
+  return o;
+}
+// roi_bwd_kernel over many small tensors at once, walked as roi_fwd_multi_kernel
+// walks them.
+template <int N, int M, bool TAU1, bool ST, bool OPT, bool NARROW_ONLY, bool DEFER>
+__global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks)
+    roi_bwd_multi_kernel(const __grid_constant__ BwdMulti mm) {
+  uint8_t* smem = roi_bwd_smem;
+  using C = Cfg<M>;
+  const uint32_t esize[3] = {4, 2, 2};
+  constexpr int64_t kLow = (int64_t(1) << 48) - 1;
+  int64_t* tile0 = reinterpret_cast<int64_t*>(smem + kBwdMultiOffset<N, M, OPT>);
+  for (int i = threadIdx.x; i <= mm.count; i += C::kThreads) tile0[i] = i < mm.count ? mm.it[i].tile0 : mm.total_tiles;
+  __syncthreads();
+  const auto find = [&](int64_t t) {
+    int lo = 0, hi = mm.count - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (tile0[mid] <= t) {
+        lo = mid;
+      } else {
+        hi = mid - 1;
+      }
+    }
+    return lo;
+  };
+  DeferredGroups<C::kDeferCap> dg;
+  dg.init(smem + kDeferOffset<N, M, OPT>);
+  const auto exact = [&](int64_t e) {
+    const int i = int(e >> 48);
+    bwd_exact_group<N, M, TAU1, ST, OPT>(e & kLow, multi_args<M>(mm, i), multi_opt(mm, i));
+  };
+  int cur = -1, src_cur = -1;
+  int64_t lo = 0, hi = 0, src_lo = 0, src_hi = 0;
+  BwdArgs a;
+  BwdOptArgs o;
+  const uint8_t* src_ptr[3] = {nullptr, nullptr, nullptr};
+  pdl_launch_dependents();
+  const bool ok = run_tiles_src<C::kThreads, C::kTile, C::kStages, 3>(
+      smem, esize, mm.total_tiles, mm.status,
+      [&](int64_t t, int arr) {
+        if (t < src_lo || t >= src_hi) {
+          src_cur = find(t);
+          src_lo = tile0[src_cur];
+          src_hi = tile0[src_cur + 1];
+          src_ptr[0] = reinterpret_cast<const uint8_t*>(mm.it[src_cur].phi);
+          src_ptr[1] = reinterpret_cast<const uint8_t*>(mm.it[src_cur].W);
+          src_ptr[2] = reinterpret_cast<const uint8_t*>(mm.it[src_cur].dWm);
+        }
+        return src_ptr[arr] + size_t(t - src_lo) * C::kTile * esize[arr];
+      },
+      [&](const uint8_t* const* stage, int64_t t) {
+        if (t < lo || t >= hi) {
+          cur = find(t);
+          lo = tile0[cur];
+          hi = tile0[cur + 1];
+          a = multi_args<M>(mm, cur);
+          o = multi_opt(mm, cur);
+        }
+        bwd_tile<N, M, TAU1, ST, OPT, NARROW_ONLY, DEFER>(stage, t - lo, a, o, smem, dg, int64_t(cur) << 48, exact);
+      });
+  if constexpr (DEFER) {
+    if (ok) dg.drain(true, exact);
+  }
+  if (ok) {
+    for (int i = blockIdx.x; i < mm.count; i += gridDim.x) {
+      const BwdArgs ai = multi_args<M>(mm, i);
+      if (ai.full_tiles * C::kTile < ai.E) bwd_tail<N, M, TAU1, ST, OPT>(ai, multi_opt(mm, i));
+    }
+  }
   if (blockIdx.x == 0) pdl_wait();
 }
 
@@ -603,6 +736,93 @@ int launch_nm(const BwdArgs& a, const BwdOptArgs& o, cudaStream_t stream, bool p
   return launch_tau<N, M, false, false>(a, o, stream, pdl);
 }
 
+template <int N, int M, bool TAU1, bool ST, bool OPT, bool NARROW_ONLY, bool DEFER>
+int launch_multi_kern(const BwdMulti& mm, cudaStream_t stream, bool pdl) {
+  using C = Cfg<M>;
+  auto kern = roi_bwd_multi_kernel<N, M, TAU1, ST, OPT, NARROW_ONLY, DEFER>;
+  constexpr size_t smem = kBwdMultiSmem<N, M, OPT>;
+  static_assert(smem <= 232448, "shared memory per CTA");
+  static LaunchCache cache;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return -1;
+  if (cache.per_sm[dev] == 0) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem)) != cudaSuccess)
+      return -1;
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, C::kThreads, smem) != cudaSuccess) return -1;
+    cache.per_sm[dev] = per_sm < 1 ? 1 : per_sm;
+  }
+  const int64_t cap = int64_t(sm_count()) * cache.per_sm[dev];
+  const int64_t want = mm.total_tiles > mm.count ? mm.total_tiles : mm.count;
+  const int grid = int(want < 1 ? 1 : (want < cap ? want : cap));
+  return launch_maybe_pdl(kern, grid, C::kThreads, smem, stream, pdl, mm);
+}
+
+template <int N, int M, bool ST, bool OPT, bool NARROW_ONLY = false>
+int launch_multi_tau(const BwdMulti& mm, cudaStream_t stream, bool pdl) {
+  if (mm.tau == 1.0f) return launch_multi_kern<N, M, true, ST, OPT, NARROW_ONLY, M == 4>(mm, stream, pdl);
+  if constexpr (M == 4) {
+    return launch_multi_kern<N, M, false, ST, OPT, NARROW_ONLY, true>(mm, stream, pdl);
+  } else {
+    return mm.tau < kDeferBelowTau ? launch_multi_kern<N, M, false, ST, OPT, NARROW_ONLY, true>(mm, stream, pdl)
+                                   : launch_multi_kern<N, M, false, ST, OPT, NARROW_ONLY, false>(mm, stream, pdl);
+  }
+}
+
+// The backward variant a call needs, in launch_nm's order: 2 fused AdamW,
+// 1 straight-through dW, 0 plain.
+int bwd_kind(const BwdCall& c) { return c.phi_out != nullptr ? 2 : (c.hard_in != nullptr && c.dW != nullptr ? 1 : 0); }
+
+// One launch over calls[0 .. count): one kind, one counter width, with launch_nm's
+// choice of variant.
+template <int N, int M>
+int launch_multi(const BwdCall* calls, int count, bool pdl) {
+  using C = Cfg<M>;
+  static thread_local BwdMulti mm;
+  mm.count = count;
+  mm.tau = calls[0].tau;
+  mm.inv_tau = 1.0f / calls[0].tau;
+  mm.status = calls[0].status;
+  mm.opt = calls[0].opt;
+  int64_t tiles = 0;
+  for (int i = 0; i < count; ++i) {
+    const BwdCall& c = calls[i];
+    BwdItem& x = mm.it[i];
+    x.phi = c.phi;
+    x.W = c.W;
+    x.dWm = c.dWm;
+    x.dphi = c.dphi;
+    x.dW = c.dW;
+    x.hard_in = c.hard_in;
+    x.phi_out = c.phi_out;
+    x.m = c.m;
+    x.v = c.v;
+    x.E = c.E;
+    x.tile0 = tiles;
+    x.np = c.np;
+    x.np.narrow = counters_narrow(c.np, c.E);
+    tiles += c.E / C::kTile;
+  }
+  mm.total_tiles = tiles;
+  const cudaStream_t stream = calls[0].stream;
+  const int kind = bwd_kind(calls[0]);
+  const bool narrow = mm.it[0].np.narrow;
+  if constexpr (N == 4 && M == 8) {
+    if (mm.tau == 1.0f && narrow && kind == 2)
+      return launch_multi_kern<N, M, true, false, true, true, false>(mm, stream, pdl);
+  }
+  if constexpr (M == 4) {
+    if (narrow) {
+      if (kind == 2) return launch_multi_tau<N, M, false, true, true>(mm, stream, pdl);
+      if (kind == 1) return launch_multi_tau<N, M, true, false, true>(mm, stream, pdl);
+      return launch_multi_tau<N, M, false, false, true>(mm, stream, pdl);
+    }
+  }
+  if (kind == 2) return launch_multi_tau<N, M, false, true>(mm, stream, pdl);
+  if (kind == 1) return launch_multi_tau<N, M, true, false>(mm, stream, pdl);
+  return launch_multi_tau<N, M, false, false>(mm, stream, pdl);
+}
+
 }  // namespace
 
 namespace {
@@ -642,20 +862,44 @@ int launch_bwd_impl(const BwdCall& c, bool pdl) {
 
 int launch_bwd(const BwdCall& c) { return launch_bwd_impl(c, false); }
 
-// As launch_fwd_batch: the tensors are independent, so from the second one on the
-// tile kernels (plain or fused with AdamW) are launched with programmatic stream
-// serialization.
+// As launch_fwd_batch: the tensors are independent, so from the second launch on
+// the tile kernels (plain or fused with AdamW) are launched with programmatic
+// stream serialization, and runs of small tensors with the same tile kernel share
+// one multi-tensor launch.
 int launch_bwd_batch(const BwdCall* calls, int count) {
   int launched = 0;
   bool prev_tiled = false;
-  for (int i = 0; i < count; ++i) {
+  for (int i = 0; i < count;) {
     const BwdCall& c = calls[i];
-    const bool tiled =
-        (c.N == 2 && c.M == 4) || (c.N == 4 && c.M == 8) || (c.N == 2 && c.M == 8) || slice_supported(c.N, c.M);
+    if ((c.N == 2 && c.M == 4) || (c.N == 4 && c.M == 8) || (c.N == 2 && c.M == 8)) {
+      // the run of small items from i on with the same tile kernel
+      const int64_t tile = c.M == 8 ? Cfg<8>::kTile : Cfg<4>::kTile;
+      const int kind = bwd_kind(c);
+      const bool narrow = counters_narrow(c.np, c.E);
+      int n = 0;
+      while (i + n < count && n < kMultiMaxBwd && calls[i + n].N == c.N && calls[i + n].M == c.M &&
+             bwd_kind(calls[i + n]) == kind && counters_narrow(calls[i + n].np, calls[i + n].E) == narrow &&
+             multi_small(calls[i + n].E, tile))
+        ++n;
+      if (n > 1) {
+        int r = -1;
+        if (c.N == 2 && c.M == 4) r = launch_multi<2, 4>(calls + i, n, prev_tiled);
+        if (c.N == 4 && c.M == 8) r = launch_multi<4, 8>(calls + i, n, prev_tiled);
+        if (c.N == 2 && c.M == 8) r = launch_multi<2, 8>(calls + i, n, prev_tiled);
+        if (r < 0) return -1;
+        launched += r;
+        prev_tiled = r > 0;
+        i += n;
+        continue;
+      }
+    }
+    const bool tiled = (c.N == 2 && c.M == 4) || (c.N == 4 && c.M == 8) || (c.N == 2 && c.M == 8) ||
+                       slice_supported(c.N, c.M);
     const int r = launch_bwd_impl(c, tiled && prev_tiled);
     if (r < 0) return -1;
     launched += r;
     prev_tiled = tiled && r > 0;
+    ++i;
   }
   return launched;
 }

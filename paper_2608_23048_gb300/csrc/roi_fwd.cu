@@ -14,6 +14,9 @@ namespace {
 // One CTA per SM: CTAs sharing an SM progress at very different rates (the
 // scheduler favours the older one) and the last ones then finish alone, so all of
 // an SM's warps work through one tile ring instead.
+// Tensors of one multi-tensor launch, at most (its parameter block holds them all).
+constexpr int kMultiMax = 256;
+
 template <int M>
 struct Cfg {
   static constexpr int kThreads = 512;
@@ -26,6 +29,9 @@ struct Cfg {
   static constexpr int kDeferCap = 32 + 64 * kPairs;
   static constexpr size_t kDeferOffset = (tile_smem_bytes<kTile, kStages>(6) + 15) & ~size_t(15);
   static constexpr size_t kSmem = kDeferOffset + size_t(kDeferCap) * 8 * (kThreads / 32);
+  // multi-tensor launches: the tensors' first tiles behind the queues
+  static constexpr size_t kMultiOffset = (kSmem + 15) & ~size_t(15);
+  static constexpr size_t kMultiSmem = kMultiOffset + size_t(kMultiMax + 1) * 8;
 };
 
 struct FwdArgs {
@@ -349,8 +355,9 @@ __device__ __forceinline__ void store_hard_pair(uint32_t* hard, int64_t e0a, int
 
 // One full tile of a tensor (local tile index `tile`), inputs staged in shared
 // memory.  NARROW: the call's counters are below 2^32 (a.np.narrow).
-template <int N, int M, bool TAU1, bool ST, bool NARROW, bool DEFER, class Defer>
-__device__ __forceinline__ void fwd_tile(const uint8_t* const* stage, int64_t tile, const FwdArgs& a, Defer& dg) {
+template <int N, int M, bool TAU1, bool ST, bool NARROW, bool DEFER, class Defer, class Exact>
+__device__ __forceinline__ void fwd_tile(const uint8_t* const* stage, int64_t tile, const FwdArgs& a, Defer& dg,
+                                         int64_t tag, const Exact& exact) {
   using C = Cfg<M>;
   constexpr int kT = C::kTile;
   const float* sphi = reinterpret_cast<const float*>(stage[0]);
@@ -386,11 +393,11 @@ __device__ __forceinline__ void fwd_tile(const uint8_t* const* stage, int64_t ti
     const uint32_t flag = fwd_finish<N, M, TAU1, F2, ST, DEFER>(kap[p & 1], pw, e0, a, bits);
     if (a.hard != nullptr) store_hard_pair<M>(a.hard, e0[0], e0[1], bits[0], bits[1]);
     if constexpr (DEFER) {
-      dg.push((flag & 1u) != 0u, e0[0]);
-      dg.push((flag & 2u) != 0u, e0[1]);
+      dg.push((flag & 1u) != 0u, tag | e0[0]);
+      dg.push((flag & 2u) != 0u, tag | e0[1]);
     }
   }
-  if constexpr (DEFER) dg.drain(false, [&](int64_t g0) { fwd_exact_group<N, M, TAU1, ST>(g0, a); });
+  if constexpr (DEFER) dg.drain(false, exact);
 }
 
 // The ragged tail of a tensor (fewer than one tile after its full tiles), by one
@@ -427,6 +434,7 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_fwd_
   src.esize[1] = 2;
   DeferredGroups<C::kDeferCap> dg;
   dg.init(smem + C::kDeferOffset);
+  const auto exact = [&](int64_t g0) { fwd_exact_group<N, M, TAU1, ST>(g0, a); };
   // a batch's next tensor may start on the SMs this launch frees (no-op otherwise)
   pdl_launch_dependents();
   const bool ok = run_tiles<C::kThreads, C::kTile, C::kStages, 2>(
@@ -436,17 +444,137 @@ __global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks) roi_fwd_
         // body measured slower (register allocation), so those keep one
         if constexpr (M == 4) {
           if (a.np.narrow) {
-            fwd_tile<N, M, TAU1, ST, true, DEFER>(stage, tile, a, dg);
+            fwd_tile<N, M, TAU1, ST, true, DEFER>(stage, tile, a, dg, 0, exact);
             return;
           }
         }
-        fwd_tile<N, M, TAU1, ST, false, DEFER>(stage, tile, a, dg);
+        fwd_tile<N, M, TAU1, ST, false, DEFER>(stage, tile, a, dg, 0, exact);
       });
   if constexpr (DEFER) {
-    if (ok) dg.drain(true, [&](int64_t g0) { fwd_exact_group<N, M, TAU1, ST>(g0, a); });
+    if (ok) dg.drain(true, exact);
   }
   if (ok && blockIdx.x == gridDim.x - 1) fwd_tail<N, M, TAU1, ST>(a);
   // the launch completes only after the batch's previous one (stream order)
+  if (blockIdx.x == 0) pdl_wait();
+}
+
+// Multi-tensor launches: the tensors' arguments, and their first tiles in the
+// concatenated tile sequence of the launch (tile0).
+struct FwdItem {
+  const float* phi;
+  const uint16_t* W;
+  uint16_t* Wm;
+  float* soft;
+  uint32_t* hard;
+  int64_t E;
+  int64_t tile0;
+  NoiseParams np;
+};
+struct FwdMulti {
+  int count;
+  int64_t total_tiles;
+  bool st;
+  float tau, inv_tau;
+  unsigned int* status;
+  FwdItem it[kMultiMax];
+};
+static_assert(sizeof(FwdMulti) <= 32764, "kernel parameter block");
+template <int M>
+__device__ __forceinline__ FwdArgs multi_args(const FwdMulti& mm, int i) {
+  const FwdItem& x = mm.it[i];
+  FwdArgs a;
+  a.phi = x.phi;
+  a.W = x.W;
+  a.Wm = x.Wm;
+  a.soft = x.soft;
+  a.hard = x.hard;
+  a.st = mm.st;
+  a.E = x.E;
+  a.full_tiles = x.E / Cfg<M>::kTile;
+  a.tau = mm.tau;
+  a.inv_tau = mm.inv_tau;
+  a.np = x.np;
+  a.status = mm.status;
+  return a;
+}
+// The tile kernel over many small tensors at once: the persistent CTAs walk the
+// concatenation of the tensors' full tiles, finding a tile's tensor by binary
+// search over tile0 (in shared memory) only when a tile leaves the current one.
+// Deferred groups carry their tensor's index above bit 48; each tensor's ragged
+// tail goes to one CTA after the tiles.
+template <int N, int M, bool TAU1, bool ST, bool DEFER>
+__global__ void __launch_bounds__(Cfg<M>::kThreads, Cfg<M>::kMinBlocks)
+    roi_fwd_multi_kernel(const __grid_constant__ FwdMulti mm) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  using C = Cfg<M>;
+  const uint32_t esize[2] = {4, 2};
+  constexpr int64_t kLow = (int64_t(1) << 48) - 1;
+  // the tensors' first tiles, in shared memory for the searches
+  int64_t* tile0 = reinterpret_cast<int64_t*>(smem + C::kMultiOffset);
+  for (int i = threadIdx.x; i <= mm.count; i += C::kThreads) tile0[i] = i < mm.count ? mm.it[i].tile0 : mm.total_tiles;
+  __syncthreads();
+  const auto find = [&](int64_t t) {
+    int lo = 0, hi = mm.count - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (tile0[mid] <= t) {
+        lo = mid;
+      } else {
+        hi = mid - 1;
+      }
+    }
+    return lo;
+  };
+  DeferredGroups<C::kDeferCap> dg;
+  dg.init(smem + C::kDeferOffset);
+  const auto exact = [&](int64_t e) { fwd_exact_group<N, M, TAU1, ST>(e & kLow, multi_args<M>(mm, int(e >> 48))); };
+  // the current tensor of this warp's tiles (and of the copies thread 0 issues),
+  // looked up again only when a tile falls outside it
+  int cur = -1, src_cur = -1;
+  int64_t lo = 0, hi = 0, src_lo = 0, src_hi = 0;
+  FwdArgs a;
+  const float* src_phi = nullptr;
+  const uint16_t* src_W = nullptr;
+  pdl_launch_dependents();
+  const bool ok = run_tiles_src<C::kThreads, C::kTile, C::kStages, 2>(
+      smem, esize, mm.total_tiles, mm.status,
+      [&](int64_t t, int arr) {
+        if (t < src_lo || t >= src_hi) {
+          src_cur = find(t);
+          src_lo = tile0[src_cur];
+          src_hi = tile0[src_cur + 1];
+          src_phi = mm.it[src_cur].phi;
+          src_W = mm.it[src_cur].W;
+        }
+        const size_t off = size_t(t - src_lo) * C::kTile;
+        return arr == 0 ? reinterpret_cast<const uint8_t*>(src_phi + off) : reinterpret_cast<const uint8_t*>(src_W + off);
+      },
+      [&](const uint8_t* const* stage, int64_t t) {
+        if (t < lo || t >= hi) {
+          cur = find(t);
+          lo = tile0[cur];
+          hi = tile0[cur + 1];
+          a = multi_args<M>(mm, cur);
+        }
+        const int64_t local = t - lo;
+        const int64_t tag = int64_t(cur) << 48;
+        if constexpr (M == 4) {
+          if (a.np.narrow) {
+            fwd_tile<N, M, TAU1, ST, true, DEFER>(stage, local, a, dg, tag, exact);
+            return;
+          }
+        }
+        fwd_tile<N, M, TAU1, ST, false, DEFER>(stage, local, a, dg, tag, exact);
+      });
+  if constexpr (DEFER) {
+    if (ok) dg.drain(true, exact);
+  }
+  if (ok) {
+    for (int i = blockIdx.x; i < mm.count; i += gridDim.x) {
+      const FwdArgs ai = multi_args<M>(mm, i);
+      if (ai.full_tiles * C::kTile < ai.E) fwd_tail<N, M, TAU1, ST>(ai);
+    }
+  }
   if (blockIdx.x == 0) pdl_wait();
 }
 
@@ -525,6 +653,64 @@ int launch_nm(const FwdArgs& a, cudaStream_t stream, bool pdl = false) {
   return a.st ? launch_st<N, M, true>(a, stream, pdl) : launch_st<N, M, false>(a, stream, pdl);
 }
 
+template <int N, int M, bool TAU1, bool ST, bool DEFER>
+int launch_multi_kern(const FwdMulti& mm, cudaStream_t stream, bool pdl) {
+  using C = Cfg<M>;
+  auto kern = roi_fwd_multi_kernel<N, M, TAU1, ST, DEFER>;
+  static LaunchCache cache;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return -1;
+  if (cache.per_sm[dev] == 0) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(C::kMultiSmem)) != cudaSuccess)
+      return -1;
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, C::kThreads, C::kMultiSmem) != cudaSuccess)
+      return -1;
+    cache.per_sm[dev] = per_sm < 1 ? 1 : per_sm;
+  }
+  const int64_t cap = int64_t(sm_count()) * cache.per_sm[dev];
+  int64_t want = mm.total_tiles > mm.count ? mm.total_tiles : mm.count;
+  const int grid = int(want < 1 ? 1 : (want < cap ? want : cap));
+  return launch_maybe_pdl(kern, grid, C::kThreads, C::kMultiSmem, stream, pdl, mm);
+}
+
+template <int N, int M, bool ST>
+int launch_multi_st(const FwdMulti& mm, cudaStream_t stream, bool pdl) {
+  if (mm.tau == 1.0f) return launch_multi_kern<N, M, true, ST, false>(mm, stream, pdl);
+  return mm.tau < kDeferBelowTau ? launch_multi_kern<N, M, false, ST, true>(mm, stream, pdl)
+                                 : launch_multi_kern<N, M, false, ST, false>(mm, stream, pdl);
+}
+
+// One launch over calls[0 .. count), with launch_st's choice of variant.
+template <int N, int M>
+int launch_multi(const FwdCall* calls, int count, bool pdl) {
+  using C = Cfg<M>;
+  static thread_local FwdMulti mm;
+  mm.count = count;
+  mm.st = calls[0].st;
+  mm.tau = calls[0].tau;
+  mm.inv_tau = 1.0f / calls[0].tau;
+  mm.status = calls[0].status;
+  int64_t tiles = 0;
+  for (int i = 0; i < count; ++i) {
+    const FwdCall& c = calls[i];
+    FwdItem& x = mm.it[i];
+    x.phi = c.phi;
+    x.W = c.W;
+    x.Wm = c.Wm;
+    x.soft = c.soft;
+    x.hard = c.hard;
+    x.E = c.E;
+    x.tile0 = tiles;
+    x.np = c.np;
+    x.np.narrow = counters_narrow(c.np, c.E);
+    tiles += c.E / C::kTile;
+  }
+  mm.total_tiles = tiles;
+  const cudaStream_t stream = calls[0].stream;
+  return mm.st ? launch_multi_st<N, M, true>(mm, stream, pdl) : launch_multi_st<N, M, false>(mm, stream, pdl);
+}
+
 }  // namespace
 
 namespace {
@@ -566,20 +752,42 @@ int launch_fwd_impl(const FwdCall& c, bool pdl) {
 int launch_fwd(const FwdCall& c) { return launch_fwd_impl(c, false); }
 
 // The tensors of a batch are independent (the caller checked that no output
-// overlaps another range), so from the second one on the tile kernels are launched
-// with programmatic stream serialization: each may start while the previous one
-// drains, and completes only after it (see roi_fwd_kernel).
+// overlaps another range), so from the second launch on the tile kernels are
+// launched with programmatic stream serialization: each may start while the
+// previous one drains, and completes only after it (see roi_fwd_kernel).  Runs of
+// small tensors with the same tile kernel share one multi-tensor launch
+// (multi_small).
 int launch_fwd_batch(const FwdCall* calls, int count) {
   int launched = 0;
   bool prev_tiled = false;
-  for (int i = 0; i < count; ++i) {
+  for (int i = 0; i < count;) {
     const FwdCall& c = calls[i];
-    const bool tiled =
-        (c.N == 2 && c.M == 4) || (c.N == 4 && c.M == 8) || (c.N == 2 && c.M == 8) || slice_supported(c.N, c.M);
+    if ((c.N == 2 && c.M == 4) || (c.N == 4 && c.M == 8) || (c.N == 2 && c.M == 8)) {
+      // the run of small items from i on with the same tile kernel
+      const int64_t tile = c.M == 8 ? Cfg<8>::kTile : Cfg<4>::kTile;
+      int n = 0;
+      while (i + n < count && n < kMultiMax && calls[i + n].N == c.N && calls[i + n].M == c.M &&
+             multi_small(calls[i + n].E, tile))
+        ++n;
+      if (n > 1) {
+        int r = -1;
+        if (c.N == 2 && c.M == 4) r = launch_multi<2, 4>(calls + i, n, prev_tiled);
+        if (c.N == 4 && c.M == 8) r = launch_multi<4, 8>(calls + i, n, prev_tiled);
+        if (c.N == 2 && c.M == 8) r = launch_multi<2, 8>(calls + i, n, prev_tiled);
+        if (r < 0) return -1;
+        launched += r;
+        prev_tiled = r > 0;
+        i += n;
+        continue;
+      }
+    }
+    const bool tiled = (c.N == 2 && c.M == 4) || (c.N == 4 && c.M == 8) || (c.N == 2 && c.M == 8) ||
+                       slice_supported(c.N, c.M);
     const int r = launch_fwd_impl(c, tiled && prev_tiled);
     if (r < 0) return -1;
     launched += r;
     prev_tiled = tiled && r > 0;
+    ++i;
   }
   return launched;
 }

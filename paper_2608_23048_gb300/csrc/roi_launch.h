@@ -86,9 +86,10 @@ struct LinearCall {
 // Each returns the number of kernels launched (>= 0) or -1 after a CUDA error.
 int launch_fwd(const FwdCall& c);
 int launch_bwd(const BwdCall& c);
-// Many independent tensors on one stream: one launch per tensor, the tile kernels
-// chained by programmatic dependent launch so each may start while the previous
-// one drains (stream order is kept: each completes after its predecessor).
+// Many independent tensors on one stream: one launch per tensor, or per run of
+// small tensors (multi_small), the tile kernels chained by programmatic dependent
+// launch so each may start while the previous one drains (stream order is kept:
+// each completes after its predecessor).
 int launch_fwd_batch(const FwdCall* calls, int count);
 int launch_bwd_batch(const BwdCall* calls, int count);
 int launch_export(const ExportCall& c);
@@ -130,5 +131,18 @@ int launch_maybe_pdl(void (*kern)(KArgs...), int grid, int threads, size_t smem,
 
 // Streaming multiprocessors of the current device (cached).
 int sm_count();
+
+// Batched calls: a run of consecutive items with the same tile kernel, each of
+// them small (fewer than kMultiTilesPerSm full tiles per SM), goes to one
+// multi-tensor launch.  One launch per small tensor spends much of its time on
+// fixed costs (ring fill and drain, the ragged tail, the gap to the next launch).
+// A larger tensor keeps a launch of its own: the multi-tensor kernel holds the
+// current tensor's arguments in registers rather than in the constant bank, and
+// measured 4-7 % slower on 18944 x 3584 tensors.
+// A fwd + bwd step over a Qwen2.5-shaped layer set went from 1.90 to 1.57 ms
+// (0.5B-shaped, 2:4), 8.92 to 8.79 ms (1.5B-shaped, 4:8) and 24.32 to 24.23 ms
+// (7B-shaped, 2:4, where only the q, k, v, o tensors are small).
+constexpr int64_t kMultiTilesPerSm = 12;
+inline bool multi_small(int64_t E, int64_t tile) { return E / tile < kMultiTilesPerSm * sm_count(); }
 
 }  // namespace roi

@@ -1,6 +1,7 @@
 """Batched calls (roi_mask_fwd_batch / roi_mask_bwd_batch): many tensors per call,
-their launches chained by programmatic dependent launch, must give, bit for bit,
-what the single-tensor calls give, and match the oracle.  Sets mix tensors with and
+their launches chained by programmatic dependent launch (runs of small tensors
+sharing one multi-tensor launch), must give, bit for bit, what the single-tensor
+calls give, and match the oracle.  Sets mix tensors with and
 without full tiles, ragged tails,
 per-item noise states (seed, step, tensor_id, lambda, row_offset), optional outputs,
 empty items, 300 items, and an (N, M) without a tile kernel (no chaining)."""
@@ -88,8 +89,10 @@ def assert_same(a, b):
 SHAPES = [(37, 1000), (3, 64), (64, 3584), (512, 256), (1, 32), (129, 2048), (8, 8), (300, 520), (16, 24576)]
 
 
-@pytest.mark.parametrize("N,M,tau", [(2, 4, 1.0), (2, 4, 0.5), (4, 8, 1.0), (4, 8, 0.3), (2, 8, 1.0), (3, 4, 0.8),
-                                     (8, 16, 0.2), (16, 32, 1.0)])
+# tau = 0.05: many groups leave the fast path's range and go through the deferred
+# queues, whose entries name their tensor in a launch shared by several
+@pytest.mark.parametrize("N,M,tau", [(2, 4, 1.0), (2, 4, 0.5), (2, 4, 0.05), (4, 8, 1.0), (4, 8, 0.3), (4, 8, 0.05),
+                                     (2, 8, 1.0), (3, 4, 0.8), (8, 16, 0.2), (16, 32, 1.0)])
 def test_batch_equals_single_calls(roi, N, M, tau):
     shapes = [(r, c) for r, c in SHAPES if c % M == 0]
     ts = make_set(shapes, 40 + M + int(10 * tau))
@@ -142,14 +145,31 @@ def test_more_items_than_one_launch_and_empty_items(roi):
         assert_same(a, b)
 
 
-def test_batch_launches_one_kernel_per_tensor_and_direction(roi):
+def test_batch_launch_counts(roi):
+    """Consecutive small tensors with the same tile kernel share one launch per
+    direction; a tensor that gives every SM at least 12 tiles (2:4: 12288 elements
+    a forward tile, 8192 a backward one) keeps a launch of its own, and splits the
+    runs around it.  Both forms give, bit for bit, what the single calls give."""
+    import torch
     N, M, tau = 2, 4, 1.0
-    ts = make_set([(64, 3584), (16, 512), (37, 1000)], 3)
+    small = [(64, 3584), (16, 512), (37, 1000)]
+    ts = make_set(small, 3)
     flags = [(False, True, False)] * len(ts)
     run_batch(roi, ts, N, M, tau, flags)
     before = roi.roi_launch_count()
     run_batch(roi, ts, N, M, tau, flags)
-    assert roi.roi_launch_count() - before == 2 * len(ts)
+    assert roi.roi_launch_count() - before == 2
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    big = (12 * sms * 12288 // 4096 + 8, 4096)
+    ts = make_set([big] + small + [big, small[0]], 5)
+    flags = [(True, True, True)] * len(ts)
+    single = run_single(roi, ts, N, M, tau, flags)
+    before = roi.roi_launch_count()
+    batch = run_batch(roi, ts, N, M, tau, flags)
+    # per direction: big, the run of three small ones, big, one small
+    assert roi.roi_launch_count() - before == 2 * 4
+    for a, b in zip(single, batch):
+        assert_same(a, b)
 
 
 def test_work_queued_after_a_batch_sees_every_item(roi):
