@@ -81,6 +81,42 @@ def test_mask_kernels_time_out_then_recover(roi, N, M, tau):
         assert not np.any(np.any(g != w, axis=1) & ~near)
 
 
+def test_multi_tensor_launches_time_out_then_recover(roi):
+    """Batched calls over small tensors (one multi-tensor launch per direction, the
+    CTAs walking every tensor's tiles): a wait that gives up ends the launch the same
+    way, and the next batch on the context gives the first batch's bits."""
+    import torch
+    dev = torch.device("cuda")
+    shapes = [(256, 4096), (64, 1024), (300, 2048), (37, 1000)]
+    ts = []
+    for k, (rows, cols) in enumerate(shapes):
+        W, phi, dWm = WL.make_inputs(rows, cols, "normal", 60 + k, device=dev)
+        ts.append((phi, W, dWm, roi.NoiseState(7, 2, k, 1.0, 0), rows, cols))
+
+    def run():
+        out = []
+        for phi, W, dWm, st, rows, cols in ts:
+            out.append((torch.empty_like(W), torch.empty(roi.hard_words(rows, cols), dtype=torch.int32, device=dev),
+                        torch.empty_like(phi)))
+        roi.roi_mask_fwd_batch([(phi, W, st, o[0], None, o[1]) for (phi, W, dWm, st, r, c), o in zip(ts, out)],
+                               2, 4, 1.0)
+        roi.roi_mask_bwd_batch([(phi, W, st, dWm, o[2], None) for (phi, W, dWm, st, r, c), o in zip(ts, out)],
+                               2, 4, 1.0)
+        return out
+
+    before = run()
+    roi.roi_device_status()
+    launches = roi.roi_launch_count()
+    _expect_timeout(roi, run)
+    assert roi.roi_launch_count() - launches == 2  # one launch per direction
+    after = run()
+    roi.roi_device_status()
+    for x, y in zip(before, after):
+        assert torch.equal(x[0].view(torch.int16), y[0].view(torch.int16))
+        assert torch.equal(x[1], y[1])
+        assert torch.equal(x[2].view(torch.int32), y[2].view(torch.int32))
+
+
 def test_masked_linear_times_out_drains_then_recovers(roi):
     """The tensor-core masked linear: on a wait that gives up, the CTA waits for the
     TMA fills and MMAs it issued before releasing shared memory and TMEM."""
