@@ -769,7 +769,7 @@ int launch_fwd_batch(const FwdCall* calls, int count) {
       while (i + n < count && n < kMultiMax && calls[i + n].N == c.N && calls[i + n].M == c.M &&
              multi_small(calls[i + n].E, tile))
         ++n;
-      if (n > 1) {
+      if (n >= multi_min_run(false)) {
         int r = -1;
         if (c.N == 2 && c.M == 4) r = launch_multi<2, 4>(calls + i, n, prev_tiled);
         if (c.N == 4 && c.M == 8) r = launch_multi<4, 8>(calls + i, n, prev_tiled);

@@ -134,15 +134,20 @@ int sm_count();
 
 // Batched calls: a run of consecutive items with the same tile kernel, each of
 // them small (fewer than kMultiTilesPerSm full tiles per SM), goes to one
-// multi-tensor launch.  One launch per small tensor spends much of its time on
-// fixed costs (ring fill and drain, the ragged tail, the gap to the next launch).
-// A larger tensor keeps a launch of its own: the multi-tensor kernel holds the
-// current tensor's arguments in registers rather than in the constant bank, and
-// measured 4-7 % slower on 18944 x 3584 tensors.
-// A fwd + bwd step over a Qwen2.5-shaped layer set went from 1.90 to 1.57 ms
-// (0.5B-shaped, 2:4), 8.92 to 8.79 ms (1.5B-shaped, 4:8) and 24.32 to 24.23 ms
-// (7B-shaped, 2:4, where only the q, k, v, o tensors are small).
+// multi-tensor launch when it holds at least multi_min_run items.  One launch per
+// small tensor spends much of its time on fixed costs (ring fill and drain, the
+// ragged tail, the gap to the next launch).  A larger tensor keeps a launch of its
+// own: the multi-tensor kernels hold the current tensor's arguments in registers
+// rather than in the constant bank, and measured 4-7 % slower on 18944 x 3584
+// tensors.  That per-tile cost also decides the run lengths: the plain backward
+// gains from runs of 2 (the q, k, v, o tensors of a 7B-shaped layer), while the
+// forward and the backward fused with AdamW lost on those runs (7B-shaped 2:4 step,
+// forward 11.72 -> 11.80 ms, fused backward 28.8 -> 29.0 ms) and gain only over long
+// ones.  A fwd + bwd step over a Qwen2.5-shaped layer set went from 1.90 to 1.57 ms
+// (0.5B-shaped, 2:4: one launch per direction), 8.92 to 8.78 ms (1.5B-shaped, 4:8)
+// and 24.31 to 24.19 ms (7B-shaped, 2:4).
 constexpr int64_t kMultiTilesPerSm = 12;
+inline int multi_min_run(bool plain_backward) { return plain_backward ? 2 : 8; }
 inline bool multi_small(int64_t E, int64_t tile) { return E / tile < kMultiTilesPerSm * sm_count(); }
 
 }  // namespace roi

@@ -146,19 +146,23 @@ def test_more_items_than_one_launch_and_empty_items(roi):
 
 
 def test_batch_launch_counts(roi):
-    """Consecutive small tensors with the same tile kernel share one launch per
-    direction; a tensor that gives every SM at least 12 tiles (2:4: 12288 elements
-    a forward tile, 8192 a backward one) keeps a launch of its own, and splits the
-    runs around it.  Both forms give, bit for bit, what the single calls give."""
+    """Consecutive small tensors with the same tile kernel share one launch: runs of
+    at least 8 in the forward, of at least 2 in the plain backward.  A tensor that
+    gives every SM at least 12 tiles (2:4: 12288 elements a forward tile, 8192 a
+    backward one) keeps a launch of its own and splits the runs around it.  Every
+    form gives, bit for bit, what the single calls give."""
     import torch
     N, M, tau = 2, 4, 1.0
-    small = [(64, 3584), (16, 512), (37, 1000)]
+    small = [(64, 3584), (16, 512), (37, 1000), (8, 256), (100, 2048), (3, 64), (129, 520), (40, 4096)]
     ts = make_set(small, 3)
     flags = [(False, True, False)] * len(ts)
     run_batch(roi, ts, N, M, tau, flags)
     before = roi.roi_launch_count()
     run_batch(roi, ts, N, M, tau, flags)
     assert roi.roi_launch_count() - before == 2
+    before = roi.roi_launch_count()
+    run_batch(roi, ts[:3], N, M, tau, flags[:3])
+    assert roi.roi_launch_count() - before == 3 + 1
     sms = torch.cuda.get_device_properties(0).multi_processor_count
     big = (12 * sms * 12288 // 4096 + 8, 4096)
     ts = make_set([big] + small + [big, small[0]], 5)
@@ -166,7 +170,7 @@ def test_batch_launch_counts(roi):
     single = run_single(roi, ts, N, M, tau, flags)
     before = roi.roi_launch_count()
     batch = run_batch(roi, ts, N, M, tau, flags)
-    # per direction: big, the run of three small ones, big, one small
+    # per direction: big, the run of eight small ones, big, one small
     assert roi.roi_launch_count() - before == 2 * 4
     for a, b in zip(single, batch):
         assert_same(a, b)

@@ -87,7 +87,7 @@ def test_multi_tensor_launches_time_out_then_recover(roi):
     way, and the next batch on the context gives the first batch's bits."""
     import torch
     dev = torch.device("cuda")
-    shapes = [(256, 4096), (64, 1024), (300, 2048), (37, 1000)]
+    shapes = [(256, 4096), (64, 1024), (300, 2048), (37, 1000), (8, 512), (128, 896), (5, 64), (90, 3584)]
     ts = []
     for k, (rows, cols) in enumerate(shapes):
         W, phi, dWm = WL.make_inputs(rows, cols, "normal", 60 + k, device=dev)
