@@ -206,10 +206,11 @@ def test_work_queued_after_a_batch_sees_every_item(roi):
 
 def test_adamw_batch_equals_single_calls(roi):
     """roi_mask_bwd_adamw_batch: logits, moments, gradients and dW after the step equal
-    the single calls' bit for bit (2:4 and 4:8, mixed shapes and noise states)."""
+    the single calls' bit for bit (2:4 and 4:8, mixed shapes and noise states; nine
+    small tensors, so the batch runs as one multi-tensor launch)."""
     import torch
-    for N, M, tau in ((2, 4, 1.0), (4, 8, 0.5)):
-        shapes = [(r, c) for r, c in SHAPES if c % M == 0][:6]
+    for N, M, tau in ((2, 4, 1.0), (4, 8, 0.5), (4, 8, 1.0)):
+        shapes = [(r, c) for r, c in SHAPES if c % M == 0]
         ts = make_set(shapes, 70 + M)
         opt = roi.AdamW(1e-3, 0.9, 0.95, 1e-8, 0.05, 4)
         def state():
@@ -237,9 +238,11 @@ def test_adamw_batch_equals_single_calls(roi):
 
 
 def test_straight_through_batch_equals_single_calls(roi):
+    """roi_mask_{fwd,bwd}_st_batch against the single straight-through calls, bit for
+    bit (nine small tensors: one multi-tensor launch per direction)."""
     import torch
     for N, M, tau in ((2, 4, 1.0), (4, 8, 0.5)):
-        shapes = [(r, c) for r, c in SHAPES if c % M == 0][:6]
+        shapes = [(r, c) for r, c in SHAPES if c % M == 0]
         ts = make_set(shapes, 50 + M)
         res = []
         for k, t in enumerate(ts):
