@@ -307,3 +307,47 @@ def test_batch_mixes_counter_widths(roi, N, M):
         g, gr = a["dphi"].cpu().numpy(), r["dphi"].cpu().numpy()
         scale = np.abs(gr).reshape(-1, M).max(-1, keepdims=True).repeat(M, -1).reshape(gr.shape)
         assert np.all(np.abs(g - gr) <= 1e-6 * scale + 1e-30)
+
+
+def _expected_launches(shapes, tile, sms, min_run):
+    """Launches of one batched direction: a run of at least min_run consecutive
+    tensors with fewer than 12 full tiles per SM each takes one, any other tensor one."""
+    small = [r * c // tile < 12 * sms for r, c in shapes]
+    n = i = 0
+    while i < len(shapes):
+        j = i
+        while j < len(shapes) and small[j]:
+            j += 1
+        n += 1
+        i = j if j - i >= min_run else i + 1
+    return n
+
+
+@pytest.mark.parametrize("set_name,layers,N,M,tau", [("qwen2.5-0.5b", 4, 2, 4, 0.1), ("qwen2.5-1.5b", 2, 4, 8, 0.5)])
+def test_layer_set_batch_equals_single_calls(roi, set_name, layers, N, M, tau):
+    """Leading layers of a benchmark layer set at its own N:M and tau, step-keyed noise
+    as the benchmark draws it: the batched calls (the 0.5B-shaped set in one forward
+    and one backward launch; the 1.5B-shaped forward in one launch, its backward
+    sharing each layer's q, k, v, o) give every tensor's Wm, hard bits and logit
+    gradients bit for bit as the single calls do."""
+    import torch
+    dev = torch.device("cuda")
+    lset = WL.LAYER_SETS[set_name]
+    kind = WL.CONFIGS[set_name].logits
+    ts = []
+    for layer, p, rows, cols in lset.tensors():
+        if layer >= layers:
+            break
+        W, phi, dWm = WL.make_inputs(rows, cols, kind, WL.tensor_seed(layer, p), device=dev)
+        ts.append({"W": W, "phi": phi, "dWm": dWm, "st": (11, 5, 7 * layer + p, 1.0, 0), "rows": rows, "cols": cols})
+    flags = [(False, True, False)] * len(ts)
+    single = run_single(roi, ts, N, M, tau, flags)
+    before = roi.roi_launch_count()
+    batch = run_batch(roi, ts, N, M, tau, flags)
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    shapes = [(t["rows"], t["cols"]) for t in ts]
+    want = (_expected_launches(shapes, 12288 if M == 4 else 8192, sms, 8)
+            + _expected_launches(shapes, 8192 if M == 4 else 6144, sms, 2))
+    assert roi.roi_launch_count() - before == want
+    for a, b in zip(single, batch):
+        assert_same(a, b)
