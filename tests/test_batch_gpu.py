@@ -263,22 +263,25 @@ def test_straight_through_batch_equals_single_calls(roi):
 @pytest.mark.parametrize("N,M", [(2, 4), (4, 8)])
 def test_batch_mixes_counter_widths(roi, N, M):
     """Items whose noise counters all fit 32 bits (the kernels form them in 32-bit
-    arithmetic) chained with items whose flat indices pass 2^34 (64-bit counters), in
+    arithmetic) followed by items whose flat indices pass 2^34 (64-bit counters), in
     one batch: each equals its single call bit for bit (plain and fused with AdamW,
-    tau = 1), and a wide item matches the oracle."""
+    tau = 1), and a wide item matches the oracle.  Eight of each: the forward runs
+    both widths in one multi-tensor launch, the backwards one launch per width."""
     import torch
-    shapes = [(37, 1024), (64, 3584), (29, 1536), (5, 2048)]
+    shapes = [(37, 1024), (64, 3584), (29, 1536), (5, 2048)] * 4
     ts = make_set(shapes, 120 + M)
     for k, t in enumerate(ts):
-        if k % 2:  # rows from flat index 2^34 on
+        if k >= 8:  # rows from flat index 2^34 on
             seed, step, tid, lam, _ = t["st"]
             t["st"] = (seed, step, tid, lam, 2 ** 34 // t["cols"] + k)
     flags = [(True, True, True)] * len(ts)
     single = run_single(roi, ts, N, M, 1.0, flags)
+    before = roi.roi_launch_count()
     batch = run_batch(roi, ts, N, M, 1.0, flags)
+    assert roi.roi_launch_count() - before == 1 + 2
     for a, b in zip(single, batch):
         assert_same(a, b)
-    t, o = ts[1], batch[1]
+    t, o = ts[9], batch[9]
     seed, step, tid, lam, roff = t["st"]
     ph, Wb = t["phi"].cpu().numpy(), WL.bf16_bits(t["W"].cpu())
     ref = O.mask_fwd(ph, Wb, N, M, 1.0, seed, step, tensor_id=tid, lam=lam, row_offset=roff)
@@ -296,9 +299,11 @@ def test_batch_mixes_counter_widths(roi, N, M):
     one, bat = state(), state()
     for t, s_ in zip(ts, one):
         roi.roi_mask_bwd_adamw(s_["phi"], t["W"], t["st"], N, M, t["dWm"], 1.0, s_["m"], s_["v"], opt, s_["dphi"])
+    before = roi.roi_launch_count()
     roi.roi_mask_bwd_adamw_batch([(b["phi"], t["W"], t["st"], t["dWm"], b["m"], b["v"], b["dphi"], None)
                                   for t, b in zip(ts, bat)], N, M, 1.0, opt)
     roi.roi_device_status()
+    assert roi.roi_launch_count() - before == 2
     for a, b, r in zip(one, bat, single):
         for k in ("phi", "m", "v", "dphi"):
             assert torch.equal(a[k].view(torch.int32), b[k].view(torch.int32)), k
