@@ -106,8 +106,8 @@ roi_status roi_mask_fwd_ex(const float* logits, const roi_bf16* W, int N, int M,
  * its predecessor, so the work queued after the call sees every item done.  For
  * (2, 4), (4, 8) and (2, 8), runs of consecutive items small enough that each would
  * give an SM fewer than 12 tiles of work share one launch (runs of at least 8 items;
- * 2 for roi_mask_bwd_batch).  Items with rows == 0 are skipped.  `items` is host
- * memory, read during the call. */
+ * 2 for roi_mask_bwd_batch at tau >= 0.075).  Items with rows == 0 are skipped.
+ * `items` is host memory, read during the call. */
 typedef struct {
     const float* logits;  /* [rows, cols] */
     const roi_bf16* W;    /* [rows, cols] */

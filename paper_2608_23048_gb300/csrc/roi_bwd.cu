@@ -881,7 +881,7 @@ int launch_bwd_batch(const BwdCall* calls, int count) {
              bwd_kind(calls[i + n]) == kind && counters_narrow(calls[i + n].np, calls[i + n].E) == narrow &&
              multi_small(calls[i + n].E, tile))
         ++n;
-      if (n >= multi_min_run(kind == 0)) {
+      if (n >= multi_min_run(kind == 0 && c.tau >= kDeferBelowTau)) {
         int r = -1;
         if (c.N == 2 && c.M == 4) r = launch_multi<2, 4>(calls + i, n, prev_tiled);
         if (c.N == 4 && c.M == 8) r = launch_multi<4, 8>(calls + i, n, prev_tiled);

@@ -143,11 +143,15 @@ int sm_count();
 // gains from runs of 2 (the q, k, v, o tensors of a 7B-shaped layer), while the
 // forward and the backward fused with AdamW lost on those runs (7B-shaped 2:4 step,
 // forward 11.72 -> 11.80 ms, fused backward 28.8 -> 29.0 ms) and gain only over long
-// ones.  A fwd + bwd step over a Qwen2.5-shaped layer set went from 1.90 to 1.57 ms
-// (0.5B-shaped, 2:4: one launch per direction), 8.92 to 8.78 ms (1.5B-shaped, 4:8)
-// and 24.31 to 24.19 ms (7B-shaped, 2:4).
+// ones.  So does the plain backward where many groups go through the deferred
+// queue (tau below the deferral threshold): each drained group reads its tensor's
+// arguments from the parameter block by a per-lane index (tau = 0.05, 1.5B-shaped
+// 4:8 backward 7.01 -> 7.24 ms with short runs shared).  A fwd + bwd step over a
+// Qwen2.5-shaped layer set went from 1.90 to 1.57 ms (0.5B-shaped, 2:4: one launch
+// per direction), 8.92 to 8.78 ms (1.5B-shaped, 4:8) and 24.31 to 24.19 ms
+// (7B-shaped, 2:4).
 constexpr int64_t kMultiTilesPerSm = 12;
-inline int multi_min_run(bool plain_backward) { return plain_backward ? 2 : 8; }
+inline int multi_min_run(bool short_runs_pay) { return short_runs_pay ? 2 : 8; }
 inline bool multi_small(int64_t E, int64_t tile) { return E / tile < kMultiTilesPerSm * sm_count(); }
 
 }  // namespace roi
