@@ -505,8 +505,8 @@ CONFIG_SWEEP = [
     ("qwen2.5-0.5b", 2, 4, 1.0, 50),
     ("qwen2.5-0.5b", 2, 4, 0.1, 50),
     ("qwen2.5-1.5b", 4, 8, 0.5, 20),
-    ("qwen2.5-3b", 8, 16, 0.2, 5),
-    ("qwen2.5-3b", 16, 32, 0.2, 5),
+    ("qwen2.5-3b", 8, 16, 0.2, 10),
+    ("qwen2.5-3b", 16, 32, 0.2, 10),
 ]
 
 
